@@ -1,0 +1,16 @@
+"""Plain fp64 CPU oracle for the frame-quantized linear layer (FrameQuant).
+
+TEST INFRASTRUCTURE. Only tests/, __graft_entry__.smoke() and bench.py's cpu_baseline leg may
+import this package.  The product library (libframequant and its Python binding) never imports
+it and shares no code with it; the two meet only in the seeded input generators of workloads/.
+
+  frames   tight fusion frame construction and random rotation (Sec. 2.2, Appendix J, K)
+  quant    frame coefficients, 2-sigma clip, per-row RTN, de-noising gain (Sec. 3, Alg. 1, App. I)
+  pack     the packed 2-bit code layout declared by the library header
+  forward  analysis -> dequantized product -> synthesis (Sec. 3.2)
+  layer    one call that builds a whole quantized layer from a workload
+
+Parity status: every function is pinned by tests/test_oracle_*.py except wiener_gain's formula,
+which the paper does not print ("parity unpinned" for the formula itself; its gamma == 1
+special case and its shrinkage property are checked).
+"""
