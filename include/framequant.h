@@ -1,0 +1,133 @@
+/*
+ * libframequant: forward pass of a frame-quantized linear layer (FrameQuant, Adepu et al.,
+ * ICML 2024, arXiv 2403.06082) on one NVIDIA GB300 GPU (sm_103a).
+ *
+ * The layer (Sec. 3.2 "Inference Procedure"; Sec. 3, D_l = P_l^T Theta_l P_prev):
+ *
+ *     z = T_in x                          analysis onto the input tight fusion frame
+ *     u_i = gamma_i (s_i sum_j q_ij z_j + zero_i sum_j z_j)
+ *                                         2-bit frame coefficients C_hat_ij = s_i q_ij + zero_i
+ *     y = T_out^T u                       synthesis from the output frame
+ *
+ * for every token x (a row of X, M x d_in).  T_in (n_in x d_in) is the analysis operator of
+ * the input frame, P_prev^T in the paper; T_out^T (d_out x n_out) is the synthesis operator of
+ * the output frame, P_l in the paper.  n = k * rho is the number of frame coefficients; r = n/d
+ * is the redundancy.  gamma is the optional diagonal de-noising gain (Sec. 3.1 (b),
+ * Appendix I); pass NULL for none.
+ *
+ * Conventions for every entry point:
+ *   - All tensor pointers are DEVICE pointers owned by the caller, row-major, 16-byte aligned.
+ *     The library allocates no device memory; scratch space is the caller's workspace `ws`.
+ *   - Work is enqueued on `stream` (a cudaStream_t; NULL is the legacy default stream) and is
+ *     asynchronous: a return of FQ_OK means every check passed and every kernel launched.
+ *   - Arguments are validated on the host before anything is launched; on any error the call
+ *     returns a status and launches nothing.  No entry point aborts the process.
+ *   - Device-side findings (code values out of range, a bounded wait that ran out) set bit
+ *     (1 << status) of an int32 status word: fq_pack's `status` argument, or the head of
+ *     fq_linear_forward's `ws`.  fq_check reads it back.
+ *   - Outputs must not alias inputs; concurrent calls must not share a workspace.
+ */
+#ifndef FRAMEQUANT_H_
+#define FRAMEQUANT_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef struct CUstream_st* fq_stream_t; /* same type as cudaStream_t */
+
+typedef enum {
+  FQ_OK = 0,
+  FQ_ERR_INVALID_ARG = 1,   /* null pointer, non-positive or inconsistent dimension, bad mode */
+  FQ_ERR_ALIGNMENT = 2,     /* a pointer is not 16-byte aligned or a row pitch not 16 bytes */
+  FQ_ERR_UNSUPPORTED = 3,   /* valid request this build cannot run (device not sm_103, sizes) */
+  FQ_ERR_WORKSPACE = 4,     /* ws is NULL or smaller than fq_workspace_bytes() */
+  FQ_ERR_CUDA = 5,          /* a CUDA runtime or launch error */
+  FQ_ERR_TIMEOUT = 6,       /* device: a bounded wait inside a kernel ran out (fq_check) */
+  FQ_ERR_DEVICE_CHECK = 7   /* device: a code value above 3 was seen by fq_pack (fq_check) */
+} fq_status;
+
+/* Arithmetic modes of fq_linear_forward. */
+enum {
+  FQ_BF16 = 0,        /* x, T_in, T_out^T, y are bf16; z and u are rounded to bf16 between the
+                         three products; every product accumulates in fp32 (tensor cores) */
+  FQ_FP32_DEBUG = 1   /* x, T_in, T_out^T, y, z, u are fp32 throughout (CUDA cores) */
+};
+
+/* Packed 2-bit frame coefficients with their per-row scale and zero ("bias and scale values
+ * for each row", Appendix K).  Code q_ij in {0,1,2,3} dequantizes to s_i q_ij + zero_i.
+ *
+ * Layout of `words` (uint32; written by fq_pack): rows are grouped in tiles of 128 and
+ * columns in blocks of 64; n_out and n_in are padded up to those multiples with code 0.  The
+ * 64 codes of one (row, column block) are 4 consecutive words, and the 512 words of one
+ * (row tile, column block) pair are contiguous:
+ *     word index = ((row/128) * KB + col/64) * 512 + (row%128) * 4 + (col%64)/16,
+ *     KB = ceil(n_in/64);
+ * inside a word, column c = col%16 occupies bits [2*(c/2) + 16*(c%2), +2): even columns in the
+ * low half-word, odd columns in the high half-word, so that one mask of 0x00030003 shifted by
+ * 2*(c/2) isolates the adjacent pair (c, c+1).
+ */
+typedef struct {
+  const uint32_t* words;   /* device, fq_packed_words(n_out, n_in) words */
+  const uint16_t* scale;   /* device, IEEE fp16 bit patterns, n_out entries */
+  const uint16_t* zero;    /* device, IEEE fp16 bit patterns, n_out entries */
+  int32_t n_out;           /* rows of C_hat, = k_out * rho, a multiple of 16 */
+  int32_t n_in;            /* columns of C_hat, = k_in * rho, a multiple of 16 */
+} fq_packed;
+
+/* Number of uint32 words of the packed layout above: ceil(n_out/128)*128 * ceil(n_in/64)*64 / 16.
+ * Returns 0 when n_out or n_in is not positive. */
+size_t fq_packed_words(int n_out, int n_in);
+
+/* Pack 2-bit codes (Algorithm 1, step 5 "store D_hat"; layout above).
+ *   codes   device uint8, n_out x n_in row-major, values 0..3 (any alignment)
+ *   words   device uint32 output, fq_packed_words(n_out, n_in) words, 16-byte aligned;
+ *           padding positions are written with code 0
+ *   status  device int32 or NULL: when a code above 3 is met, bit (1 << FQ_ERR_DEVICE_CHECK)
+ *           is set there (the code's low 2 bits are packed); fq_pack never clears it
+ * Errors: FQ_ERR_INVALID_ARG (null codes/words, n_out or n_in <= 0), FQ_ERR_ALIGNMENT,
+ *         FQ_ERR_CUDA. */
+fq_status fq_pack(const uint8_t* codes, int n_out, int n_in, uint32_t* words, int32_t* status,
+                  fq_stream_t stream);
+
+/* Bytes of workspace fq_linear_forward needs for these sizes and mode (independent of the
+ * device).  Returns 0 for invalid sizes. */
+size_t fq_workspace_bytes(int M, int d_in, int n_in, int n_out, int d_out, int mode);
+
+/* Forward pass of the frame-quantized linear layer (Sec. 3.2; see the top of this file).
+ *   x        device, M x d_in tokens (bf16 or fp32 by mode)
+ *   T_in     device, n_in x d_in analysis operator of the input frame (P_prev^T)
+ *   C        host pointer to a descriptor of device data (codes, scale, zero); C->n_in and
+ *            C->n_out give the frame sizes
+ *   T_out_t  device, d_out x n_out synthesis operator of the output frame (T_out^T = P_l)
+ *   gamma    device fp32 [n_out] de-noising gain, or NULL for none
+ *   y        device, M x d_out output (bf16 or fp32 by mode)
+ *   ws       device workspace of at least fq_workspace_bytes(M, d_in, n_in, n_out, d_out,
+ *            mode) bytes, 256-byte aligned; its first 4 bytes hold the device status word,
+ *            which every call clears before its kernels run
+ *   mode     FQ_BF16 or FQ_FP32_DEBUG
+ * Requirements: M, d_in, d_out >= 1; d_in and d_out multiples of 8; C->n_in and C->n_out
+ * positive multiples of 16; all device pointers 16-byte aligned.
+ * Errors: FQ_ERR_INVALID_ARG, FQ_ERR_ALIGNMENT, FQ_ERR_WORKSPACE, FQ_ERR_UNSUPPORTED (the
+ * current device is not compute capability 10.3 in FQ_BF16 mode), FQ_ERR_CUDA. */
+fq_status fq_linear_forward(const void* x, int M, int d_in, const void* T_in,
+                            const fq_packed* C, const void* T_out_t, int d_out,
+                            const float* gamma, void* y, void* ws, size_t ws_bytes, int mode,
+                            fq_stream_t stream);
+
+/* Synchronize `stream` and read the device status word at `status_word` (the head of a
+ * forward workspace, or the `status` given to fq_pack).  Returns FQ_OK, FQ_ERR_TIMEOUT,
+ * FQ_ERR_DEVICE_CHECK, or FQ_ERR_CUDA if the synchronization itself failed. */
+fq_status fq_check(const void* status_word, fq_stream_t stream);
+
+/* Static string naming a status. */
+const char* fq_status_str(fq_status status);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* FRAMEQUANT_H_ */

@@ -161,7 +161,7 @@ def rotate_rows(T: np.ndarray, draws) -> np.ndarray:
     n, d = T.shape
     X = (T * draws.signs[None, :]).reshape(n, draws.a, draws.b)
     Y = np.matmul(np.matmul(Qa[None, :, :], X), Qb.T[None, :, :]).reshape(n, d)
-    return Y[:, draws.perm]
+    return np.ascontiguousarray(Y[:, draws.perm])
 
 
 def frame(k: int, rho: int, d: int, draws=None) -> np.ndarray:

@@ -1,0 +1,144 @@
+"""Python binding of libframequant: the forward pass of a frame-quantized linear layer
+(FrameQuant, arXiv 2403.06082) on a GB300 GPU.
+
+Argument marshalling only.  Every function here has the name and the arguments of a C entry
+point declared in include/framequant.h; tensors are torch tensors on the GPU (torch provides
+device memory and streams), passed to the library as raw pointers.  The computation itself
+runs in the library's CUDA kernels; there is no other implementation to fall back to, and a
+missing library is an error.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+from dataclasses import dataclass
+
+__all__ = [
+    "FQ_BF16", "FQ_FP32_DEBUG", "FrameQuantError", "Packed", "lib", "lib_path",
+    "fq_packed_words", "fq_pack", "fq_workspace_bytes", "fq_linear_forward", "fq_check",
+    "fq_status_str", "EXPORTED",
+]
+
+FQ_BF16 = 0
+FQ_FP32_DEBUG = 1
+STATUS = {0: "FQ_OK", 1: "FQ_ERR_INVALID_ARG", 2: "FQ_ERR_ALIGNMENT", 3: "FQ_ERR_UNSUPPORTED",
+          4: "FQ_ERR_WORKSPACE", 5: "FQ_ERR_CUDA", 6: "FQ_ERR_TIMEOUT",
+          7: "FQ_ERR_DEVICE_CHECK"}
+EXPORTED = ("fq_packed_words", "fq_pack", "fq_workspace_bytes", "fq_linear_forward",
+            "fq_check", "fq_status_str")
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+
+
+def lib_path() -> str:
+    return os.path.join(_HERE, "libframequant.so")
+
+
+class FrameQuantError(RuntimeError):
+    def __init__(self, status: int, where: str):
+        self.status = status
+        super().__init__(f"{where}: {STATUS.get(status, status)}")
+
+
+class _Packed(ctypes.Structure):
+    _fields_ = [("words", ctypes.c_void_p), ("scale", ctypes.c_void_p),
+                ("zero", ctypes.c_void_p), ("n_out", ctypes.c_int32), ("n_in", ctypes.c_int32)]
+
+
+_lib = None
+
+
+def lib() -> ctypes.CDLL:
+    """The loaded libframequant.so; raises if it has not been built."""
+    global _lib
+    if _lib is None:
+        path = lib_path()
+        if not os.path.exists(path):
+            raise ImportError(f"libframequant.so is missing ({path}); build it with "
+                              "`python -m paper_2403_06082_gb300._build`")
+        L = ctypes.CDLL(path)
+        L.fq_packed_words.restype = ctypes.c_size_t
+        L.fq_packed_words.argtypes = [ctypes.c_int, ctypes.c_int]
+        L.fq_pack.restype = ctypes.c_int
+        L.fq_pack.argtypes = [ctypes.c_void_p, ctypes.c_int, ctypes.c_int, ctypes.c_void_p,
+                              ctypes.c_void_p, ctypes.c_void_p]
+        L.fq_workspace_bytes.restype = ctypes.c_size_t
+        L.fq_workspace_bytes.argtypes = [ctypes.c_int] * 6
+        L.fq_linear_forward.restype = ctypes.c_int
+        L.fq_linear_forward.argtypes = [
+            ctypes.c_void_p, ctypes.c_int, ctypes.c_int, ctypes.c_void_p,
+            ctypes.POINTER(_Packed), ctypes.c_void_p, ctypes.c_int, ctypes.c_void_p,
+            ctypes.c_void_p, ctypes.c_void_p, ctypes.c_size_t, ctypes.c_int, ctypes.c_void_p]
+        L.fq_check.restype = ctypes.c_int
+        L.fq_check.argtypes = [ctypes.c_void_p, ctypes.c_void_p]
+        L.fq_status_str.restype = ctypes.c_char_p
+        L.fq_status_str.argtypes = [ctypes.c_int]
+        _lib = L
+    return _lib
+
+
+def _ptr(t) -> int | None:
+    """Raw device pointer of a dense row-major tensor (the C ABI takes no strides)."""
+    if t is None:
+        return None
+    if not t.is_contiguous():
+        raise ValueError("libframequant takes contiguous row-major tensors only")
+    return t.data_ptr()
+
+
+def _stream(stream) -> int | None:
+    if stream is None:
+        import torch
+        return torch.cuda.current_stream().cuda_stream
+    return stream if isinstance(stream, int) else stream.cuda_stream
+
+
+def _ok(st: int, where: str) -> None:
+    if st != 0:
+        raise FrameQuantError(st, where)
+
+
+@dataclass
+class Packed:
+    """Device tensors of packed codes (int32 view of the uint32 words), fp16 scale and zero."""
+    words: object
+    scale: object
+    zero: object
+    n_out: int
+    n_in: int
+
+    def _c(self) -> _Packed:
+        return _Packed(_ptr(self.words), _ptr(self.scale), _ptr(self.zero), self.n_out,
+                       self.n_in)
+
+
+def fq_packed_words(n_out: int, n_in: int) -> int:
+    return lib().fq_packed_words(n_out, n_in)
+
+
+def fq_pack(codes, n_out: int, n_in: int, words, status=None, stream=None) -> None:
+    _ok(lib().fq_pack(_ptr(codes), n_out, n_in, _ptr(words), _ptr(status), _stream(stream)),
+        "fq_pack")
+
+
+def fq_workspace_bytes(M: int, d_in: int, n_in: int, n_out: int, d_out: int,
+                       mode: int = FQ_BF16) -> int:
+    return lib().fq_workspace_bytes(M, d_in, n_in, n_out, d_out, mode)
+
+
+def fq_linear_forward(x, M: int, d_in: int, T_in, C: Packed, T_out_t, d_out: int, gamma, y,
+                      ws, ws_bytes: int, mode: int = FQ_BF16, stream=None) -> None:
+    pc = C._c()
+    _ok(lib().fq_linear_forward(_ptr(x), M, d_in, _ptr(T_in), ctypes.byref(pc), _ptr(T_out_t),
+                                d_out, _ptr(gamma), _ptr(y), _ptr(ws), ws_bytes, mode,
+                                _stream(stream)), "fq_linear_forward")
+
+
+def fq_check(status_word, stream=None) -> int:
+    """Synchronize and return the device status (0 = FQ_OK) at a workspace head or fq_pack
+    status word."""
+    return lib().fq_check(_ptr(status_word), _stream(stream))
+
+
+def fq_status_str(status: int) -> str:
+    return lib().fq_status_str(status).decode()

@@ -1,0 +1,106 @@
+// C ABI of libframequant (declared in include/framequant.h): argument checks on the host, then
+// dispatch to the bf16 tensor-core path (fq_tc.cu) or the fp32 debug path (fq_debug.cu).
+#include <cuda_runtime.h>
+
+#include "fq_internal.h"
+
+using namespace fq;
+
+namespace {
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+fq_status cuda_status(cudaError_t e) { return e == cudaSuccess ? FQ_OK : FQ_ERR_CUDA; }
+
+// Compute capability of the current device, or -1.
+int current_cc() {
+  int dev = 0, major = 0, minor = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return -1;
+  if (cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, dev) != cudaSuccess ||
+      cudaDeviceGetAttribute(&minor, cudaDevAttrComputeCapabilityMinor, dev) != cudaSuccess)
+    return -1;
+  return major * 10 + minor;
+}
+
+}  // namespace
+
+extern "C" {
+
+size_t fq_packed_words(int n_out, int n_in) {
+  if (n_out <= 0 || n_in <= 0) return 0;
+  return static_cast<size_t>(round_up(n_out, kRowTile)) * round_up(n_in, kColBlock) / 16;
+}
+
+fq_status fq_pack(const uint8_t* codes, int n_out, int n_in, uint32_t* words, int32_t* status,
+                  fq_stream_t stream) {
+  if (!codes || !words || n_out <= 0 || n_in <= 0) return FQ_ERR_INVALID_ARG;
+  if (!aligned16(words)) return FQ_ERR_ALIGNMENT;
+  return cuda_status(launch_pack(codes, n_out, n_in, words, status,
+                                 reinterpret_cast<cudaStream_t>(stream)));
+}
+
+size_t fq_workspace_bytes(int M, int d_in, int n_in, int n_out, int d_out, int mode) {
+  if (M <= 0 || d_in <= 0 || n_in <= 0 || n_out <= 0 || d_out <= 0) return 0;
+  if (mode == FQ_BF16) return tc_workspace_bytes(M, d_in, n_in, n_out, d_out);
+  if (mode == FQ_FP32_DEBUG) return debug_workspace_bytes(M, n_in, n_out);
+  return 0;
+}
+
+fq_status fq_linear_forward(const void* x, int M, int d_in, const void* T_in,
+                            const fq_packed* C, const void* T_out_t, int d_out,
+                            const float* gamma, void* y, void* ws, size_t ws_bytes, int mode,
+                            fq_stream_t stream) {
+  if (!x || !T_in || !C || !T_out_t || !y) return FQ_ERR_INVALID_ARG;
+  if (!C->words || !C->scale || !C->zero) return FQ_ERR_INVALID_ARG;
+  if (mode != FQ_BF16 && mode != FQ_FP32_DEBUG) return FQ_ERR_INVALID_ARG;
+  if (M <= 0 || d_in <= 0 || d_out <= 0 || C->n_in <= 0 || C->n_out <= 0)
+    return FQ_ERR_INVALID_ARG;
+  if (C->n_in % 16 || C->n_out % 16 || d_in % 8 || d_out % 8) return FQ_ERR_ALIGNMENT;
+  if (!aligned16(x) || !aligned16(T_in) || !aligned16(T_out_t) || !aligned16(y) ||
+      !aligned16(C->words) || !aligned16(C->scale) || !aligned16(C->zero) ||
+      (gamma && !aligned16(gamma)))
+    return FQ_ERR_ALIGNMENT;
+  if (!ws) return FQ_ERR_WORKSPACE;
+  if ((reinterpret_cast<uintptr_t>(ws) & 255u) != 0) return FQ_ERR_ALIGNMENT;
+  const size_t need = fq_workspace_bytes(M, d_in, C->n_in, C->n_out, d_out, mode);
+  if (ws_bytes < need) return FQ_ERR_WORKSPACE;
+  auto s = reinterpret_cast<cudaStream_t>(stream);
+  if (mode == FQ_FP32_DEBUG) {
+    if (cudaMemsetAsync(ws, 0, kWsHeader, s) != cudaSuccess) return FQ_ERR_CUDA;
+    return cuda_status(launch_debug_forward(
+        static_cast<const float*>(x), M, d_in, static_cast<const float*>(T_in), *C,
+        static_cast<const float*>(T_out_t), d_out, gamma, static_cast<float*>(y),
+        static_cast<char*>(ws), s));
+  }
+  if (current_cc() != 103) return FQ_ERR_UNSUPPORTED;
+  return launch_tc_forward(x, M, d_in, T_in, *C, T_out_t, d_out, gamma, y,
+                           static_cast<char*>(ws), ws_bytes, s);
+}
+
+fq_status fq_check(const void* status_word, fq_stream_t stream) {
+  if (!status_word) return FQ_ERR_INVALID_ARG;
+  auto s = reinterpret_cast<cudaStream_t>(stream);
+  int32_t v = 0;
+  if (cudaStreamSynchronize(s) != cudaSuccess) return FQ_ERR_CUDA;
+  if (cudaMemcpy(&v, status_word, sizeof(v), cudaMemcpyDeviceToHost) != cudaSuccess)
+    return FQ_ERR_CUDA;
+  if (v & (1 << FQ_ERR_TIMEOUT)) return FQ_ERR_TIMEOUT;
+  if (v & (1 << FQ_ERR_DEVICE_CHECK)) return FQ_ERR_DEVICE_CHECK;
+  return FQ_OK;
+}
+
+const char* fq_status_str(fq_status st) {
+  switch (st) {
+    case FQ_OK: return "FQ_OK";
+    case FQ_ERR_INVALID_ARG: return "FQ_ERR_INVALID_ARG";
+    case FQ_ERR_ALIGNMENT: return "FQ_ERR_ALIGNMENT";
+    case FQ_ERR_UNSUPPORTED: return "FQ_ERR_UNSUPPORTED";
+    case FQ_ERR_WORKSPACE: return "FQ_ERR_WORKSPACE";
+    case FQ_ERR_CUDA: return "FQ_ERR_CUDA";
+    case FQ_ERR_TIMEOUT: return "FQ_ERR_TIMEOUT";
+    case FQ_ERR_DEVICE_CHECK: return "FQ_ERR_DEVICE_CHECK";
+  }
+  return "FQ_UNKNOWN";
+}
+
+}  // extern "C"

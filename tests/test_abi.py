@@ -1,0 +1,96 @@
+"""The C-ABI library loads, exports every entry point include/framequant.h declares, and
+rejects bad arguments on the host with a status and without touching the GPU."""
+import ctypes
+import os
+import re
+
+import pytest
+
+import paper_2403_06082_gb300 as fq
+
+HEADER = os.path.join(os.path.dirname(os.path.dirname(os.path.abspath(__file__))), "include",
+                      "framequant.h")
+
+
+def _declared():
+    text = open(HEADER).read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return sorted(set(re.findall(r"\b(fq_[a-z_]+)\s*\(", text)))
+
+
+@pytest.fixture(scope="module")
+def L():
+    if not os.path.exists(fq.lib_path()):
+        import __graft_entry__
+        __graft_entry__.build()
+    return fq.lib()
+
+
+def test_exports_every_declared_symbol(L):
+    names = _declared()
+    assert set(names) == set(fq.EXPORTED)
+    for n in names:
+        assert hasattr(L, n), n
+
+
+def test_packed_words(L):
+    assert fq.fq_packed_words(288, 288) == 384 * 320 // 16
+    assert fq.fq_packed_words(128, 64) == 512
+    assert fq.fq_packed_words(0, 64) == 0
+    assert fq.fq_packed_words(12112, 4512) == 12160 * 4544 // 16
+
+
+def test_status_strings(L):
+    for k, v in fq.STATUS.items():
+        assert fq.fq_status_str(k) == v
+
+
+def test_workspace_bytes(L):
+    a = fq.fq_workspace_bytes(16, 4096, 4512, 4512, 4096, fq.FQ_BF16)
+    b = fq.fq_workspace_bytes(2048, 4096, 4512, 4512, 4096, fq.FQ_BF16)
+    assert 0 < a < b
+    assert fq.fq_workspace_bytes(16, 4096, 4512, 4512, 4096, fq.FQ_FP32_DEBUG) > 0
+    assert fq.fq_workspace_bytes(0, 4096, 4512, 4512, 4096, fq.FQ_BF16) == 0
+    assert fq.fq_workspace_bytes(16, 4096, 4512, 4512, 4096, 7) == 0
+    # z and u alone are M * (n_in + n_out) bf16
+    assert b >= 2048 * (4512 + 4512) * 2
+
+
+_P = fq._Packed
+
+
+def _call(L, x=0x1000, M=8, d_in=256, T_in=0x2000, C=None, T_out=0x3000, d_out=256, gamma=None,
+          y=0x4000, ws=0x10000, ws_bytes=1 << 30, mode=0):
+    C = C or _P(0x5000, 0x6000, 0x7000, 288, 288)
+    return L.fq_linear_forward(x, M, d_in, T_in, ctypes.byref(C), T_out, d_out, gamma, y, ws,
+                               ws_bytes, mode, None)
+
+
+def test_host_validation_without_gpu(L):
+    # every rejection happens before any device work (the pointers here are never touched)
+    assert _call(L, x=None) == 1
+    assert _call(L, y=None) == 1
+    assert _call(L, M=0) == 1
+    assert _call(L, d_in=-8) == 1
+    assert _call(L, mode=5) == 1
+    assert _call(L, C=_P(0, 0x6000, 0x7000, 288, 288)) == 1
+    assert _call(L, C=_P(0x5000, 0x6000, 0x7000, 0, 288)) == 1
+    assert _call(L, x=0x1002) == 2                      # misaligned pointer
+    assert _call(L, d_in=260) == 2                      # row pitch not 16 bytes
+    assert _call(L, C=_P(0x5000, 0x6000, 0x7000, 280, 288)) == 2   # n_out not a multiple of 16
+    assert _call(L, ws=None) == 4
+    assert _call(L, ws_bytes=1024) == 4
+    assert _call(L, ws=0x10010) == 2                    # workspace not 256-byte aligned
+    assert L.fq_pack(None, 4, 4, 0x1000, None, None) == 1
+    assert L.fq_pack(0x1000, 4, 4, 0x1004, None, None) == 2
+
+
+def test_valid_bf16_request_needs_sm103(L):
+    try:
+        import torch
+        if torch.cuda.is_available():
+            pytest.skip("a GPU is present")
+    except ImportError:
+        pass
+    # no CUDA device: the bf16 path refuses instead of falling back to anything
+    assert _call(L) == 3
