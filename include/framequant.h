@@ -118,6 +118,62 @@ fq_status fq_linear_forward(const void* x, int M, int d_in, const void* T_in,
                             const float* gamma, void* y, void* ws, size_t ws_bytes, int mode,
                             fq_stream_t stream);
 
+/* ------------------------------------------------------------------------------------------
+ * Offline preparation of a layer (not on the inference path).  These produce the inputs of
+ * fq_linear_forward on the device from a weight matrix W and the frame parameters.
+ * ---------------------------------------------------------------------------------------- */
+
+/* Random rotation R = Pi (Q_a kron Q_b) D of R^d, d = a * b (Sec. 2.2 remarks; Appendix K,
+ * P_l = R_l T_l).  The raw random numbers are the caller's (HOST pointers): Q_a and Q_b are the
+ * orthogonal factors of the QR decompositions of the a x a and b x b Gaussian matrices
+ * gauss_a and gauss_b, with columns signed so that R has a positive diagonal; D = diag(signs);
+ * (Pi v)[i] = v[perm[i]]. */
+typedef struct {
+  int32_t a;
+  int32_t b;
+  const double* gauss_a;   /* host, a x a row-major */
+  const double* gauss_b;   /* host, b x b row-major */
+  const int64_t* perm;     /* host, a permutation of 0 .. d-1 */
+  const double* signs;     /* host, d entries, each +1 or -1 */
+} fq_rotation;
+
+/* Workspace bytes of fq_frame_build (a = b = 0 without rotation). */
+size_t fq_frame_workspace_bytes(int k, int rho, int d, int a, int b);
+
+/* Analysis operator of the real (k, rho, d) tight fusion frame (Sec. 2.2 Definition "Tight
+ * Fusion Frames"; construction of Appendix J): spectral tetris gives F (rho/2 x d/2, unit
+ * columns, orthogonal rows); row j of F modulated by (w^(k_i n))_n, w = exp(2 pi i / k), spans
+ * subspace k_i of C^(d/2); each modulated vector is divided by sqrt(k) (Parseval, T^T T = I);
+ * the entrywise map x + iy -> [[x, -y], [y, x]] makes it real.  Rows are ordered (row j of F,
+ * k_i, real/imaginary part), columns (2c, 2c+1) are complex coordinate c.  With rot != NULL the
+ * operator is T R^T.  (1, d, d) gives the identity (the trivial frame).
+ *   T    device fp32 output, (k*rho) x d row-major
+ *   ws   device workspace of fq_frame_workspace_bytes(k, rho, d, a, b) bytes
+ * Synchronizes `stream` before returning (host staging buffers are released on return).
+ * Errors: FQ_ERR_INVALID_ARG (invalid triple: rho and d even, d >= 2 rho, and k at least the
+ * width of each row of F; bad rotation), FQ_ERR_WORKSPACE, FQ_ERR_CUDA. */
+fq_status fq_frame_build(int k, int rho, int d, const fq_rotation* rot, float* T, void* ws,
+                         size_t ws_bytes, fq_stream_t stream);
+
+/* Workspace bytes of fq_coefficients. */
+size_t fq_coefficients_workspace_bytes(int d_out, int n_in);
+
+/* Frame coefficients C = T_out W T_in^T (Sec. 3: D_l = P_l^T Theta_l P_prev), fp32 on CUDA
+ * cores.  W is d_out x d_in, T_in n_in x d_in, T_out n_out x d_out (analysis operators), C is
+ * n_out x n_in; all device fp32 row-major. */
+fq_status fq_coefficients(const float* W, int d_out, int d_in, const float* T_in, int n_in,
+                          const float* T_out, int n_out, float* C, void* ws, size_t ws_bytes,
+                          fq_stream_t stream);
+
+/* Per-row 2-bit round-to-nearest of C (n_out x n_in, device fp32): zero_i = fp16(min_j C_ij),
+ * scale_i = fp16((max_j C_ij - min_j C_ij) / 3) (1 when that is 0),
+ * q_ij = clamp(rint((C_ij - zero_i) / scale_i), 0, 3) with the fp16 values (Algorithm 1 with
+ * round-to-nearest in place of step 4).  gamma (nullable) receives the diagonal de-noising
+ * gain P_i / (P_i + scale_i^2 / 12), P_i the mean square of row i (Sec. 3.1 (b), Appendix I).
+ *   codes  device uint8 n_out x n_in;  scale, zero  device fp16 bits [n_out] */
+fq_status fq_quantize_rtn(const float* C, int n_out, int n_in, uint8_t* codes, uint16_t* scale,
+                          uint16_t* zero, float* gamma, fq_stream_t stream);
+
 /* Synchronize `stream` and read the device status word at `status_word` (the head of a
  * forward workspace, or the `status` given to fq_pack).  Returns FQ_OK, FQ_ERR_TIMEOUT,
  * FQ_ERR_DEVICE_CHECK, or FQ_ERR_CUDA if the synchronization itself failed. */

@@ -16,7 +16,8 @@ from dataclasses import dataclass
 __all__ = [
     "FQ_BF16", "FQ_FP32_DEBUG", "FrameQuantError", "Packed", "lib", "lib_path",
     "fq_packed_words", "fq_pack", "fq_workspace_bytes", "fq_linear_forward", "fq_check",
-    "fq_status_str", "EXPORTED",
+    "fq_status_str", "EXPORTED", "fq_frame_workspace_bytes", "fq_frame_build",
+    "fq_coefficients_workspace_bytes", "fq_coefficients", "fq_quantize_rtn",
 ]
 
 FQ_BF16 = 0
@@ -25,7 +26,8 @@ STATUS = {0: "FQ_OK", 1: "FQ_ERR_INVALID_ARG", 2: "FQ_ERR_ALIGNMENT", 3: "FQ_ERR
           4: "FQ_ERR_WORKSPACE", 5: "FQ_ERR_CUDA", 6: "FQ_ERR_TIMEOUT",
           7: "FQ_ERR_DEVICE_CHECK"}
 EXPORTED = ("fq_packed_words", "fq_pack", "fq_workspace_bytes", "fq_linear_forward",
-            "fq_check", "fq_status_str")
+            "fq_check", "fq_status_str", "fq_frame_workspace_bytes", "fq_frame_build",
+            "fq_coefficients_workspace_bytes", "fq_coefficients", "fq_quantize_rtn")
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
 
@@ -43,6 +45,12 @@ class FrameQuantError(RuntimeError):
 class _Packed(ctypes.Structure):
     _fields_ = [("words", ctypes.c_void_p), ("scale", ctypes.c_void_p),
                 ("zero", ctypes.c_void_p), ("n_out", ctypes.c_int32), ("n_in", ctypes.c_int32)]
+
+
+class _Rotation(ctypes.Structure):
+    _fields_ = [("a", ctypes.c_int32), ("b", ctypes.c_int32), ("gauss_a", ctypes.c_void_p),
+                ("gauss_b", ctypes.c_void_p), ("perm", ctypes.c_void_p),
+                ("signs", ctypes.c_void_p)]
 
 
 _lib = None
@@ -73,6 +81,23 @@ def lib() -> ctypes.CDLL:
         L.fq_check.argtypes = [ctypes.c_void_p, ctypes.c_void_p]
         L.fq_status_str.restype = ctypes.c_char_p
         L.fq_status_str.argtypes = [ctypes.c_int]
+        L.fq_frame_workspace_bytes.restype = ctypes.c_size_t
+        L.fq_frame_workspace_bytes.argtypes = [ctypes.c_int] * 5
+        L.fq_frame_build.restype = ctypes.c_int
+        L.fq_frame_build.argtypes = [ctypes.c_int, ctypes.c_int, ctypes.c_int,
+                                     ctypes.POINTER(_Rotation), ctypes.c_void_p, ctypes.c_void_p,
+                                     ctypes.c_size_t, ctypes.c_void_p]
+        L.fq_coefficients_workspace_bytes.restype = ctypes.c_size_t
+        L.fq_coefficients_workspace_bytes.argtypes = [ctypes.c_int, ctypes.c_int]
+        L.fq_coefficients.restype = ctypes.c_int
+        L.fq_coefficients.argtypes = [ctypes.c_void_p, ctypes.c_int, ctypes.c_int,
+                                      ctypes.c_void_p, ctypes.c_int, ctypes.c_void_p,
+                                      ctypes.c_int, ctypes.c_void_p, ctypes.c_void_p,
+                                      ctypes.c_size_t, ctypes.c_void_p]
+        L.fq_quantize_rtn.restype = ctypes.c_int
+        L.fq_quantize_rtn.argtypes = [ctypes.c_void_p, ctypes.c_int, ctypes.c_int,
+                                      ctypes.c_void_p, ctypes.c_void_p, ctypes.c_void_p,
+                                      ctypes.c_void_p, ctypes.c_void_p]
         _lib = L
     return _lib
 
@@ -142,3 +167,41 @@ def fq_check(status_word, stream=None) -> int:
 
 def fq_status_str(status: int) -> str:
     return lib().fq_status_str(status).decode()
+
+
+# ------------------------------------------------------------------ offline preparation
+def fq_frame_workspace_bytes(k: int, rho: int, d: int, a: int = 0, b: int = 0) -> int:
+    return lib().fq_frame_workspace_bytes(k, rho, d, a, b)
+
+
+def fq_frame_build(k: int, rho: int, d: int, rotation, T, ws, ws_bytes: int,
+                   stream=None) -> None:
+    """rotation: None or (a, b, gauss_a, gauss_b, perm, signs) with host numpy arrays
+    (float64, float64, int64, float64)."""
+    import numpy as np
+    rot = None
+    keep = None
+    if rotation is not None:
+        a, b, ga, gb, perm, signs = rotation
+        keep = [np.ascontiguousarray(ga, np.float64), np.ascontiguousarray(gb, np.float64),
+                np.ascontiguousarray(perm, np.int64), np.ascontiguousarray(signs, np.float64)]
+        rot = _Rotation(a, b, *(k_.ctypes.data for k_ in keep))
+    _ok(lib().fq_frame_build(k, rho, d, ctypes.byref(rot) if rot is not None else None,
+                             _ptr(T), _ptr(ws), ws_bytes, _stream(stream)), "fq_frame_build")
+    del keep
+
+
+def fq_coefficients_workspace_bytes(d_out: int, n_in: int) -> int:
+    return lib().fq_coefficients_workspace_bytes(d_out, n_in)
+
+
+def fq_coefficients(W, d_out: int, d_in: int, T_in, n_in: int, T_out, n_out: int, C, ws,
+                    ws_bytes: int, stream=None) -> None:
+    _ok(lib().fq_coefficients(_ptr(W), d_out, d_in, _ptr(T_in), n_in, _ptr(T_out), n_out,
+                              _ptr(C), _ptr(ws), ws_bytes, _stream(stream)), "fq_coefficients")
+
+
+def fq_quantize_rtn(C, n_out: int, n_in: int, codes, scale, zero, gamma=None,
+                    stream=None) -> None:
+    _ok(lib().fq_quantize_rtn(_ptr(C), n_out, n_in, _ptr(codes), _ptr(scale), _ptr(zero),
+                              _ptr(gamma), _stream(stream)), "fq_quantize_rtn")

@@ -73,6 +73,7 @@ fq_status fq_linear_forward(const void* x, int M, int d_in, const void* T_in,
         static_cast<char*>(ws), s));
   }
   if (current_cc() != 103) return FQ_ERR_UNSUPPORTED;
+  // the status word is cleared by the forward's first kernel, in stream order
   return launch_tc_forward(x, M, d_in, T_in, *C, T_out_t, d_out, gamma, y,
                            static_cast<char*>(ws), ws_bytes, s);
 }

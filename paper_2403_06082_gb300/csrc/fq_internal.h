@@ -18,6 +18,11 @@ inline int64_t round_up(int64_t a, int64_t b) { return ceil_div(a, b) * b; }
 // Workspace header: [0, 4) status word, [4, 256) reserved; counters follow.
 constexpr size_t kWsHeader = 256;
 
+// ---- fq_api.cu
+}  // namespace fq
+extern "C" size_t fq_packed_words(int n_out, int n_in);
+namespace fq {
+
 // ---- fq_pack.cu
 cudaError_t launch_pack(const uint8_t* codes, int n_out, int n_in, uint32_t* words,
                         int32_t* status, cudaStream_t s);

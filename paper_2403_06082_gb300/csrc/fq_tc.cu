@@ -5,7 +5,7 @@
 // with the weight-side operand A as the 128-row MMA operand and the tokens as the N operand
 // (N = BN in {16, ..., 256}), so one kernel serves decode (M <= 16) and prefill (M in the
 // thousands).  Phases (Sec. 3.2):
-//   analysis   A = T_in (n_in x d_in),  B = x,  out = z (bf16) and per-tile sums of z
+//   analysis   A = T_in (n_in x d_in),  B = x,  out = z (bf16)
 //   core       A = 2-bit codes of C_hat (n_out x n_in) decoded to bf16 in shared memory,
 //              B = z, out = u = gamma * (s * acc + zero * sum(z))   (bf16)
 //   synthesis  A = T_out^T (d_out x n_out), B = u, out = y (bf16)
@@ -14,18 +14,28 @@
 //              warps 2-5 epilogue (thread = accumulator row), warps 6-9 code decoders (core).
 // Operand tiles are 64 bf16 wide in K (one 128-byte swizzle atom) and staged through a ring
 // of shared-memory stages guarded by mbarriers; accumulators are double-buffered in TMEM so
-// the epilogue of one work unit overlaps the MMAs of the next.  Work units are (row tile,
-// token tile, K split); when a tile's K range is split, fp32 partials go to the workspace and
-// the last CTA to finish the tile (an atomic ticket, no spinning) reduces them in a fixed
-// order and applies the epilogue.  Consecutive phases are chained with programmatic
-// dependent launch: a dependent kernel starts on SMs as they free up, prefetches its weight
-// operand into L2, and waits (griddepcontrol.wait) before it touches the previous phase's
-// output.
+// the epilogue of one tile overlaps the MMAs of the next.
+//
+// Small batches (BN <= 64) leave too few row tiles to occupy the GPU, so the K range of a
+// tile is split over the S CTAs of a thread-block cluster.  Each CTA writes its fp32 partial
+// tile to its own shared memory, the CTAs signal one another through cluster-scope mbarrier
+// arrivals, and each reduces a slice of the tile's rows by reading all S partials through
+// distributed shared memory in a fixed order (deterministic, no global partials, no atomics).
+// In the core phase the decoder warps also sum the bf16 z values of every B tile they see, so
+// each split carries its own share of sum(z) from exactly the values its MMAs consumed; with
+// larger batches (one split) the analysis epilogue produces per-tile sums of z instead.
+//
+// The three phases are chained with programmatic dependent launch (the analysis kernel too,
+// so consecutive layers chain as well): a kernel's CTAs start on SMs as they free up, load
+// weight tiles that do not depend on the previous kernel, and wait (griddepcontrol.wait)
+// before reading activations or writing anything the previous kernel may still read.
 #include <cuda.h>
 #include <cudaTypedefs.h>
 
 #include <algorithm>
+#include <map>
 #include <mutex>
+#include <utility>
 
 #include "fq_device.cuh"
 #include "fq_internal.h"
@@ -39,51 +49,55 @@ constexpr int kBM = 128;                    // MMA M (rows of A per tile)
 constexpr int kBK = 64;                     // K per stage (one 128-byte swizzle atom of bf16)
 constexpr int kATileBytes = kBM * kBK * 2;  // 16 KiB
 constexpr int kCodeBytes = kBM * kBK / 4;   // 2 KiB of packed codes per stage
-constexpr int kMaxSplits = 16;
-constexpr int kMaxSMs = 160;                // upper bound on SMs, for the workspace bound
-constexpr int kMaxCounterTiles = 1024;
+constexpr int kMaxSplits = 8;               // portable cluster size
 constexpr int kSmemBudget = 200 * 1024;
+constexpr int64_t kL2PrefetchBudget = 64ll << 20;   // bytes of later-phase weights warmed in L2
+constexpr int kEpi = 128;                   // epilogue threads
+constexpr int kChunk = 16;                  // accumulator columns per TMEM load
 
 struct PhaseArgs {
   int R, K, M;
-  int RT, TT, S, KB, kb_per_split, units;
+  int RT, TT, S, KB, kb_per_split, tiles;
   const uint32_t* words;     // core: packed codes
   __nv_bfloat16* out;        // [M][R]
-  float* partial;            // [S][M][R] when S > 1
-  unsigned* counters;        // [RT * TT] tickets when S > 1
-  float* zsum_part;          // analysis writes [RT][M]; core reads [zsum_tiles][M]
+  float* zsum_part;          // BN >= 128: analysis writes [RT][M] sums of z; core reads them
   int zsum_tiles;
   const __half* scale;
   const __half* zero;
   const float* gamma;
   int32_t* status;
+  const char* pf_base[2];    // analysis: later phases' weights to warm in L2 (or null)
+  int64_t pf_bytes[2];
 };
 
-template <int BN>
-struct Cfg {
+template <int PHASE, int BN>
+struct Layout {
+  static constexpr bool kCodes = PHASE == kCore;
+  static constexpr bool kSplit = BN <= 64;              // cluster split-K allowed
+  static constexpr bool kDecoderZsum = kCodes && BN <= 64;
   static constexpr int kBTileBytes = BN * kBK * 2;
-  static constexpr int kStageBytes = kATileBytes + kBTileBytes + kCodeBytes;
-  static constexpr int kStages = std::min(12, kSmemBudget / kStageBytes);
-  static constexpr int kChunk = 16;                      // accumulator columns per TMEM load
+  static constexpr int kCodesStage = kCodes ? kCodeBytes : 0;
+  static constexpr int kStageBytes = kATileBytes + kBTileBytes + kCodesStage;
+  static constexpr int kRedBytes = kSplit ? BN * kBM * 4 : 0;
+  static constexpr int kStages = std::min(12, (kSmemBudget - kRedBytes) / kStageBytes);
   static constexpr uint32_t kTmemCols = 2 * BN < 32 ? 32 : 2 * BN;
+  // byte offsets from the 1024-aligned base
+  static constexpr int oA = 0;
+  static constexpr int oB = oA + kStages * kATileBytes;
+  static constexpr int oCodes = oB + kStages * kBTileBytes;
+  static constexpr int oRed = oCodes + kStages * kCodesStage;
+  static constexpr int oBar = oRed + kRedBytes;
+  static constexpr int kNumBars = 4 * kStages + 2 + 2 + 1 + 2 + 2 + 2;
+  static constexpr int oMisc = oBar + kNumBars * 8;
+  static constexpr int oRedSmall = oMisc + 16;                      // [4][kChunk] floats
+  static constexpr int oZsum = oRedSmall + 4 * kChunk * 4;          // [2][BN] floats
+  static constexpr int kBytes = oZsum + 2 * BN * 4 + 1024;          // + alignment slack
+  static_assert(kBTileBytes % 1024 == 0, "B tiles must keep 1024-byte alignment");
+  static_assert(kBytes <= 227 * 1024, "shared memory");
 };
 
 template <int PHASE>
 constexpr int threads_for() { return PHASE == kCore ? 320 : 192; }
-
-template <int BN>
-constexpr int smem_bytes_for() {
-  // stages + barriers/bookkeeping + 1 KiB alignment slack
-  return Cfg<BN>::kStages * Cfg<BN>::kStageBytes + 2048 + BN * 4 + 1024;
-}
-
-__device__ __forceinline__ void unit_coords(const PhaseArgs& p, int u, int& rt, int& tt,
-                                            int& ks) {
-  rt = u % p.RT;
-  const int rest = u / p.RT;
-  tt = rest % p.TT;
-  ks = rest / p.TT;
-}
 
 // Decode 64 2-bit codes (4 words, layout of framequant.h) into 64 exact bf16 values and store
 // them as one 128-byte row of a K-major tile with the 128-byte swizzle (16-byte chunk c of row
@@ -113,6 +127,15 @@ __device__ __forceinline__ void decode_row(const uint4 w4, uint8_t* tile, int r)
   }
 }
 
+__device__ __forceinline__ float sum_bf16x8(const uint4 v) {
+  const uint32_t w[4] = {v.x, v.y, v.z, v.w};
+  float s = 0.f;
+#pragma unroll
+  for (int i = 0; i < 4; ++i)
+    s += __uint_as_float(w[i] << 16) + __uint_as_float(w[i] & 0xffff0000u);
+  return s;
+}
+
 __device__ __forceinline__ bool bar_red_or(uint32_t id, uint32_t n, bool v) {
   uint32_t out;
   asm volatile(
@@ -130,123 +153,178 @@ template <int PHASE, int BN>
 __global__ void __launch_bounds__(threads_for<PHASE>(), 1)
     tc_phase_kernel(const __grid_constant__ CUtensorMap tmA,
                     const __grid_constant__ CUtensorMap tmB, const PhaseArgs p) {
-  using C = Cfg<BN>;
-  constexpr int S_ = C::kStages;
-  constexpr bool kCodes = PHASE == kCore;
+  using Lo = Layout<PHASE, BN>;
+  constexpr int S_ = Lo::kStages;
+  constexpr bool kCodes = Lo::kCodes;
+  constexpr int kBTile = Lo::kBTileBytes;
 
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>(
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
-  uint8_t* sA = smem;
-  uint8_t* sB = sA + S_ * kATileBytes;
-  uint8_t* sCodes = sB + S_ * C::kBTileBytes;
-  uint64_t* full = reinterpret_cast<uint64_t*>(sCodes + S_ * kCodeBytes);
-  uint64_t* empty = full + S_;
-  uint64_t* aready = empty + S_;
-  uint64_t* tfull = aready + S_;
-  uint64_t* tempty = tfull + 2;
+  uint8_t* sA = smem + Lo::oA;
+  uint8_t* sB = smem + Lo::oB;
+  uint8_t* sCodes = smem + Lo::oCodes;
+  float* red_buf = reinterpret_cast<float*>(smem + Lo::oRed);      // [BN][128] partial tile
+  uint64_t* full = reinterpret_cast<uint64_t*>(smem + Lo::oBar);   // A (+B) landed / B landed
+  uint64_t* empty = full + S_;      // stage consumed by the MMAs
+  uint64_t* aready = empty + S_;    // decoded A tile written (core)
+  uint64_t* cfull = aready + S_;    // codes landed (core)
+  uint64_t* tfull = cfull + S_;     // accumulator ready
+  uint64_t* tempty = tfull + 2;     // accumulator drained
   uint64_t* mma_done = tempty + 2;
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(mma_done + 1);
+  uint64_t* rdy = mma_done + 1;     // cluster: partials of every CTA written
+  uint64_t* cons = rdy + 1;         // cluster: every CTA done reading partials
+  uint64_t* zready = cons + 1;      // core: decoders' sum(z) for the buffer written
+  uint64_t* zfree = zready + 2;     // core: epilogue done reading it
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + Lo::oMisc);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
-  int* ticket = reinterpret_cast<int*>(tmem_slot + 2);
-  float* red = reinterpret_cast<float*>(tmem_slot + 4);       // [4][kChunk] cross-warp sums
-  float* zsum_s = red + 4 * C::kChunk;                        // [BN] sum of z per token
+  float* red = reinterpret_cast<float*>(smem + Lo::oRedSmall);     // [4][kChunk]
+  float* zsum_s = reinterpret_cast<float*>(smem + Lo::oZsum);      // [2][BN]
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const bool clustered = p.S > 1;
+  uint32_t rank = 0, cid = blockIdx.x, ncl = gridDim.x;
+  if (clustered) {
+    rank = cluster_ctarank();
+    cid = cluster_id_x();
+    ncl = cluster_count_x();
+  }
+  const int ks = static_cast<int>(rank);
+  const int k0 = ks * p.kb_per_split;
+  const int k1 = min(p.KB, k0 + p.kb_per_split);
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < S_; ++s) {
       mbar_init(&full[s], 1);
       mbar_init(&empty[s], 1);
       mbar_init(&aready[s], kBM);
+      mbar_init(&cfull[s], 1);
     }
     for (int b = 0; b < 2; ++b) {
       mbar_init(&tfull[b], 1);
-      mbar_init(&tempty[b], kBM);
+      mbar_init(&tempty[b], kEpi);
+      mbar_init(&zready[b], kBM);
+      mbar_init(&zfree[b], kEpi);
     }
     mbar_init(mma_done, 1);
+    mbar_init(rdy, static_cast<uint32_t>(p.S));
+    mbar_init(cons, static_cast<uint32_t>(p.S));
     *abort_flag = 0;
     fence_barrier_init();
     if (!kCodes) prefetch_tmap(&tmA);
     prefetch_tmap(&tmB);
   }
-  if (warp == 1) tmem_alloc(tmem_slot, C::kTmemCols);
+  if (warp == 1) tmem_alloc(tmem_slot, Lo::kTmemCols);
   tc_fence_before_sync();
   __syncthreads();
+  if (clustered) cluster_sync();   // every CTA's barriers exist before any remote arrival
   tc_fence_after_sync();
   const uint32_t tmem_base = *tmem_slot;
 
-  // Let the next phase's CTAs launch as soon as SMs free up; they wait for this grid's
+  // Let the next kernel's CTAs launch as soon as SMs free up; they wait for this grid's
   // completion (griddepcontrol.wait) before reading what it writes.
   pdl_launch_dependents();
-
-  const int first_unit = blockIdx.x;
-  const int unit_step = gridDim.x;
 
   if (warp == 0) {
     // ---------------------------------------------------------------- TMA producer
     if (lane == 0) {
       const uint64_t pol_w = policy_evict_first();   // weights: streamed once
       const uint64_t pol_x = policy_evict_last();    // activations: re-read by other tiles
-      if (PHASE != kAnalysis) {
-        // Warm L2 with this CTA's first weight tiles while the previous phase finishes.
-        if (first_unit < p.units) {
-          int rt, tt, ks;
-          unit_coords(p, first_unit, rt, tt, ks);
-          const int k0 = ks * p.kb_per_split, k1 = min(p.KB, k0 + p.kb_per_split);
-          for (int kb = k0; kb < k1; ++kb) {
-            if (kCodes) {
-              const uint32_t* src = p.words + (static_cast<int64_t>(rt) * p.KB + kb) * 512;
-              asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(src),
-                           "r"(kCodeBytes)
-                           : "memory");
-            } else {
-              asm volatile(
-                  "cp.async.bulk.prefetch.tensor.2d.L2.global.tile [%0, {%1, %2}];" ::"l"(
-                      reinterpret_cast<uint64_t>(&tmA)),
-                  "r"(kb * kBK), "r"(rt * kBM)
-                  : "memory");
-            }
+      // Weight tiles of the first tile do not depend on the previous kernel: issue up to a
+      // full ring of them before waiting for it, and warm L2 with the rest.
+      int pre = 0;
+      if (static_cast<int>(cid) < p.tiles) {
+        const int rt = static_cast<int>(cid) % p.RT;
+        pre = min(S_, k1 - k0);
+        for (int i = 0; i < pre; ++i) {
+          const int kb = k0 + i;
+          if (kCodes) {
+            mbar_arrive_expect_tx(&cfull[i], kCodeBytes);
+            bulk_load(sCodes + i * kCodeBytes,
+                      p.words + (static_cast<int64_t>(rt) * p.KB + kb) * 512, kCodeBytes,
+                      &cfull[i], pol_w);
+          } else {
+            mbar_arrive_expect_tx(&full[i], kATileBytes + kBTile);
+            tma_load_2d(sA + i * kATileBytes, &tmA, &full[i], kb * kBK, rt * kBM, pol_w);
           }
         }
-        pdl_wait();
+        for (int kb = k0 + pre; kb < k1; ++kb) {
+          if (kCodes) {
+            const uint32_t* src = p.words + (static_cast<int64_t>(rt) * p.KB + kb) * 512;
+            asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(src),
+                         "r"(kCodeBytes)
+                         : "memory");
+          } else {
+            asm volatile(
+                "cp.async.bulk.prefetch.tensor.2d.L2.global.tile [%0, {%1, %2}];" ::"l"(
+                    reinterpret_cast<uint64_t>(&tmA)),
+                "r"(kb * kBK), "r"(rt * kBM)
+                : "memory");
+          }
+        }
       }
+      pdl_wait();   // the previous kernel is complete and its writes are visible
+      if (PHASE == kAnalysis && blockIdx.x == 0) *p.status = 0;   // new call: clear status
       int stage = 0;
       uint32_t phase = 0;
+      int it = 0;
       uint32_t issued_parity[S_];
       bool issued[S_];
 #pragma unroll
       for (int s = 0; s < S_; ++s) issued[s] = false, issued_parity[s] = 0;
-      for (int u = first_unit; u < p.units && !*abort_flag; u += unit_step) {
-        int rt, tt, ks;
-        unit_coords(p, u, rt, tt, ks);
-        const int k0 = ks * p.kb_per_split, k1 = min(p.KB, k0 + p.kb_per_split);
-        for (int kb = k0; kb < k1; ++kb) {
-          if (!mbar_wait(&empty[stage], phase ^ 1)) {
-            report(p.status, FQ_ERR_TIMEOUT);
-            *abort_flag = 1;
-            break;
+      for (int tile = static_cast<int>(cid); tile < p.tiles && !*abort_flag;
+           tile += static_cast<int>(ncl)) {
+        const int rt = tile % p.RT, tt = tile / p.RT;
+        for (int kb = k0; kb < k1; ++kb, ++it) {
+          if (it >= pre) {
+            if (!mbar_wait(&empty[stage], phase ^ 1, abort_flag)) {
+              report(p.status, FQ_ERR_TIMEOUT);
+              *abort_flag = 1;
+              break;
+            }
+            if (kCodes) {
+              mbar_arrive_expect_tx(&cfull[stage], kCodeBytes);
+              bulk_load(sCodes + stage * kCodeBytes,
+                        p.words + (static_cast<int64_t>(rt) * p.KB + kb) * 512, kCodeBytes,
+                        &cfull[stage], pol_w);
+            } else {
+              mbar_arrive_expect_tx(&full[stage], kATileBytes + kBTile);
+              tma_load_2d(sA + stage * kATileBytes, &tmA, &full[stage], kb * kBK, rt * kBM,
+                          pol_w);
+            }
           }
-          if (kCodes) {
-            mbar_arrive_expect_tx(&full[stage], kCodeBytes + C::kBTileBytes);
-            bulk_load(sCodes + stage * kCodeBytes,
-                      p.words + (static_cast<int64_t>(rt) * p.KB + kb) * 512, kCodeBytes,
-                      &full[stage], pol_w);
-          } else {
-            mbar_arrive_expect_tx(&full[stage], kATileBytes + C::kBTileBytes);
-            tma_load_2d(sA + stage * kATileBytes, &tmA, &full[stage], kb * kBK, rt * kBM,
-                        pol_w);
-          }
-          tma_load_2d(sB + stage * C::kBTileBytes, &tmB, &full[stage], kb * kBK, tt * BN,
-                      pol_x);
+          if (kCodes) mbar_arrive_expect_tx(&full[stage], kBTile);
+          tma_load_2d(sB + stage * kBTile, &tmB, &full[stage], kb * kBK, tt * BN, pol_x);
           issued[stage] = true;
           issued_parity[stage] = phase;
           if (++stage == S_) stage = 0, phase ^= 1;
+          if (PHASE == kAnalysis && it + 1 == pre) {
+            // this CTA's share of the later phases' weights, into L2 while T_in streams
+            for (int r = 0; r < 2; ++r) {
+              if (!p.pf_base[r]) continue;
+              const int64_t share =
+                  ((p.pf_bytes[r] + gridDim.x - 1) / gridDim.x + 255) & ~255LL;
+              const int64_t beg = static_cast<int64_t>(blockIdx.x) * share;
+              const int64_t end = p.pf_bytes[r] < beg + share ? p.pf_bytes[r] : beg + share;
+              for (int64_t off = beg; off < end; off += 32768) {
+                const uint32_t len =
+                    static_cast<uint32_t>(end - off < 32768 ? end - off : 32768);
+                asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(
+                                 p.pf_base[r] + off),
+                             "r"(len)
+                             : "memory");
+              }
+            }
+          }
         }
       }
       // Never leave with copies in flight: wait (bounded) for the last round of each stage.
-      for (int s = 0; s < S_; ++s)
-        if (issued[s] && !mbar_wait(&full[s], issued_parity[s])) report(p.status, FQ_ERR_TIMEOUT);
+      for (int s = 0; s < S_; ++s) {
+        if (!issued[s]) continue;
+        if (!mbar_wait(&full[s], issued_parity[s], nullptr) ||
+            (kCodes && !mbar_wait(&cfull[s], issued_parity[s], nullptr)))
+          report(p.status, FQ_ERR_TIMEOUT);
+      }
     }
   } else if (warp == 1) {
     // ---------------------------------------------------------------- MMA issuer
@@ -257,11 +335,9 @@ __global__ void __launch_bounds__(threads_for<PHASE>(), 1)
       int buf = 0;
       uint32_t acc_phase = 0;
       bool issued_any = false;
-      for (int u = first_unit; u < p.units && !*abort_flag; u += unit_step) {
-        int rt, tt, ks;
-        unit_coords(p, u, rt, tt, ks);
-        const int k0 = ks * p.kb_per_split, k1 = min(p.KB, k0 + p.kb_per_split);
-        if (!mbar_wait(&tempty[buf], acc_phase ^ 1)) {
+      for (int tile = static_cast<int>(cid); tile < p.tiles && !*abort_flag;
+           tile += static_cast<int>(ncl)) {
+        if (!mbar_wait(&tempty[buf], acc_phase ^ 1, abort_flag)) {
           report(p.status, FQ_ERR_TIMEOUT);
           *abort_flag = 1;
           break;
@@ -270,11 +346,12 @@ __global__ void __launch_bounds__(threads_for<PHASE>(), 1)
         const uint32_t d_tmem = tmem_base + static_cast<uint32_t>(buf * BN);
         bool ok = true;
         for (int kb = k0; kb < k1; ++kb) {
-          ok = mbar_wait(&full[stage], phase) && (!kCodes || mbar_wait(&aready[stage], phase));
+          ok = mbar_wait(&full[stage], phase, abort_flag) &&
+               (!kCodes || mbar_wait(&aready[stage], phase, abort_flag));
           if (!ok) break;
           tc_fence_after_sync();
           const uint64_t adesc = umma_desc_sw128(smem_u32(sA + stage * kATileBytes));
-          const uint64_t bdesc = umma_desc_sw128(smem_u32(sB + stage * C::kBTileBytes));
+          const uint64_t bdesc = umma_desc_sw128(smem_u32(sB + stage * kBTile));
 #pragma unroll
           for (int k = 0; k < kBK / 16; ++k) {
             // advance 16 bf16 = 32 bytes along K inside the swizzle atom
@@ -296,7 +373,7 @@ __global__ void __launch_bounds__(threads_for<PHASE>(), 1)
       // Drain: every MMA issued has completed before the TMEM is released.
       if (issued_any) {
         umma_commit(mma_done);
-        if (!mbar_wait(mma_done, 0)) report(p.status, FQ_ERR_TIMEOUT);
+        if (!mbar_wait(mma_done, 0, nullptr)) report(p.status, FQ_ERR_TIMEOUT);
       }
     }
   } else if (warp < 6) {
@@ -305,156 +382,182 @@ __global__ void __launch_bounds__(threads_for<PHASE>(), 1)
     const int r_in_tile = quarter * 32 + lane;
     const int et = threadIdx.x - 64;              // 0..127 within the epilogue group
     const int ew = warp - 2;
-    if (PHASE != kAnalysis) pdl_wait();
+    pdl_wait();
     int buf = 0;
     uint32_t acc_phase = 0;
-    for (int u = first_unit; u < p.units; u += unit_step) {
-      int rt, tt, ks;
-      unit_coords(p, u, rt, tt, ks);
+    int j = 0;                                    // tiles finished by this CTA
+    // the slice of each tile's rows this CTA reduces when the tile's K range is split
+    const int rows_per = (kBM + p.S - 1) / p.S;
+    const int r0 = ks * rows_per;
+    const int rcnt = max(0, min(kBM - r0, rows_per));
+    const uint32_t red_addr = smem_u32(red_buf);
+    for (int tile = static_cast<int>(cid); tile < p.tiles; tile += static_cast<int>(ncl), ++j) {
+      const int rt = tile % p.RT, tt = tile / p.RT;
       const int row = rt * kBM + r_in_tile;
       const int t0 = tt * BN;
       const bool row_ok = row < p.R;
-      float s_i = 0.f, z_i = 0.f, g_i = 1.f;
+      float s_i = 0.f, z_i = 0.f;
       if (PHASE == kCore && row_ok) {
         s_i = __half2float(p.scale[row]);
         z_i = __half2float(p.zero[row]);
-        if (p.gamma) g_i = p.gamma[row];
       }
-      const bool fail = !mbar_wait(&tfull[buf], acc_phase);
+      if (PHASE == kCore && !Lo::kDecoderZsum) {
+        // sum_j z[t][j] for the tile's tokens, from the analysis phase's per-tile sums
+        named_barrier_sync(1, kEpi);
+        for (int q = et; q < BN; q += kEpi) {
+          const int t = t0 + q;
+          float s = 0.f;
+          if (t < p.M)
+            for (int g = 0; g < p.zsum_tiles; ++g)
+              s += ldcg_f32(p.zsum_part + static_cast<int64_t>(g) * p.M + t);
+          zsum_s[buf * BN + q] = s;
+        }
+        named_barrier_sync(1, kEpi);
+      }
+      bool fail = !mbar_wait(&tfull[buf], acc_phase, abort_flag);
+      if (Lo::kDecoderZsum && !fail) fail = !mbar_wait(&zready[buf], acc_phase, abort_flag);
+      if (clustered && j > 0 && !fail) fail = !mbar_wait_cluster(cons, (j - 1) & 1);
       if (fail) report(p.status, FQ_ERR_TIMEOUT);
-      if (bar_red_or(1, 128, fail || *abort_flag)) {
-        if (threadIdx.x == 64) *abort_flag = 1;
+      if (bar_red_or(1, kEpi, fail || *abort_flag)) {
+        if (et == 0) *abort_flag = 1;
         break;
       }
       tc_fence_after_sync();
       const uint32_t t_row = tmem_base + (static_cast<uint32_t>(quarter * 32) << 16) +
                              static_cast<uint32_t>(buf * BN);
+      const float* zs = zsum_s + buf * BN;
 
-      // Final value of this thread's row for tokens t0 + c .. + kChunk - 1 -> epilogue, store.
-      auto finish_chunk = [&](int c, const float (&acc)[C::kChunk]) {
-        float v[C::kChunk];
-#pragma unroll
-        for (int j = 0; j < C::kChunk; ++j) {
-          float a = acc[j];
-          if (PHASE == kCore) a = g_i * fmaf(s_i, a, z_i * zsum_s[c + j]);
-          v[j] = a;
-        }
-#pragma unroll
-        for (int j = 0; j < C::kChunk; ++j) {
-          const int t = t0 + c + j;
-          const __nv_bfloat16 b = __float2bfloat16_rn(v[j]);
-          v[j] = __bfloat162float(b);
-          if (row_ok && t < p.M) p.out[static_cast<int64_t>(t) * p.R + row] = b;
-        }
-        if (PHASE == kAnalysis) {
-          // per-token sum over the tile's 128 rows of the bf16 z actually stored
-#pragma unroll
-          for (int j = 0; j < C::kChunk; ++j) {
-            float s = row_ok ? v[j] : 0.f;
-#pragma unroll
-            for (int off = 16; off > 0; off >>= 1) s += __shfl_xor_sync(0xffffffffu, s, off);
-            v[j] = s;
-          }
-          if (lane == 0) {
-#pragma unroll
-            for (int j = 0; j < C::kChunk; ++j) red[ew * C::kChunk + j] = v[j];
-          }
-          named_barrier_sync(1, 128);
-          if (et < C::kChunk) {
-            const int t = t0 + c + et;
-            // fixed order over the four warps (TMEM quarters 2, 3, 0, 1 -> rows 64.., 96.., 0.., 32..)
-            const float s = (red[2 * C::kChunk + et] + red[3 * C::kChunk + et]) +
-                            (red[0 * C::kChunk + et] + red[1 * C::kChunk + et]);
-            if (t < p.M) p.zsum_part[static_cast<int64_t>(rt) * p.M + t] = s;
-          }
-          named_barrier_sync(1, 128);
-        }
-      };
-
-      if (PHASE == kCore) {
-        // sum_j z[t][j] for the tile's tokens, from the analysis phase's per-tile sums
-        named_barrier_sync(1, 128);
-        for (int j = et; j < BN; j += 128) {
-          const int t = t0 + j;
-          float s = 0.f;
-          if (t < p.M)
-            for (int q = 0; q < p.zsum_tiles; ++q)
-              s += ldcg_f32(p.zsum_part + static_cast<int64_t>(q) * p.M + t);
-          zsum_s[j] = s;
-        }
-        named_barrier_sync(1, 128);
-      }
-
-      if (p.S == 1) {
+      if (!clustered) {
+        const float g_i = (PHASE == kCore && row_ok && p.gamma) ? p.gamma[row] : 1.f;
 #pragma unroll 1
-        for (int c = 0; c < BN; c += C::kChunk) {
-          float acc[C::kChunk];
-          tmem_ld16(t_row + c, acc);
-          tmem_wait_ld();
-          finish_chunk(c, acc);
-        }
-        tc_fence_before_sync();
-        mbar_arrive(&tempty[buf]);
-      } else {
-        float* part = p.partial + static_cast<int64_t>(ks) * p.M * p.R;
-#pragma unroll 1
-        for (int c = 0; c < BN; c += C::kChunk) {
-          float acc[C::kChunk];
-          tmem_ld16(t_row + c, acc);
+        for (int c = 0; c < BN; c += kChunk) {
+          float v[kChunk];
+          tmem_ld16(t_row + c, v);
           tmem_wait_ld();
 #pragma unroll
-          for (int j = 0; j < C::kChunk; ++j) {
-            const int t = t0 + c + j;
-            if (row_ok && t < p.M) part[static_cast<int64_t>(t) * p.R + row] = acc[j];
+          for (int q = 0; q < kChunk; ++q) {
+            if (PHASE == kCore) v[q] = g_i * fmaf(s_i, v[q], z_i * zs[c + q]);
+            const __nv_bfloat16 b = __float2bfloat16_rn(v[q]);
+            v[q] = __bfloat162float(b);
+            const int t = t0 + c + q;
+            if (row_ok && t < p.M) p.out[static_cast<int64_t>(t) * p.R + row] = b;
           }
-        }
-        tc_fence_before_sync();
-        mbar_arrive(&tempty[buf]);
-        __threadfence();
-        named_barrier_sync(1, 128);
-        if (et == 0) {
-          const unsigned old = atomicInc(&p.counters[rt * p.TT + tt], static_cast<unsigned>(p.S - 1));
-          *ticket = (old == static_cast<unsigned>(p.S - 1)) ? 1 : 0;
-        }
-        named_barrier_sync(1, 128);
-        if (*ticket) {
-          __threadfence();
-#pragma unroll 1
-          for (int c = 0; c < BN; c += C::kChunk) {
-            float acc[C::kChunk];
+          if (PHASE == kAnalysis && !Lo::kSplit) {
+            // per-token sum over the tile's 128 rows of the bf16 z actually stored
 #pragma unroll
-            for (int j = 0; j < C::kChunk; ++j) {
-              const int t = t0 + c + j;
-              float s = 0.f;
-              if (row_ok && t < p.M)
-                for (int q = 0; q < p.S; ++q)
-                  s += ldcg_f32(p.partial + (static_cast<int64_t>(q) * p.M + t) * p.R + row);
-              acc[j] = s;
+            for (int q = 0; q < kChunk; ++q) {
+              float s = row_ok ? v[q] : 0.f;
+#pragma unroll
+              for (int off = 16; off > 0; off >>= 1) s += __shfl_xor_sync(0xffffffffu, s, off);
+              v[q] = s;
             }
-            finish_chunk(c, acc);
+            if (lane == 0) {
+#pragma unroll
+              for (int q = 0; q < kChunk; ++q) red[ew * kChunk + q] = v[q];
+            }
+            named_barrier_sync(1, kEpi);
+            if (et < kChunk) {
+              const int t = t0 + c + et;
+              // fixed order over the TMEM quarters (rows 0.., 32.., 64.., 96..)
+              const float s = (red[2 * kChunk + et] + red[3 * kChunk + et]) +
+                              (red[0 * kChunk + et] + red[1 * kChunk + et]);
+              if (t < p.M) p.zsum_part[static_cast<int64_t>(rt) * p.M + t] = s;
+            }
+            named_barrier_sync(1, kEpi);
           }
         }
+        tc_fence_before_sync();
+        mbar_arrive(&tempty[buf]);
+        if (Lo::kDecoderZsum) mbar_arrive(&zfree[buf]);
+      } else if (Lo::kSplit) {
+        // ---- cluster split-K: partial tile -> own shared memory, token-major [BN][128]
+#pragma unroll 1
+        for (int c = 0; c < BN; c += kChunk) {
+          float v[kChunk];
+          tmem_ld16(t_row + c, v);
+          tmem_wait_ld();
+#pragma unroll
+          for (int q = 0; q < kChunk; ++q) {
+            if (PHASE == kCore) v[q] = fmaf(s_i, v[q], z_i * zs[c + q]);
+            red_buf[(c + q) * kBM + r_in_tile] = v[q];
+          }
+        }
+        tc_fence_before_sync();
+        mbar_arrive(&tempty[buf]);
+        if (Lo::kDecoderZsum) mbar_arrive(&zfree[buf]);
+        fence_acq_rel_cluster();
+        named_barrier_sync(1, kEpi);
+        if (et == 0)
+          for (int q = 0; q < p.S; ++q) mbar_arrive_cluster(mapa(smem_u32(rdy), q));
+        const bool ok = mbar_wait_cluster(rdy, j & 1);
+        if (!ok) report(p.status, FQ_ERR_TIMEOUT);
+        if (bar_red_or(1, kEpi, !ok)) {
+          if (et == 0) *abort_flag = 1;
+          break;
+        }
+        // reduce rows r0 .. r0 + rcnt of the tile over the S partials, in rank order
+        for (int idx = et; idx < rcnt * BN; idx += kEpi) {
+          const int tok = idx / rcnt, rl = r0 + idx % rcnt;
+          const uint32_t off = red_addr + static_cast<uint32_t>((tok * kBM + rl) * 4);
+          float part[kMaxSplits];
+#pragma unroll
+          for (int q = 0; q < kMaxSplits; ++q)
+            part[q] = q < p.S ? ld_dsmem_f32(mapa(off, q)) : 0.f;
+          float s = part[0];
+#pragma unroll
+          for (int q = 1; q < kMaxSplits; ++q)
+            if (q < p.S) s += part[q];
+          const int orow = rt * kBM + rl, t = t0 + tok;
+          if (orow < p.R && t < p.M) {
+            if (PHASE == kCore && p.gamma) s *= p.gamma[orow];
+            p.out[static_cast<int64_t>(t) * p.R + orow] = __float2bfloat16_rn(s);
+          }
+        }
+        named_barrier_sync(1, kEpi);    // this CTA's reads of every partial are done
+        if (et == 0)
+          for (int q = 0; q < p.S; ++q) mbar_arrive_cluster(mapa(smem_u32(cons), q));
       }
       if (++buf == 2) buf = 0, acc_phase ^= 1;
     }
+    // Peers may still be reading this CTA's partial tile: do not exit before they are done.
+    if (clustered && j > 0 && !mbar_wait_cluster(cons, (j - 1) & 1))
+      report(p.status, FQ_ERR_TIMEOUT);
   } else {
     // ---------------------------------------------------------------- code decoders (core)
     if (kCodes) {
       const int r = threadIdx.x - 192;    // row of the tile this thread decodes
       int stage = 0;
       uint32_t phase = 0;
-      for (int u = first_unit; u < p.units && !*abort_flag; u += unit_step) {
-        int rt, tt, ks;
-        unit_coords(p, u, rt, tt, ks);
-        const int k0 = ks * p.kb_per_split, k1 = min(p.KB, k0 + p.kb_per_split);
+      int buf = 0;
+      uint32_t zphase = 0;
+      constexpr int kSlots = Lo::kDecoderZsum ? (BN * 8 + 127) / 128 : 1;
+      for (int tile = static_cast<int>(cid); tile < p.tiles && !*abort_flag;
+           tile += static_cast<int>(ncl)) {
+        float zacc[kSlots];
+#pragma unroll
+        for (int i = 0; i < kSlots; ++i) zacc[i] = 0.f;
         bool ok = true;
         for (int kb = k0; kb < k1; ++kb) {
-          if (!mbar_wait(&full[stage], phase)) {
+          if (!mbar_wait(&cfull[stage], phase, abort_flag)) {
             ok = false;
             break;
           }
           const uint4 w4 = reinterpret_cast<const uint4*>(sCodes + stage * kCodeBytes)[r];
           decode_row(w4, sA + stage * kATileBytes, r);
+          if (Lo::kDecoderZsum) {
+            // sum of this stage's z values (the B tile), 16-byte chunks r + 128 i
+            if (!mbar_wait(&full[stage], phase, abort_flag)) {
+              ok = false;
+              break;
+            }
+            const uint8_t* bt = sB + stage * kBTile;
+#pragma unroll
+            for (int i = 0; i < kSlots; ++i) {
+              const int ci = r + 128 * i;
+              if (ci < BN * 8)
+                zacc[i] += sum_bf16x8(*reinterpret_cast<const uint4*>(bt + ci * 16));
+            }
+          }
           fence_proxy_async_smem();
           mbar_arrive(&aready[stage]);
           if (++stage == S_) stage = 0, phase ^= 1;
@@ -464,6 +567,29 @@ __global__ void __launch_bounds__(threads_for<PHASE>(), 1)
           *abort_flag = 1;
           break;
         }
+        if (Lo::kDecoderZsum) {
+          // the 8 threads of one token row hold its partial sums: combine, publish
+#pragma unroll
+          for (int i = 0; i < kSlots; ++i) {
+            zacc[i] += __shfl_xor_sync(0xffffffffu, zacc[i], 1);
+            zacc[i] += __shfl_xor_sync(0xffffffffu, zacc[i], 2);
+            zacc[i] += __shfl_xor_sync(0xffffffffu, zacc[i], 4);
+          }
+          if (!mbar_wait(&zfree[buf], zphase ^ 1, abort_flag)) {
+            report(p.status, FQ_ERR_TIMEOUT);
+            *abort_flag = 1;
+            break;
+          }
+          if ((r & 7) == 0) {
+#pragma unroll
+            for (int i = 0; i < kSlots; ++i) {
+              const int tok = (r + 128 * i) >> 3;
+              if (tok < BN) zsum_s[buf * BN + tok] = zacc[i];
+            }
+          }
+          mbar_arrive(&zready[buf]);
+          if (++buf == 2) buf = 0, zphase ^= 1;
+        }
       }
     }
   }
@@ -472,7 +598,7 @@ __global__ void __launch_bounds__(threads_for<PHASE>(), 1)
   __syncthreads();
   if (warp == 1) {
     tc_fence_after_sync();
-    tmem_dealloc(tmem_base, C::kTmemCols);
+    tmem_dealloc(tmem_base, Lo::kTmemCols);
   }
 }
 
@@ -515,117 +641,152 @@ int pick_bn(int M) {
   return 256;
 }
 
-// Largest split count the planner may choose (also sizes the workspace, so it must not
-// depend on the device).
-int max_splits(int RT, int TT, int KB) {
-  if (static_cast<int64_t>(RT) * TT >= kMaxSMs) return 1;
-  return std::max(1, std::min(kMaxSplits, KB));
+struct DeviceInfo {
+  int dev = -1;
+  int sms = 0;
+};
+
+DeviceInfo device_info() {
+  DeviceInfo d;
+  cudaGetDevice(&d.dev);
+  cudaDeviceGetAttribute(&d.sms, cudaDevAttrMultiProcessorCount, d.dev);
+  if (d.sms <= 0) d.sms = 148;
+  return d;
 }
 
-// Split K so that RT*TT*S units spread evenly over the SMs: minimise the busiest CTA's
-// K blocks plus a fixed per-unit overhead.
-void plan_phase(PhaseArgs& a, int R, int K, int M, int BN, int sms) {
-  a.R = R;
-  a.K = K;
-  a.M = M;
-  a.RT = static_cast<int>(ceil_div(R, kBM));
-  a.TT = static_cast<int>(ceil_div(M, BN));
-  a.KB = static_cast<int>(ceil_div(K, kBK));
-  const int base = a.RT * a.TT;
-  const int smax = std::min(max_splits(a.RT, a.TT, a.KB), a.KB);
-  int best_s = 1;
-  double best = 1e30;
-  for (int s = 1; s <= smax; ++s) {
-    const int kbs = static_cast<int>(ceil_div(a.KB, s));
-    const int seff = static_cast<int>(ceil_div(a.KB, kbs));
-    if (seff != s) continue;
-    const double waves = static_cast<double>(ceil_div(static_cast<int64_t>(base) * s, sms));
-    const double cost = waves * (kbs + 3.0) + (s > 1 ? 2.0 : 0.0);
-    if (cost < best - 1e-9) best = cost, best_s = s;
+template <int PHASE, int BN>
+cudaError_t prepare_kernel(int dev) {
+  static std::mutex mu;
+  static std::map<int, bool> done;
+  std::lock_guard<std::mutex> g(mu);
+  if (done[dev]) return cudaSuccess;
+  cudaError_t e = cudaFuncSetAttribute(tc_phase_kernel<PHASE, BN>,
+                                       cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       Layout<PHASE, BN>::kBytes);
+  if (e == cudaSuccess) done[dev] = true;
+  return e;
+}
+
+// Largest number of co-resident clusters of `S` CTAs for this kernel (0 if none).
+template <int PHASE, int BN>
+int max_clusters(int dev, int S) {
+  static std::mutex mu;
+  static std::map<std::pair<int, int>, int> cache;
+  std::lock_guard<std::mutex> g(mu);
+  const auto key = std::make_pair(dev, S);
+  const auto it = cache.find(key);
+  if (it != cache.end()) return it->second;
+  cudaLaunchConfig_t cfg{};
+  cfg.gridDim = dim3(static_cast<unsigned>(S * 64));
+  cfg.blockDim = dim3(threads_for<PHASE>());
+  cfg.dynamicSmemBytes = Layout<PHASE, BN>::kBytes;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = static_cast<unsigned>(S);
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  int n = 0;
+  if (cudaOccupancyMaxActiveClusters(&n, tc_phase_kernel<PHASE, BN>, &cfg) != cudaSuccess) {
+    cudaGetLastError();
+    n = 0;
+  }
+  cache[key] = n;
+  return n;
+}
+
+// Split K over clusters of S CTAs so that the tiles' K blocks spread evenly over the
+// co-resident clusters: minimise waves * (K blocks per split + fixed per-tile cost).
+template <int PHASE, int BN>
+void plan_phase(PhaseArgs& a, const DeviceInfo& d, int& grid) {
+  a.RT = static_cast<int>(ceil_div(a.R, kBM));
+  a.TT = static_cast<int>(ceil_div(a.M, BN));
+  a.KB = static_cast<int>(ceil_div(a.K, kBK));
+  a.tiles = a.RT * a.TT;
+  int best_s = 1, best_par = std::min(a.tiles, d.sms);
+  double best = static_cast<double>(ceil_div(a.tiles, best_par)) * (a.KB + 3.0);
+  if (Layout<PHASE, BN>::kSplit) {
+    for (int s = 2; s <= std::min(kMaxSplits, a.KB); ++s) {
+      const int kbs = static_cast<int>(ceil_div(a.KB, s));
+      if (ceil_div(a.KB, kbs) != s) continue;
+      const int cl = std::min(max_clusters<PHASE, BN>(d.dev, s), a.tiles);
+      if (cl <= 0) continue;
+      const double cost = static_cast<double>(ceil_div(a.tiles, cl)) * (kbs + 3.0) + 1.0;
+      if (cost < best - 1e-9) best = cost, best_s = s, best_par = cl;
+    }
   }
   a.S = best_s;
   a.kb_per_split = static_cast<int>(ceil_div(a.KB, best_s));
-  a.units = base * best_s;
+  grid = best_par * best_s;
 }
 
 struct WsLayout {
-  size_t counters, z, u, zsum, partial, total;
+  size_t z, u, zsum, total;
 };
 
-WsLayout ws_layout(int M, int d_in, int n_in, int n_out, int d_out) {
+WsLayout ws_layout(int M, int n_in, int n_out) {
   WsLayout L{};
-  const int BN = pick_bn(M);
-  const int TT = static_cast<int>(ceil_div(M, BN));
   size_t off = kWsHeader;
-  L.counters = off;
-  off += round_up(3 * kMaxCounterTiles * sizeof(unsigned), 256);
   L.z = off;
   off += round_up(static_cast<int64_t>(M) * n_in * 2, 256);
   L.u = off;
   off += round_up(static_cast<int64_t>(M) * n_out * 2, 256);
   L.zsum = off;
   off += round_up(ceil_div(n_in, kBM) * M * 4, 256);
-  L.partial = off;
-  const int R[3] = {n_in, n_out, d_out};
-  const int K[3] = {d_in, n_in, n_out};
-  int64_t part = 0;
-  for (int ph = 0; ph < 3; ++ph) {
-    const int RT = static_cast<int>(ceil_div(R[ph], kBM));
-    const int KB = static_cast<int>(ceil_div(K[ph], kBK));
-    const int s = max_splits(RT, TT, KB);
-    if (s > 1) part = std::max<int64_t>(part, static_cast<int64_t>(s) * M * R[ph] * 4);
-  }
-  off += round_up(part, 256);
   L.total = off;
   return L;
 }
 
-int device_sms() {
-  int dev = 0, sms = 0;
-  cudaGetDevice(&dev);
-  cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
-  return sms > 0 ? sms : 148;
-}
-
 template <int PHASE, int BN>
 cudaError_t launch_phase(const CUtensorMap& tmA, const CUtensorMap& tmB, const PhaseArgs& a,
-                         int sms, bool pdl, cudaStream_t s) {
-  auto kern = tc_phase_kernel<PHASE, BN>;
-  constexpr int smem = smem_bytes_for<BN>();
-  static bool attr_set = false;   // per instantiation; harmless to repeat
-  if (!attr_set) {
-    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
-    if (e != cudaSuccess) return e;
-    attr_set = true;
-  }
+                         int grid, cudaStream_t s) {
   cudaLaunchConfig_t cfg{};
-  cfg.gridDim = dim3(static_cast<unsigned>(std::min(a.units, sms)));
+  cfg.gridDim = dim3(static_cast<unsigned>(grid));
   cfg.blockDim = dim3(threads_for<PHASE>());
-  cfg.dynamicSmemBytes = smem;
+  cfg.dynamicSmemBytes = Layout<PHASE, BN>::kBytes;
   cfg.stream = s;
-  cudaLaunchAttribute attr[1];
+  cudaLaunchAttribute attr[2];
   attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
   attr[0].val.programmaticStreamSerializationAllowed = 1;
+  attr[1].id = cudaLaunchAttributeClusterDimension;
+  attr[1].val.clusterDim.x = static_cast<unsigned>(a.S);
+  attr[1].val.clusterDim.y = 1;
+  attr[1].val.clusterDim.z = 1;
   cfg.attrs = attr;
-  cfg.numAttrs = pdl ? 1 : 0;
-  return cudaLaunchKernelEx(&cfg, kern, tmA, tmB, a);
+  cfg.numAttrs = a.S > 1 ? 2 : 1;
+  return cudaLaunchKernelEx(&cfg, tc_phase_kernel<PHASE, BN>, tmA, tmB, a);
 }
 
 // maps: {T_in, x, z, T_out^T, u}.  The core phase's A operand is the packed codes, so it gets
 // an unused map in that slot.
 template <int BN>
-cudaError_t launch_all(const CUtensorMap* maps, PhaseArgs* a, int sms, cudaStream_t s) {
-  cudaError_t e = launch_phase<kAnalysis, BN>(maps[0], maps[1], a[0], sms, false, s);
-  if (e != cudaSuccess) return e;
-  e = launch_phase<kCore, BN>(maps[1], maps[2], a[1], sms, true, s);   // A map unused
-  if (e != cudaSuccess) return e;
-  return launch_phase<kSynthesis, BN>(maps[3], maps[4], a[2], sms, true, s);
+fq_status run_forward(const CUtensorMap* maps, PhaseArgs* a, cudaStream_t s) {
+  const DeviceInfo d = device_info();
+  if (prepare_kernel<kAnalysis, BN>(d.dev) != cudaSuccess ||
+      prepare_kernel<kCore, BN>(d.dev) != cudaSuccess ||
+      prepare_kernel<kSynthesis, BN>(d.dev) != cudaSuccess)
+    return FQ_ERR_CUDA;
+  int g[3];
+  plan_phase<kAnalysis, BN>(a[0], d, g[0]);
+  plan_phase<kCore, BN>(a[1], d, g[1]);
+  plan_phase<kSynthesis, BN>(a[2], d, g[2]);
+  // the per-tile sums of z come from the analysis epilogue only when it is not split
+  if (!Layout<kCore, BN>::kDecoderZsum && a[0].S != 1) return FQ_ERR_UNSUPPORTED;
+  a[1].zsum_tiles = a[0].RT;
+  if (launch_phase<kAnalysis, BN>(maps[0], maps[1], a[0], g[0], s) != cudaSuccess ||
+      launch_phase<kCore, BN>(maps[1], maps[2], a[1], g[1], s) != cudaSuccess ||
+      launch_phase<kSynthesis, BN>(maps[3], maps[4], a[2], g[2], s) != cudaSuccess)
+    return FQ_ERR_CUDA;
+  return FQ_OK;
 }
 
 }  // namespace
 
 size_t tc_workspace_bytes(int M, int d_in, int n_in, int n_out, int d_out) {
-  return ws_layout(M, d_in, n_in, n_out, d_out).total;
+  (void)d_in;
+  (void)d_out;
+  return ws_layout(M, n_in, n_out).total;
 }
 
 fq_status launch_tc_forward(const void* x, int M, int d_in, const void* T_in,
@@ -633,16 +794,13 @@ fq_status launch_tc_forward(const void* x, int M, int d_in, const void* T_in,
                             const float* gamma, void* y, char* ws, size_t ws_bytes,
                             cudaStream_t s) {
   const int n_in = Cq.n_in, n_out = Cq.n_out;
-  const WsLayout L = ws_layout(M, d_in, n_in, n_out, d_out);
+  const WsLayout L = ws_layout(M, n_in, n_out);
   if (ws_bytes < L.total) return FQ_ERR_WORKSPACE;
   const int BN = pick_bn(M);
-  const int sms = device_sms();
   auto* status = reinterpret_cast<int32_t*>(ws);
-  auto* counters = reinterpret_cast<unsigned*>(ws + L.counters);
   auto* z = reinterpret_cast<__nv_bfloat16*>(ws + L.z);
   auto* u = reinterpret_cast<__nv_bfloat16*>(ws + L.u);
   auto* zsum = reinterpret_cast<float*>(ws + L.zsum);
-  auto* partial = reinterpret_cast<float*>(ws + L.partial);
 
   PhaseArgs a[3];
   const int R[3] = {n_in, n_out, d_out};
@@ -650,14 +808,24 @@ fq_status launch_tc_forward(const void* x, int M, int d_in, const void* T_in,
   __nv_bfloat16* outs[3] = {z, u, reinterpret_cast<__nv_bfloat16*>(y)};
   for (int ph = 0; ph < 3; ++ph) {
     a[ph] = PhaseArgs{};
-    plan_phase(a[ph], R[ph], K[ph], M, BN, sms);
-    if (a[ph].S > 1 && a[ph].RT * a[ph].TT > kMaxCounterTiles) return FQ_ERR_UNSUPPORTED;
+    a[ph].R = R[ph];
+    a[ph].K = K[ph];
+    a[ph].M = M;
     a[ph].out = outs[ph];
-    a[ph].partial = partial;
-    a[ph].counters = counters + ph * kMaxCounterTiles;
     a[ph].zsum_part = zsum;
-    a[ph].zsum_tiles = static_cast<int>(ceil_div(n_in, kBM));
     a[ph].status = status;
+  }
+  // Warm L2 with the code words, and with T_out^T when both fit comfortably, while the
+  // analysis phase streams T_in (small batches only: there the phases are HBM-bound).
+  const int64_t code_bytes = static_cast<int64_t>(fq_packed_words(n_out, n_in)) * 4;
+  const int64_t tout_bytes = static_cast<int64_t>(d_out) * n_out * 2;
+  if (M <= 64 && code_bytes <= kL2PrefetchBudget) {
+    a[0].pf_base[0] = reinterpret_cast<const char*>(Cq.words);
+    a[0].pf_bytes[0] = code_bytes;
+    if (code_bytes + tout_bytes <= kL2PrefetchBudget) {
+      a[0].pf_base[1] = static_cast<const char*>(T_out_t);
+      a[0].pf_bytes[1] = tout_bytes;
+    }
   }
   a[1].words = Cq.words;
   a[1].scale = reinterpret_cast<const __half*>(Cq.scale);
@@ -670,17 +838,14 @@ fq_status launch_tc_forward(const void* x, int M, int d_in, const void* T_in,
       !make_tmap(&maps[2], z, M, n_in, BN) || !make_tmap(&maps[3], T_out_t, d_out, n_out, kBM) ||
       !make_tmap(&maps[4], u, M, n_out, BN))
     return FQ_ERR_CUDA;
-  if (cudaMemsetAsync(ws, 0, L.z, s) != cudaSuccess) return FQ_ERR_CUDA;
 
-  cudaError_t e;
   switch (BN) {
-    case 16: e = launch_all<16>(maps, a, sms, s); break;
-    case 32: e = launch_all<32>(maps, a, sms, s); break;
-    case 64: e = launch_all<64>(maps, a, sms, s); break;
-    case 128: e = launch_all<128>(maps, a, sms, s); break;
-    default: e = launch_all<256>(maps, a, sms, s); break;
+    case 16: return run_forward<16>(maps, a, s);
+    case 32: return run_forward<32>(maps, a, s);
+    case 64: return run_forward<64>(maps, a, s);
+    case 128: return run_forward<128>(maps, a, s);
+    default: return run_forward<256>(maps, a, s);
   }
-  return e == cudaSuccess ? FQ_OK : FQ_ERR_CUDA;
 }
 
 }  // namespace fq
