@@ -174,6 +174,31 @@ fq_status fq_coefficients(const float* W, int d_out, int d_in, const float* T_in
 fq_status fq_quantize_rtn(const float* C, int n_out, int n_in, uint8_t* codes, uint16_t* scale,
                           uint16_t* zero, float* gamma, fq_stream_t stream);
 
+/* ------------------------------------------------------------------------------------------
+ * Forward pass without a caller-provided workspace.  The paper has no counterpart: this is a
+ * convenience of the library for callers that cannot allocate device memory.
+ * ---------------------------------------------------------------------------------------- */
+
+/* Bytes of the library's own device scratch array used by fq_linear_forward_static. */
+#define FQ_STATIC_SCRATCH_BYTES (16u << 20)
+
+/* fq_linear_forward without `ws`: for callers that cannot allocate device memory (a host
+ * framework that owns every allocation, a plugin interface that passes only inputs and
+ * outputs, a C program without an allocator).  The scratch space is a __device__ array of
+ * FQ_STATIC_SCRATCH_BYTES inside this library, reserved on every GPU that loads it until the
+ * process exits; this call allocates nothing.
+ *   - Requests whose fq_workspace_bytes(M, d_in, C->n_in, C->n_out, d_out, mode) exceeds
+ *     FQ_STATIC_SCRATCH_BYTES return FQ_ERR_UNSUPPORTED and launch nothing.
+ *   - The first call on a device looks up the array's device address for that device (with
+ *     that device current); make that first call before any stream capture.
+ *   - All calls share the array and it keeps the last call's contents: calls whose work may
+ *     overlap on the GPU (other streams, other host threads) race on it.
+ *   - The device status word is inside the array, so device-side findings are not reported.
+ * Other arguments, requirements and errors are those of fq_linear_forward. */
+fq_status fq_linear_forward_static(const void* x, int M, int d_in, const void* T_in,
+                                   const fq_packed* C, const void* T_out_t, int d_out,
+                                   const float* gamma, void* y, int mode, fq_stream_t stream);
+
 /* Synchronize `stream` and read the device status word at `status_word` (the head of a
  * forward workspace, or the `status` given to fq_pack).  Returns FQ_OK, FQ_ERR_TIMEOUT,
  * FQ_ERR_DEVICE_CHECK, or FQ_ERR_CUDA if the synchronization itself failed. */

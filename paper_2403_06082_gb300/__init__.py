@@ -18,7 +18,9 @@ __all__ = [
     "fq_packed_words", "fq_pack", "fq_workspace_bytes", "fq_linear_forward", "fq_check",
     "fq_status_str", "EXPORTED", "fq_frame_workspace_bytes", "fq_frame_build",
     "fq_coefficients_workspace_bytes", "fq_coefficients", "fq_quantize_rtn",
+    "fq_linear_forward_static", "FQ_STATIC_SCRATCH_BYTES",
 ]
+FQ_STATIC_SCRATCH_BYTES = 16 << 20
 
 FQ_BF16 = 0
 FQ_FP32_DEBUG = 1
@@ -27,7 +29,8 @@ STATUS = {0: "FQ_OK", 1: "FQ_ERR_INVALID_ARG", 2: "FQ_ERR_ALIGNMENT", 3: "FQ_ERR
           7: "FQ_ERR_DEVICE_CHECK"}
 EXPORTED = ("fq_packed_words", "fq_pack", "fq_workspace_bytes", "fq_linear_forward",
             "fq_check", "fq_status_str", "fq_frame_workspace_bytes", "fq_frame_build",
-            "fq_coefficients_workspace_bytes", "fq_coefficients", "fq_quantize_rtn")
+            "fq_coefficients_workspace_bytes", "fq_coefficients", "fq_quantize_rtn",
+            "fq_linear_forward_static")
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
 
@@ -94,6 +97,11 @@ def lib() -> ctypes.CDLL:
                                       ctypes.c_void_p, ctypes.c_int, ctypes.c_void_p,
                                       ctypes.c_int, ctypes.c_void_p, ctypes.c_void_p,
                                       ctypes.c_size_t, ctypes.c_void_p]
+        L.fq_linear_forward_static.restype = ctypes.c_int
+        L.fq_linear_forward_static.argtypes = [
+            ctypes.c_void_p, ctypes.c_int, ctypes.c_int, ctypes.c_void_p,
+            ctypes.POINTER(_Packed), ctypes.c_void_p, ctypes.c_int, ctypes.c_void_p,
+            ctypes.c_void_p, ctypes.c_int, ctypes.c_void_p]
         L.fq_quantize_rtn.restype = ctypes.c_int
         L.fq_quantize_rtn.argtypes = [ctypes.c_void_p, ctypes.c_int, ctypes.c_int,
                                       ctypes.c_void_p, ctypes.c_void_p, ctypes.c_void_p,
@@ -157,6 +165,16 @@ def fq_linear_forward(x, M: int, d_in: int, T_in, C: Packed, T_out_t, d_out: int
     _ok(lib().fq_linear_forward(_ptr(x), M, d_in, _ptr(T_in), ctypes.byref(pc), _ptr(T_out_t),
                                 d_out, _ptr(gamma), _ptr(y), _ptr(ws), ws_bytes, mode,
                                 _stream(stream)), "fq_linear_forward")
+
+
+def fq_linear_forward_static(x, M: int, d_in: int, T_in, C: Packed, T_out_t, d_out: int, gamma,
+                             y, mode: int = FQ_BF16, stream=None) -> None:
+    """fq_linear_forward with the library's own device scratch array instead of a workspace
+    (for callers that cannot allocate device memory; see include/framequant.h)."""
+    pc = C._c()
+    _ok(lib().fq_linear_forward_static(_ptr(x), M, d_in, _ptr(T_in), ctypes.byref(pc),
+                                       _ptr(T_out_t), d_out, _ptr(gamma), _ptr(y), mode,
+                                       _stream(stream)), "fq_linear_forward_static")
 
 
 def fq_check(status_word, stream=None) -> int:
