@@ -194,7 +194,7 @@ class Regime:
         ws_bytes = max(fq.fq_workspace_bytes(M, L["d_in"], L["n_in"], L["n_out"], L["d_out"], 0)
                        for L in self.layers)
         self.ws_bytes = ws_bytes
-        self.ws = torch.empty(ws_bytes, dtype=torch.uint8, device=dev)
+        self.ws = torch.zeros(ws_bytes, dtype=torch.uint8, device=dev)
         for L, layer in zip(self.layers, self.wk.layers):
             X = wl.activations(self.wk, layer, M)
             if rank:
@@ -378,6 +378,52 @@ def reference_arm(args, rank):
     }), flush=True)
 
 
+def measure_prefill(args, fq, wl, torch, dev, rank, world, dist, stream, peaks):
+    """Prefill regime: the same block at M = 2048 with the de-noising filter on."""
+    pre = Regime(fq, wl, torch, "llama2_7b_prefill", 2048, dev, rank, use_gamma=True)
+    pg = pre.capture(pre.layers, stream)
+    torch.cuda.synchronize()
+    if dist is not None:
+        dist.barrier()
+    p_ms, _ = timed_replays(torch, [pg], stream, args.prefill_steps, 3)
+    p_ms = max_over_ranks(p_ms, dist, dev)
+    lgs = [pre.capture([L], stream) for L in pre.layers]
+    _, p_per = timed_replays(torch, lgs, stream, max(5, args.prefill_steps // 2), 3,
+                             events_between=True)
+    fl = [pre.bytes_flops(L)[1] for L in pre.layers]
+    step_fl = sum(fl)
+    tflops = step_fl / (p_ms / args.prefill_steps * 1e-3) / 1e12
+    pdom = max(range(len(fl)), key=lambda i: p_per[i])
+    out = {
+        "M": 2048, "gamma": True, "steps": args.prefill_steps,
+        "us_per_layer": round(aggregate(p_ms, args.prefill_steps, len(fl), world), 2),
+        "tflops": round(tflops * world, 1),
+        "tensor_frac": round(tflops / peaks["bf16_tflops_sustained"], 3),
+        "peak_tflops": peaks["bf16_tflops_sustained"],
+        "per_layer_us": {L["name"]: round(p_per[i] * 1e3, 1) for i, L in enumerate(pre.layers)},
+        "dominant": {"kernel": f"fq_linear_forward[{pre.layers[pdom]['name']}]",
+                     "achieved_tflops": round(fl[pdom] / (p_per[pdom] * 1e-3) / 1e12, 1),
+                     "frac": round(fl[pdom] / (p_per[pdom] * 1e-3) / 1e12
+                                   / peaks["bf16_tflops_sustained"], 3)},
+    }
+    del pg, lgs, pre
+    torch.cuda.empty_cache()
+    return out
+
+
+def prefill_only(args, fq, wl, torch, dev, rank, world, dist, stream, peaks):
+    """--regime prefill: one JSON line for the prefill regime alone (value in us/layer)."""
+    pf = measure_prefill(args, fq, wl, torch, dev, rank, world, dist, stream, peaks)
+    if rank == 0:
+        print(json.dumps({"metric": METRIC, "value": pf["us_per_layer"], "unit": UNIT,
+                          "n_gpus": world, "steps": args.prefill_steps, "warmup": 3,
+                          "higher_is_better": False, "scaling": "weak", "dtype": "bf16",
+                          "config": {"workload": "llama2_7b_block_prefill", "M": 2048},
+                          "prefill": pf}), flush=True)
+    if dist is not None:
+        dist.destroy_process_group()
+
+
 # --------------------------------------------------------------------------- main
 def aggregate(elapsed_ms, steps, layers_per_step, world):
     """Whole-job microseconds per layer from the slowest rank's elapsed time: every rank
@@ -403,6 +449,8 @@ def main(argv=None):
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--prefill-steps", type=int, default=20)
     ap.add_argument("--no-prefill", action="store_true")
+    ap.add_argument("--regime", default="both", choices=["both", "decode", "prefill"],
+                    help="decode (the headline), prefill, or both (default)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     args = ap.parse_args(argv)
     if args.warmup < 3:
@@ -437,6 +485,12 @@ def main(argv=None):
         torch.cuda.synchronize()
         if dist is not None:
             dist.barrier()
+
+    if args.regime == "prefill":
+        prefill_only(args, fq, wl, torch, dev, rank, world, dist, stream, peaks)
+        return
+    if args.regime == "decode":
+        args.no_prefill = True
 
     # ---------------- decode: Llama-2-7B block, M = 16
     dec = Regime(fq, wl, torch, "llama2_7b_decode", 16, dev, rank)
@@ -488,35 +542,8 @@ def main(argv=None):
     torch.cuda.empty_cache()
 
     # ---------------- prefill: same block, M = 2048, de-noising filter on
-    prefill = None
-    if not args.no_prefill:
-        pre = Regime(fq, wl, torch, "llama2_7b_prefill", 2048, dev, rank, use_gamma=True)
-        pg = pre.capture(pre.layers, stream)
-        barrier()
-        p_ms, _ = timed_replays(torch, [pg], stream, args.prefill_steps, 3)
-        p_ms = max_over_ranks(p_ms, dist, dev)
-        lgs = [pre.capture([L], stream) for L in pre.layers]
-        _, p_per = timed_replays(torch, lgs, stream, max(5, args.prefill_steps // 2), 3,
-                                 events_between=True)
-        fl = [pre.bytes_flops(L)[1] for L in pre.layers]
-        step_fl = sum(fl)
-        tflops = step_fl / (p_ms / args.prefill_steps * 1e-3) / 1e12
-        pdom = max(range(len(fl)), key=lambda i: p_per[i])
-        prefill = {
-            "M": 2048, "gamma": True, "steps": args.prefill_steps,
-            "us_per_layer": round(aggregate(p_ms, args.prefill_steps, len(fl), world), 2),
-            "tflops": round(tflops * world, 1),
-            "tensor_frac": round(tflops / peaks["bf16_tflops_sustained"], 3),
-            "peak_tflops": peaks["bf16_tflops_sustained"],
-            "per_layer_us": {L["name"]: round(p_per[i] * 1e3, 1)
-                             for i, L in enumerate(pre.layers)},
-            "dominant": {"kernel": f"fq_linear_forward[{pre.layers[pdom]['name']}]",
-                         "achieved_tflops": round(fl[pdom] / (p_per[pdom] * 1e-3) / 1e12, 1),
-                         "frac": round(fl[pdom] / (p_per[pdom] * 1e-3) / 1e12
-                                       / peaks["bf16_tflops_sustained"], 3)},
-        }
-        del pg, lgs, pre
-        torch.cuda.empty_cache()
+    prefill = None if args.no_prefill else measure_prefill(args, fq, wl, torch, dev, rank, world,
+                                                            dist, stream, peaks)
 
     if dist is not None:
         dist.barrier()

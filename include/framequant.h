@@ -106,8 +106,12 @@ size_t fq_workspace_bytes(int M, int d_in, int n_in, int n_out, int d_out, int m
  *   gamma    device fp32 [n_out] de-noising gain, or NULL for none
  *   y        device, M x d_out output (bf16 or fp32 by mode)
  *   ws       device workspace of at least fq_workspace_bytes(M, d_in, n_in, n_out, d_out,
- *            mode) bytes, 256-byte aligned; its first 4 bytes hold the device status word,
- *            which every call clears before its kernels run
+ *            mode) bytes, 256-byte aligned, ZERO-FILLED BEFORE ITS FIRST USE.  Its first 64 KiB
+ *            are a header at fixed offsets (status word, a call generation counter, per-tile
+ *            ready flags and split tickets) that every completed call leaves ready for the
+ *            next, so a workspace can be reused across calls and layer shapes without being
+ *            cleared again; zero it again after a call reported FQ_ERR_TIMEOUT.  Its first 4
+ *            bytes are the device status word, which each call clears before reporting.
  *   mode     FQ_BF16 or FQ_FP32_DEBUG
  * Requirements: M, d_in, d_out >= 1; d_in and d_out multiples of 8; C->n_in and C->n_out
  * positive multiples of 16; all device pointers 16-byte aligned.

@@ -41,7 +41,9 @@ fq_status fq_pack(const uint8_t* codes, int n_out, int n_in, uint32_t* words, in
 
 size_t fq_workspace_bytes(int M, int d_in, int n_in, int n_out, int d_out, int mode) {
   if (M <= 0 || d_in <= 0 || n_in <= 0 || n_out <= 0 || d_out <= 0) return 0;
-  if (mode == FQ_BF16) return tc_workspace_bytes(M, d_in, n_in, n_out, d_out);
+  if (mode == FQ_BF16)
+    return M <= kDecodeMaxM ? decode_workspace_bytes(M, d_in, n_in, n_out, d_out)
+                            : tc_workspace_bytes(M, d_in, n_in, n_out, d_out);
   if (mode == FQ_FP32_DEBUG) return debug_workspace_bytes(M, n_in, n_out);
   return 0;
 }
@@ -74,6 +76,9 @@ fq_status fq_linear_forward(const void* x, int M, int d_in, const void* T_in,
   }
   if (current_cc() != 103) return FQ_ERR_UNSUPPORTED;
   // the status word is cleared by the forward's first kernel, in stream order
+  if (M <= kDecodeMaxM)
+    return launch_decode_forward(x, M, d_in, T_in, *C, T_out_t, d_out, gamma, y,
+                                 static_cast<char*>(ws), ws_bytes, s);
   return launch_tc_forward(x, M, d_in, T_in, *C, T_out_t, d_out, gamma, y,
                            static_cast<char*>(ws), ws_bytes, s);
 }

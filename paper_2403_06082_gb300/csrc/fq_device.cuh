@@ -284,6 +284,33 @@ __device__ __forceinline__ void fence_acq_rel_cluster() {
 }
 
 // ---------------------------------------------------------------------------------------------
+// gpu-scope flags
+// ---------------------------------------------------------------------------------------------
+__device__ __forceinline__ uint32_t ld_acquire_gpu(const uint32_t* p) {
+  uint32_t v;
+  asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+  return v;
+}
+
+__device__ __forceinline__ void st_release_gpu(uint32_t* p, uint32_t v) {
+  asm volatile("st.release.gpu.global.u32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
+}
+
+// Bounded wait until *flag == want (flags only move forward by one generation per call).
+// Returns false when the limit ran out or `abort_flag` was raised.
+__device__ __forceinline__ bool wait_flag(const uint32_t* flag, uint32_t want,
+                                          const volatile int* abort_flag) {
+  if (ld_acquire_gpu(flag) == want) return true;
+  const long long t0 = clock64();
+  while (ld_acquire_gpu(flag) != want) {
+    if (clock64() - t0 > kWaitLimitCycles) return false;
+    if (abort_flag && *abort_flag) return false;
+    __nanosleep(64);
+  }
+  return true;
+}
+
+// ---------------------------------------------------------------------------------------------
 // misc
 // ---------------------------------------------------------------------------------------------
 __device__ __forceinline__ void named_barrier_sync(uint32_t id, uint32_t nthreads) {

@@ -15,8 +15,18 @@ constexpr int kColBlock = 64;   // columns per packed block and per K stage
 inline int64_t ceil_div(int64_t a, int64_t b) { return (a + b - 1) / b; }
 inline int64_t round_up(int64_t a, int64_t b) { return ceil_div(a, b) * b; }
 
-// Workspace header: [0, 4) status word, [4, 256) reserved; counters follow.
-constexpr size_t kWsHeader = 256;
+// Workspace header (64 KiB, at fixed offsets whatever the layer's sizes, so that one workspace
+// can serve layers of different shapes): [0] device status word, [4] generation counter,
+// [8] end-of-call ticket, [1024] ready flags and [kWsTickets] split tickets of up to
+// kWsMaxTiles row tiles per phase.  A zero-filled header is a valid initial state and every
+// completed call leaves it valid for the next one.
+constexpr size_t kWsHeader = 64 * 1024;
+constexpr size_t kWsGen = 4;
+constexpr size_t kWsDone = 8;
+constexpr int kWsMaxTiles = 2048;
+constexpr size_t kWsFlags = 1024;
+constexpr size_t kWsTickets = kWsFlags + 3 * kWsMaxTiles * 4;
+constexpr int kDecodeMaxM = 64;   // batches up to this size take the fused decode kernel
 
 // ---- fq_api.cu
 }  // namespace fq
@@ -32,6 +42,13 @@ size_t debug_workspace_bytes(int M, int n_in, int n_out);
 cudaError_t launch_debug_forward(const float* x, int M, int d_in, const float* T_in,
                                  const fq_packed& C, const float* T_out_t, int d_out,
                                  const float* gamma, float* y, char* ws, cudaStream_t s);
+
+// ---- fq_decode.cu: bf16 path for small batches (one fused persistent kernel)
+size_t decode_workspace_bytes(int M, int d_in, int n_in, int n_out, int d_out);
+fq_status launch_decode_forward(const void* x, int M, int d_in, const void* T_in,
+                                const fq_packed& C, const void* T_out_t, int d_out,
+                                const float* gamma, void* y, char* ws, size_t ws_bytes,
+                                cudaStream_t s);
 
 // ---- fq_tc.cu: bf16 tensor-core path
 size_t tc_workspace_bytes(int M, int d_in, int n_in, int n_out, int d_out);

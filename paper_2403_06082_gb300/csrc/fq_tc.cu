@@ -21,9 +21,12 @@
 // tile to its own shared memory, the CTAs signal one another through cluster-scope mbarrier
 // arrivals, and each reduces a slice of the tile's rows by reading all S partials through
 // distributed shared memory in a fixed order (deterministic, no global partials, no atomics).
-// In the core phase the decoder warps also sum the bf16 z values of every B tile they see, so
-// each split carries its own share of sum(z) from exactly the values its MMAs consumed; with
-// larger batches (one split) the analysis epilogue produces per-tile sums of z instead.
+// In the core phase with small batches, sum(z) comes from the tensor cores: every K step also
+// multiplies the z tile by a constant all-ones A tile into a second accumulator, so each split
+// carries its own share of sum(z), accumulated in fp32 from exactly the bf16 values its MMAs
+// consumed.  With larger batches (one split) the analysis epilogue produces per-tile sums of z
+// instead, which costs no tensor time.  Decoder warps take whole stages in turn (stage i goes
+// to warp i mod 4), so four stages are decoded at once.
 //
 // The three phases are chained with programmatic dependent launch (the analysis kernel too,
 // so consecutive layers chain as well): a kernel's CTAs start on SMs as they free up, load
@@ -74,20 +77,25 @@ template <int PHASE, int BN>
 struct Layout {
   static constexpr bool kCodes = PHASE == kCore;
   static constexpr bool kSplit = BN <= 64;              // cluster split-K allowed
-  static constexpr bool kDecoderZsum = kCodes && BN <= 64;
+  static constexpr bool kOnesZsum = kCodes && BN <= 64;   // sum(z) by an all-ones MMA
   static constexpr int kBTileBytes = BN * kBK * 2;
   static constexpr int kCodesStage = kCodes ? kCodeBytes : 0;
   static constexpr int kStageBytes = kATileBytes + kBTileBytes + kCodesStage;
   static constexpr int kRedBytes = kSplit ? BN * kBM * 4 : 0;
-  static constexpr int kStages = std::min(12, (kSmemBudget - kRedBytes) / kStageBytes);
-  static constexpr uint32_t kTmemCols = 2 * BN < 32 ? 32 : 2 * BN;
+  static constexpr int kOnesBytes = kOnesZsum ? kATileBytes : 0;
+  static constexpr int kStages =
+      std::min(12, (kSmemBudget - kRedBytes - kOnesBytes) / kStageBytes);
+  // accumulators [0, 2 BN); sum(z) accumulators [2 BN, 4 BN)
+  static constexpr int kAccCols = kOnesZsum ? 4 * BN : 2 * BN;
+  static constexpr uint32_t kTmemCols = kAccCols <= 32 ? 32 : (kAccCols <= 64 ? 64 : (kAccCols <= 128 ? 128 : (kAccCols <= 256 ? 256 : 512)));
   // byte offsets from the 1024-aligned base
-  static constexpr int oA = 0;
+  static constexpr int oOnes = 0;
+  static constexpr int oA = oOnes + kOnesBytes;
   static constexpr int oB = oA + kStages * kATileBytes;
   static constexpr int oCodes = oB + kStages * kBTileBytes;
   static constexpr int oRed = oCodes + kStages * kCodesStage;
   static constexpr int oBar = oRed + kRedBytes;
-  static constexpr int kNumBars = 4 * kStages + 2 + 2 + 1 + 2 + 2 + 2;
+  static constexpr int kNumBars = 4 * kStages + 2 + 2 + 1 + 2;
   static constexpr int oMisc = oBar + kNumBars * 8;
   static constexpr int oRedSmall = oMisc + 16;                      // [4][kChunk] floats
   static constexpr int oZsum = oRedSmall + 4 * kChunk * 4;          // [2][BN] floats
@@ -125,15 +133,6 @@ __device__ __forceinline__ void decode_row(const uint4 w4, uint8_t* tile, int r)
       *reinterpret_cast<uint4*>(row + ((c ^ (r & 7)) << 4)) = q;
     }
   }
-}
-
-__device__ __forceinline__ float sum_bf16x8(const uint4 v) {
-  const uint32_t w[4] = {v.x, v.y, v.z, v.w};
-  float s = 0.f;
-#pragma unroll
-  for (int i = 0; i < 4; ++i)
-    s += __uint_as_float(w[i] << 16) + __uint_as_float(w[i] & 0xffff0000u);
-  return s;
 }
 
 __device__ __forceinline__ bool bar_red_or(uint32_t id, uint32_t n, bool v) {
@@ -174,12 +173,11 @@ __global__ void __launch_bounds__(threads_for<PHASE>(), 1)
   uint64_t* mma_done = tempty + 2;
   uint64_t* rdy = mma_done + 1;     // cluster: partials of every CTA written
   uint64_t* cons = rdy + 1;         // cluster: every CTA done reading partials
-  uint64_t* zready = cons + 1;      // core: decoders' sum(z) for the buffer written
-  uint64_t* zfree = zready + 2;     // core: epilogue done reading it
+  uint8_t* sOnes = smem + Lo::oOnes;                               // all-ones A tile
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + Lo::oMisc);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
   float* red = reinterpret_cast<float*>(smem + Lo::oRedSmall);     // [4][kChunk]
-  float* zsum_s = reinterpret_cast<float*>(smem + Lo::oZsum);      // [2][BN]
+  float* zsum_s = reinterpret_cast<float*>(smem + Lo::oZsum);      // [2][BN] (BN >= 128)
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const bool clustered = p.S > 1;
@@ -197,14 +195,12 @@ __global__ void __launch_bounds__(threads_for<PHASE>(), 1)
     for (int s = 0; s < S_; ++s) {
       mbar_init(&full[s], 1);
       mbar_init(&empty[s], 1);
-      mbar_init(&aready[s], kBM);
+      mbar_init(&aready[s], 32);     // one decoder warp per stage
       mbar_init(&cfull[s], 1);
     }
     for (int b = 0; b < 2; ++b) {
       mbar_init(&tfull[b], 1);
       mbar_init(&tempty[b], kEpi);
-      mbar_init(&zready[b], kBM);
-      mbar_init(&zfree[b], kEpi);
     }
     mbar_init(mma_done, 1);
     mbar_init(rdy, static_cast<uint32_t>(p.S));
@@ -213,6 +209,13 @@ __global__ void __launch_bounds__(threads_for<PHASE>(), 1)
     fence_barrier_init();
     if (!kCodes) prefetch_tmap(&tmA);
     prefetch_tmap(&tmB);
+  }
+  if (Lo::kOnesZsum) {
+    // bf16 1.0 everywhere (the swizzle permutes identical chunks, so no layout is needed)
+    for (int i = threadIdx.x; i < kATileBytes / 16; i += blockDim.x)
+      reinterpret_cast<uint4*>(sOnes)[i] = make_uint4(0x3F803F80u, 0x3F803F80u, 0x3F803F80u,
+                                                      0x3F803F80u);
+    fence_proxy_async_smem();
   }
   if (warp == 1) tmem_alloc(tmem_slot, Lo::kTmemCols);
   tc_fence_before_sync();
@@ -344,6 +347,8 @@ __global__ void __launch_bounds__(threads_for<PHASE>(), 1)
         }
         tc_fence_after_sync();
         const uint32_t d_tmem = tmem_base + static_cast<uint32_t>(buf * BN);
+        const uint32_t d_ones = tmem_base + static_cast<uint32_t>(2 * BN + buf * BN);
+        const uint64_t odesc = umma_desc_sw128(smem_u32(sOnes));
         bool ok = true;
         for (int kb = k0; kb < k1; ++kb) {
           ok = mbar_wait(&full[stage], phase, abort_flag) &&
@@ -357,6 +362,9 @@ __global__ void __launch_bounds__(threads_for<PHASE>(), 1)
             // advance 16 bf16 = 32 bytes along K inside the swizzle atom
             umma_bf16(d_tmem, adesc + 2 * k, bdesc + 2 * k, idesc,
                       (kb > k0 || k > 0) ? 1u : 0u);
+            if (Lo::kOnesZsum)
+              umma_bf16(d_ones, odesc + 2 * k, bdesc + 2 * k, idesc,
+                        (kb > k0 || k > 0) ? 1u : 0u);
           }
           issued_any = true;
           umma_commit(&empty[stage]);
@@ -401,7 +409,7 @@ __global__ void __launch_bounds__(threads_for<PHASE>(), 1)
         s_i = __half2float(p.scale[row]);
         z_i = __half2float(p.zero[row]);
       }
-      if (PHASE == kCore && !Lo::kDecoderZsum) {
+      if (PHASE == kCore && !Lo::kOnesZsum) {
         // sum_j z[t][j] for the tile's tokens, from the analysis phase's per-tile sums
         named_barrier_sync(1, kEpi);
         for (int q = et; q < BN; q += kEpi) {
@@ -415,7 +423,6 @@ __global__ void __launch_bounds__(threads_for<PHASE>(), 1)
         named_barrier_sync(1, kEpi);
       }
       bool fail = !mbar_wait(&tfull[buf], acc_phase, abort_flag);
-      if (Lo::kDecoderZsum && !fail) fail = !mbar_wait(&zready[buf], acc_phase, abort_flag);
       if (clustered && j > 0 && !fail) fail = !mbar_wait_cluster(cons, (j - 1) & 1);
       if (fail) report(p.status, FQ_ERR_TIMEOUT);
       if (bar_red_or(1, kEpi, fail || *abort_flag)) {
@@ -426,17 +433,20 @@ __global__ void __launch_bounds__(threads_for<PHASE>(), 1)
       const uint32_t t_row = tmem_base + (static_cast<uint32_t>(quarter * 32) << 16) +
                              static_cast<uint32_t>(buf * BN);
       const float* zs = zsum_s + buf * BN;
+      const uint32_t t_ones = t_row + static_cast<uint32_t>(2 * BN);
 
       if (!clustered) {
         const float g_i = (PHASE == kCore && row_ok && p.gamma) ? p.gamma[row] : 1.f;
 #pragma unroll 1
         for (int c = 0; c < BN; c += kChunk) {
-          float v[kChunk];
+          float v[kChunk], zv[kChunk];
           tmem_ld16(t_row + c, v);
+          if (Lo::kOnesZsum) tmem_ld16(t_ones + c, zv);
           tmem_wait_ld();
 #pragma unroll
           for (int q = 0; q < kChunk; ++q) {
-            if (PHASE == kCore) v[q] = g_i * fmaf(s_i, v[q], z_i * zs[c + q]);
+            const float zsq = Lo::kOnesZsum ? zv[q] : zs[c + q];
+            if (PHASE == kCore) v[q] = g_i * fmaf(s_i, v[q], z_i * zsq);
             const __nv_bfloat16 b = __float2bfloat16_rn(v[q]);
             v[q] = __bfloat162float(b);
             const int t = t0 + c + q;
@@ -468,23 +478,23 @@ __global__ void __launch_bounds__(threads_for<PHASE>(), 1)
         }
         tc_fence_before_sync();
         mbar_arrive(&tempty[buf]);
-        if (Lo::kDecoderZsum) mbar_arrive(&zfree[buf]);
       } else if (Lo::kSplit) {
         // ---- cluster split-K: partial tile -> own shared memory, token-major [BN][128]
 #pragma unroll 1
         for (int c = 0; c < BN; c += kChunk) {
-          float v[kChunk];
+          float v[kChunk], zv[kChunk];
           tmem_ld16(t_row + c, v);
+          if (Lo::kOnesZsum) tmem_ld16(t_ones + c, zv);
           tmem_wait_ld();
 #pragma unroll
           for (int q = 0; q < kChunk; ++q) {
-            if (PHASE == kCore) v[q] = fmaf(s_i, v[q], z_i * zs[c + q]);
+            const float zsq = Lo::kOnesZsum ? zv[q] : zs[c + q];
+            if (PHASE == kCore) v[q] = fmaf(s_i, v[q], z_i * zsq);
             red_buf[(c + q) * kBM + r_in_tile] = v[q];
           }
         }
         tc_fence_before_sync();
         mbar_arrive(&tempty[buf]);
-        if (Lo::kDecoderZsum) mbar_arrive(&zfree[buf]);
         fence_acq_rel_cluster();
         named_barrier_sync(1, kEpi);
         if (et == 0)
@@ -495,22 +505,34 @@ __global__ void __launch_bounds__(threads_for<PHASE>(), 1)
           if (et == 0) *abort_flag = 1;
           break;
         }
-        // reduce rows r0 .. r0 + rcnt of the tile over the S partials, in rank order
-        for (int idx = et; idx < rcnt * BN; idx += kEpi) {
-          const int tok = idx / rcnt, rl = r0 + idx % rcnt;
-          const uint32_t off = red_addr + static_cast<uint32_t>((tok * kBM + rl) * 4);
-          float part[kMaxSplits];
+        // reduce rows r0 .. r0 + rcnt of the tile over the S partials, in rank order; the
+        // loads of four elements are issued together
+        const int total = rcnt * BN;
+        for (int base = et; base < total; base += 4 * kEpi) {
+          float part[4][kMaxSplits];
 #pragma unroll
-          for (int q = 0; q < kMaxSplits; ++q)
-            part[q] = q < p.S ? ld_dsmem_f32(mapa(off, q)) : 0.f;
-          float s = part[0];
+          for (int g = 0; g < 4; ++g) {
+            const int idx = base + g * kEpi;
+            const int tok = idx / rcnt, rl = r0 + idx % rcnt;
+            const uint32_t off = red_addr + static_cast<uint32_t>((tok * kBM + rl) * 4);
 #pragma unroll
-          for (int q = 1; q < kMaxSplits; ++q)
-            if (q < p.S) s += part[q];
-          const int orow = rt * kBM + rl, t = t0 + tok;
-          if (orow < p.R && t < p.M) {
-            if (PHASE == kCore && p.gamma) s *= p.gamma[orow];
-            p.out[static_cast<int64_t>(t) * p.R + orow] = __float2bfloat16_rn(s);
+            for (int q = 0; q < kMaxSplits; ++q)
+              part[g][q] = (idx < total && q < p.S) ? ld_dsmem_f32(mapa(off, q)) : 0.f;
+          }
+#pragma unroll
+          for (int g = 0; g < 4; ++g) {
+            const int idx = base + g * kEpi;
+            if (idx >= total) break;
+            const int tok = idx / rcnt, rl = r0 + idx % rcnt;
+            float sum = part[g][0];
+#pragma unroll
+            for (int q = 1; q < kMaxSplits; ++q)
+              if (q < p.S) sum += part[g][q];
+            const int orow = rt * kBM + rl, t = t0 + tok;
+            if (orow < p.R && t < p.M) {
+              if (PHASE == kCore && p.gamma) sum *= p.gamma[orow];
+              p.out[static_cast<int64_t>(t) * p.R + orow] = __float2bfloat16_rn(sum);
+            }
           }
         }
         named_barrier_sync(1, kEpi);    // this CTA's reads of every partial are done
@@ -525,71 +547,33 @@ __global__ void __launch_bounds__(threads_for<PHASE>(), 1)
   } else {
     // ---------------------------------------------------------------- code decoders (core)
     if (kCodes) {
-      const int r = threadIdx.x - 192;    // row of the tile this thread decodes
+      // stage i of this CTA is decoded by decoder warp i mod 4, four rows per lane
+      const int dw = warp - 6;
       int stage = 0;
       uint32_t phase = 0;
-      int buf = 0;
-      uint32_t zphase = 0;
-      constexpr int kSlots = Lo::kDecoderZsum ? (BN * 8 + 127) / 128 : 1;
-      for (int tile = static_cast<int>(cid); tile < p.tiles && !*abort_flag;
+      int it = 0;
+      bool ok = true;
+      for (int tile = static_cast<int>(cid); tile < p.tiles && ok && !*abort_flag;
            tile += static_cast<int>(ncl)) {
-        float zacc[kSlots];
-#pragma unroll
-        for (int i = 0; i < kSlots; ++i) zacc[i] = 0.f;
-        bool ok = true;
-        for (int kb = k0; kb < k1; ++kb) {
-          if (!mbar_wait(&cfull[stage], phase, abort_flag)) {
-            ok = false;
-            break;
-          }
-          const uint4 w4 = reinterpret_cast<const uint4*>(sCodes + stage * kCodeBytes)[r];
-          decode_row(w4, sA + stage * kATileBytes, r);
-          if (Lo::kDecoderZsum) {
-            // sum of this stage's z values (the B tile), 16-byte chunks r + 128 i
-            if (!mbar_wait(&full[stage], phase, abort_flag)) {
+        for (int kb = k0; kb < k1; ++kb, ++it) {
+          if ((it & 3) == dw) {
+            if (!mbar_wait(&cfull[stage], phase, abort_flag)) {
               ok = false;
               break;
             }
-            const uint8_t* bt = sB + stage * kBTile;
+            const uint4* codes = reinterpret_cast<const uint4*>(sCodes + stage * kCodeBytes);
+            uint8_t* tile_a = sA + stage * kATileBytes;
 #pragma unroll
-            for (int i = 0; i < kSlots; ++i) {
-              const int ci = r + 128 * i;
-              if (ci < BN * 8)
-                zacc[i] += sum_bf16x8(*reinterpret_cast<const uint4*>(bt + ci * 16));
-            }
+            for (int rr = 0; rr < 4; ++rr) decode_row(codes[lane + 32 * rr], tile_a, lane + 32 * rr);
+            fence_proxy_async_smem();
+            mbar_arrive(&aready[stage]);
           }
-          fence_proxy_async_smem();
-          mbar_arrive(&aready[stage]);
           if (++stage == S_) stage = 0, phase ^= 1;
         }
-        if (!ok) {
-          report(p.status, FQ_ERR_TIMEOUT);
-          *abort_flag = 1;
-          break;
-        }
-        if (Lo::kDecoderZsum) {
-          // the 8 threads of one token row hold its partial sums: combine, publish
-#pragma unroll
-          for (int i = 0; i < kSlots; ++i) {
-            zacc[i] += __shfl_xor_sync(0xffffffffu, zacc[i], 1);
-            zacc[i] += __shfl_xor_sync(0xffffffffu, zacc[i], 2);
-            zacc[i] += __shfl_xor_sync(0xffffffffu, zacc[i], 4);
-          }
-          if (!mbar_wait(&zfree[buf], zphase ^ 1, abort_flag)) {
-            report(p.status, FQ_ERR_TIMEOUT);
-            *abort_flag = 1;
-            break;
-          }
-          if ((r & 7) == 0) {
-#pragma unroll
-            for (int i = 0; i < kSlots; ++i) {
-              const int tok = (r + 128 * i) >> 3;
-              if (tok < BN) zsum_s[buf * BN + tok] = zacc[i];
-            }
-          }
-          mbar_arrive(&zready[buf]);
-          if (++buf == 2) buf = 0, zphase ^= 1;
-        }
+      }
+      if (!ok) {
+        report(p.status, FQ_ERR_TIMEOUT);
+        *abort_flag = 1;
       }
     }
   }
@@ -772,7 +756,7 @@ fq_status run_forward(const CUtensorMap* maps, PhaseArgs* a, cudaStream_t s) {
   plan_phase<kCore, BN>(a[1], d, g[1]);
   plan_phase<kSynthesis, BN>(a[2], d, g[2]);
   // the per-tile sums of z come from the analysis epilogue only when it is not split
-  if (!Layout<kCore, BN>::kDecoderZsum && a[0].S != 1) return FQ_ERR_UNSUPPORTED;
+  if (!Layout<kCore, BN>::kOnesZsum && a[0].S != 1) return FQ_ERR_UNSUPPORTED;
   a[1].zsum_tiles = a[0].RT;
   if (launch_phase<kAnalysis, BN>(maps[0], maps[1], a[0], g[0], s) != cudaSuccess ||
       launch_phase<kCore, BN>(maps[1], maps[2], a[1], g[1], s) != cudaSuccess ||

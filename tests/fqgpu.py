@@ -47,7 +47,7 @@ class DeviceLayer:
         y = torch.full((M, L.d_out), float("nan"), dtype=self.dtype, device=DEV)
         nbytes = fq.fq_workspace_bytes(M, L.d_in, L.n_in, L.n_out, L.d_out, mode)
         if ws is None:
-            ws = torch.empty(nbytes, dtype=torch.uint8, device=DEV)
+            ws = torch.zeros(nbytes, dtype=torch.uint8, device=DEV)
         fq.fq_linear_forward(x, M, L.d_in, self.T_in, self.C, self.T_out_t, L.d_out,
                              self.gamma if use_gamma else None, y, ws, nbytes, mode)
         st = fq.fq_check(ws)

@@ -151,7 +151,7 @@ def test_stream_argument():
     x = torch.from_numpy(X).to(DEV, BF16)
     y = torch.empty(16, L.d_out, dtype=BF16, device=DEV)
     nb = fq.fq_workspace_bytes(16, L.d_in, L.n_in, L.n_out, L.d_out, 0)
-    ws = torch.empty(nb, dtype=torch.uint8, device=DEV)
+    ws = torch.zeros(nb, dtype=torch.uint8, device=DEV)
     torch.cuda.synchronize()
     with torch.cuda.stream(s):
         fq.fq_linear_forward(x, 16, L.d_in, D.T_in, D.C, D.T_out_t, L.d_out, D.gamma, y, ws, nb,
