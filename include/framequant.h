@@ -107,16 +107,18 @@ size_t fq_workspace_bytes(int M, int d_in, int n_in, int n_out, int d_out, int m
  *   y        device, M x d_out output (bf16 or fp32 by mode)
  *   ws       device workspace of at least fq_workspace_bytes(M, d_in, n_in, n_out, d_out,
  *            mode) bytes, 256-byte aligned, ZERO-FILLED BEFORE ITS FIRST USE.  Its first 64 KiB
- *            are a header at fixed offsets (status word, a call generation counter, per-tile
- *            ready flags and split tickets) that every completed call leaves ready for the
- *            next, so a workspace can be reused across calls and layer shapes without being
- *            cleared again; zero it again after a call reported FQ_ERR_TIMEOUT.  Its first 4
+ *            are a header at fixed offsets (status word, a call generation counter and
+ *            ready flags per slice of a 128-row output tile) that every completed call leaves
+ *            ready for the next, so a workspace can be reused across calls and layer shapes
+ *            without being cleared again; zero it again after a call reported
+ *            FQ_ERR_TIMEOUT.  Its first 4
  *            bytes are the device status word, which each call clears before reporting.
  *   mode     FQ_BF16 or FQ_FP32_DEBUG
  * Requirements: M, d_in, d_out >= 1; d_in and d_out multiples of 8; C->n_in and C->n_out
  * positive multiples of 16; all device pointers 16-byte aligned.
  * Errors: FQ_ERR_INVALID_ARG, FQ_ERR_ALIGNMENT, FQ_ERR_WORKSPACE, FQ_ERR_UNSUPPORTED (the
- * current device is not compute capability 10.3 in FQ_BF16 mode), FQ_ERR_CUDA. */
+ * current device is not compute capability 10.3 in FQ_BF16 mode, or M <= 64 in FQ_BF16 mode
+ * with n_in, n_out or d_out above 81920 = 640 tiles of 128 rows), FQ_ERR_CUDA. */
 fq_status fq_linear_forward(const void* x, int M, int d_in, const void* T_in,
                             const fq_packed* C, const void* T_out_t, int d_out,
                             const float* gamma, void* y, void* ws, size_t ws_bytes, int mode,

@@ -5,25 +5,31 @@
 //     analysis   z = T_in x              A = T_in   (n_in x d_in),   B = x
 //     core       u = gamma (C_hat z)     A = codes  (n_out x n_in),  B = z
 //     synthesis  y = T_out^T u           A = T_out^T (d_out x n_out), B = u
-// are cut into tasks = (phase, 128-row tile, K split).  CTA b of G runs tasks b, b + G, ... in
-// order; since task indices grow with the phase, every CTA finishes its analysis tasks before
-// its core tasks and those before its synthesis tasks, so no CTA ever waits on work that is
-// queued behind a wait.  A task reads its activations only after the tiles it needs are
-// final: when the last split of a tile has been reduced, its finaliser stamps the tile's
-// ready flag with this call's generation (release), and the activation producer of a
-// dependent task waits for exactly those flags (acquire, bounded).  No phase waits for the
-// whole grid, a split's reduction overlaps other tasks, and the weight producer runs ahead
-// into the next tasks (and warms L2 with this CTA's later weight tiles) while activations
-// are still being produced.
+// are cut into tasks = (phase, 128-row tile).  The kernel runs as clusters of S CTAs; CTA r of
+// a cluster takes K split r of every task of its cluster and reduces slice r (128/S rows) of
+// the task's output tile.  The split-K exchange is one-way: every epilogue thread pushes its
+// row of fp32 partial sums from registers into the receive buffer of the CTA that owns the
+// row (st.async into distributed shared memory, counted by that CTA's own mbarrier), and each
+// CTA adds the S partials of its slice in rank order (deterministic; no global partials, no
+// atomics, no remote arrivals).  Receive buffers alternate between consecutive tasks; a buffer
+// is only written again after its owner has sent the next task's partials, which it does only
+// after reading the buffer, so no back-pressure signal is needed.  Cluster c runs tasks c,
+// c + C, ... in order; task indices grow with the phase, so every cluster finishes its
+// analysis tasks before its core tasks and those before its synthesis tasks, and no cluster
+// waits on work queued behind a wait.  Each CTA stamps the ready flag of its slice with this
+// call's generation (release) once the slice is stored, and the activation producer of a
+// dependent task waits for exactly the slices its K range reads (acquire, bounded, one lane
+// per flag).  No phase waits for the whole grid, and the weight producer runs ahead into the
+// next tasks (and warms L2 with this CTA's later weight tiles) while activations are still
+// being produced.
 //
-// sum(z), needed by the core's zero term, is produced by the analysis finaliser as one sum
-// per 64-column block of z and token, from the bf16 values it stores; a core split adds the
-// blocks of its own K range.
+// sum(z), needed by the core's zero term, is produced with the analysis output as one sum per
+// 16 columns of z and token, from the bf16 values stored; a core split adds the groups of its
+// own K range.
 //
-// The workspace header holds the generation counter, the tiles' ready flags and the split
-// tickets; they must start at zero (a zero-filled workspace) and every call leaves them ready
-// for the next: tickets wrap back to zero, flags keep generations that are all in the past,
-// and the last CTA to finish advances the generation.
+// The workspace header holds the generation counter and the tiles' ready flags; a zero-filled
+// header is a valid start and every call leaves it valid for the next (flags keep
+// generations that are all in the past; the last CTA to finish advances the generation).
 //
 // Warps: 0 weight (A) producer, 1 TMEM owner + MMA issuer, 2-5 epilogue (thread = tile row),
 // 6 activation (B) producer, 7-10 code decoders (core stages, stage i -> warp i mod 4).
@@ -33,6 +39,7 @@
 #include <algorithm>
 #include <map>
 #include <mutex>
+#include <utility>
 
 #include "fq_device.cuh"
 #include "fq_internal.h"
@@ -45,28 +52,28 @@ constexpr int kBK = 64;
 constexpr int kATile = kBM * kBK * 2;      // 16 KiB
 constexpr int kCodeBytes = kBM * kBK / 4;  // 2 KiB
 constexpr int kMaxSplit = 8;
+static_assert(kMaxSplit <= kWsSlices, "one ready flag per slice");
 constexpr int kEpi = 128;
 constexpr int kChunk = 16;
+constexpr int kGroup = 16;                 // columns of z per partial sum
 constexpr int kThreads = 352;
 constexpr int64_t kL2PrefetchBudget = 64ll << 20;
 
 struct DecPhase {
-  int R, K, RT, S, KB, kbs, tasks, base;
+  int R, K, RT, KB, kbs, base;
   __nv_bfloat16* out;     // [M][R]
-  float* partial;         // [S][M][R] when S > 1
-  uint32_t* flags;        // [RT] tile final in this call when == generation + 1
-  uint32_t* tickets;      // [RT] split arrivals (wrap to zero)
+  uint32_t* flags;        // [RT][kWsSlices] slice final in this call when == generation + 1
 };
 
 struct DecArgs {
-  int M, total;
+  int M, S, total;
   DecPhase ph[3];
   const uint32_t* words;
   const __half* scale;
   const __half* zero;
   const float* gamma;
-  float* zsum64;          // [nblk][M] sums of z over 64-column blocks
-  int nblk;
+  float* zsum;            // [ngroups][M] sums of z over groups of 16 columns
+  int ngroups;
   int32_t* status;
   uint32_t* gen;
   uint32_t* done;
@@ -77,22 +84,26 @@ template <int BN>
 struct DecLayout {
   static constexpr int kBTile = BN * kBK * 2;
   static constexpr int kStage = kATile + kBTile + kCodeBytes;
-  static constexpr int kStages = std::min(12, (200 * 1024 - 4096) / kStage);
+  static constexpr int kRecvRow = BN + 4;                     // floats per received row
+  static constexpr int kRecv = kBM * kRecvRow * 4;            // [S][128/S][BN + 4] fp32
+  static constexpr int kStages = std::min(12, (200 * 1024 - 4096 - 2 * kRecv) / kStage);
   static constexpr uint32_t kTmemCols = 2 * BN < 32 ? 32 : 2 * BN;
   static constexpr int oA = 0;
   static constexpr int oB = oA + kStages * kATile;
   static constexpr int oC = oB + kStages * kBTile;
-  static constexpr int oBar = oC + kStages * kCodeBytes;
-  static constexpr int kBars = 4 * kStages + 5;
+  static constexpr int oRecv = oC + kStages * kCodeBytes;    // two receive buffers
+  static constexpr int oBar = oRecv + 2 * kRecv;
+  static constexpr int kBars = 4 * kStages + 7;
   static constexpr int oMisc = oBar + kBars * 8;
-  static constexpr int oRed = oMisc + 16;            // [4][BN] floats
-  static constexpr int oZs = oRed + 4 * BN * 4;      // [BN] floats
-  static constexpr int kBytes = oZs + BN * 4 + 1024;
+  static constexpr int oZs = oMisc + 32;                     // [BN] floats
+  static constexpr int oZsPart = oZs + BN * 4;               // [128] floats
+  static constexpr int kBytes = oZsPart + kEpi * 4 + 1024;
   static_assert(kBTile % 1024 == 0, "B tiles keep 1024-byte alignment");
+  static_assert(kStages >= 3, "pipeline depth");
 };
 
 struct Task {
-  int p, tile, ks;
+  int p, tile;
 };
 
 __device__ __forceinline__ DecPhase phase_of(const DecArgs& a, int p) {
@@ -101,12 +112,11 @@ __device__ __forceinline__ DecPhase phase_of(const DecArgs& a, int p) {
 
 __device__ __forceinline__ Task task_of(const DecArgs& a, int i) {
   const int p = (i >= a.ph[1].base) + (i >= a.ph[2].base);
-  const DecPhase ph = phase_of(a, p);
-  const int j = i - ph.base;
-  return {p, j / ph.S, j % ph.S};
+  return {p, i - phase_of(a, p).base};
 }
 
-// Same code decoding as the three-kernel path: q -> bf16(128 + q) - 128, swizzled row store.
+// q -> bf16(128 + q) - 128 (exact), one 128-byte row of a K-major tile with the 128-byte
+// swizzle (16-byte chunk c of row r lands at chunk c ^ (r mod 8)).
 __device__ __forceinline__ void decode_row_dec(const uint4 w4, uint8_t* tile, int r) {
   const uint32_t wv[4] = {w4.x, w4.y, w4.z, w4.w};
   const __nv_bfloat162 bias = __floats2bfloat162_rn(128.f, 128.f);
@@ -144,7 +154,7 @@ __device__ __forceinline__ bool bar_red_or_dec(uint32_t id, uint32_t n, bool v) 
 }
 
 // First timeout of a call: role, task, stage and a detail word go to status[4..7] (the rest
-// of the header's first 64 bytes), for diagnosis with the status word.
+// of the header's first 32 bytes), for diagnosis together with the status word.
 __device__ __forceinline__ void note_timeout(int32_t* status, int role, int task, int stage,
                                              int detail) {
   report(status, FQ_ERR_TIMEOUT);
@@ -172,8 +182,9 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint8_t* sA = smem + Lo::oA;
   uint8_t* sB = smem + Lo::oB;
   uint8_t* sC = smem + Lo::oC;
+  float* recv_buf = reinterpret_cast<float*>(smem + Lo::oRecv);
   // fullA completes every round of a stage (a weight tile or, for core tasks, its codes);
-  // aready only in core rounds, so its parity is tracked per stage
+  // aready only in core rounds, so the MMA tracks its parity per stage
   uint64_t* fullA = reinterpret_cast<uint64_t*>(smem + Lo::oBar);
   uint64_t* fullB = fullA + S_;
   uint64_t* empty = fullB + S_;
@@ -181,15 +192,23 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint64_t* tfull = aready + S_;
   uint64_t* tempty = tfull + 2;
   uint64_t* mma_done = tempty + 2;
+  uint64_t* recv_bar = mma_done + 1;   // [2] the peers' partials of this CTA's slice arrived
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + Lo::oMisc);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
   uint32_t* gen_s = tmem_slot + 2;
-  int* ticket_s = reinterpret_cast<int*>(tmem_slot + 3);
-  float* red = reinterpret_cast<float*>(smem + Lo::oRed);
   float* zs_s = reinterpret_cast<float*>(smem + Lo::oZs);
+  float* zs_part = reinterpret_cast<float*>(smem + Lo::oZsPart);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int G = gridDim.x;
+  const int S = a.S;
+  const bool clustered = S > 1;
+  uint32_t rank = 0, cid = blockIdx.x, ncl = gridDim.x;
+  if (clustered) {
+    rank = cluster_ctarank();
+    cid = cluster_id_x();
+    ncl = cluster_count_x();
+  }
+  const int ks = static_cast<int>(rank);
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < S_; ++s) {
@@ -203,8 +222,17 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_init(&tempty[b], kEpi);
     }
     mbar_init(mma_done, 1);
+    mbar_init(&recv_bar[0], 1);
+    mbar_init(&recv_bar[1], 1);
     *abort_flag = 0;
     fence_barrier_init();
+    if (clustered) {
+      // arm the receive buffers for this CTA's first two tasks (later tasks re-arm them)
+      const uint32_t bytes = static_cast<uint32_t>((S - 1) * (kBM / S) * BN * 4);
+      for (int b = 0; b < 2; ++b)
+        if (static_cast<int>(cid) + b * static_cast<int>(ncl) < a.total)
+          mbar_arrive_expect_tx(&recv_bar[b], bytes);
+    }
     prefetch_tmap(&tmTin);
     prefetch_tmap(&tmX);
     prefetch_tmap(&tmZ);
@@ -214,9 +242,16 @@ __global__ void __launch_bounds__(kThreads, 1)
   if (warp == 1) tmem_alloc(tmem_slot, Lo::kTmemCols);
   tc_fence_before_sync();
   __syncthreads();
+  if (clustered) cluster_sync();   // every CTA's barriers exist before any remote arrival
   tc_fence_after_sync();
   const uint32_t tmem_base = *tmem_slot;
   pdl_launch_dependents();
+
+  // this CTA's K range of a task of phase ph
+  auto krange = [&](const DecPhase& ph, int& k0, int& k1) {
+    k0 = ks * ph.kbs;
+    k1 = min(ph.KB, k0 + ph.kbs);
+  };
 
   if (warp == 0) {
     // -------------------------------------------------------------- weight (A) producer
@@ -229,10 +264,11 @@ __global__ void __launch_bounds__(kThreads, 1)
       bool used[S_];
 #pragma unroll
       for (int s = 0; s < S_; ++s) last_par[s] = 0, used[s] = false;
-      for (int i = blockIdx.x; i < a.total && !*abort_flag; i += G) {
+      for (int i = static_cast<int>(cid); i < a.total && !*abort_flag; i += static_cast<int>(ncl)) {
         const Task t = task_of(a, i);
         const DecPhase ph = phase_of(a, t.p);
-        const int k0 = t.ks * ph.kbs, k1 = min(ph.KB, k0 + ph.kbs);
+        int k0, k1;
+        krange(ph, k0, k1);
         for (int kb = k0; kb < k1; ++kb) {
           if (!mbar_wait(&empty[stage], phase ^ 1, abort_flag)) {
             if (!*abort_flag) note_timeout(a.status, 1, i, stage, static_cast<int>(phase));
@@ -256,11 +292,13 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (first) {
           first = false;
           // warm L2 with the weight tiles of this CTA's later tasks
-          for (int j = i + G; j < a.total && a.prefetch_later > 0; j += G) {
+          for (int j = i + static_cast<int>(ncl); j < a.total && a.prefetch_later > 0;
+               j += static_cast<int>(ncl)) {
             const Task u = task_of(a, j);
             const DecPhase q = phase_of(a, u.p);
-            const int u0 = u.ks * q.kbs, u1 = min(q.KB, u0 + q.kbs);
-            if (u.p == 1) {
+            int u0, u1;
+            krange(q, u0, u1);
+            if (u.p == 1 && u1 > u0) {
               const uint32_t* src = a.words + (static_cast<int64_t>(u.tile) * q.KB + u0) * 512;
               asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(src),
                            "r"(static_cast<uint32_t>((u1 - u0) * kCodeBytes))
@@ -282,41 +320,48 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
   } else if (warp == 6) {
     // -------------------------------------------------------------- activation (B) producer
-    if (lane == 0) {
-      const uint64_t pol_x = policy_evict_last();
-      pdl_wait();
-      if (blockIdx.x == 0) *a.status = 0;      // a new call
-      const uint32_t g = ld_acquire_gpu(a.gen) + 1;
-      int stage = 0;
-      uint32_t phase = 0;
-      uint32_t last_par[S_];
-      bool used[S_];
+    // the whole warp polls ready flags (one lane per slice); lane 0 issues the loads
+    const uint64_t pol_x = policy_evict_last();
+    pdl_wait();
+    if (blockIdx.x == 0 && lane == 0) *a.status = 0;      // a new call
+    const uint32_t g = ld_acquire_gpu(a.gen) + 1;
+    const int rows_per = kBM / S;
+    int stage = 0;
+    uint32_t phase = 0;
+    uint32_t last_par[S_];
+    bool used[S_];
 #pragma unroll
-      for (int s = 0; s < S_; ++s) last_par[s] = 0, used[s] = false;
-      for (int i = blockIdx.x; i < a.total && !*abort_flag; i += G) {
-        const Task t = task_of(a, i);
-        const DecPhase ph = phase_of(a, t.p);
-        const int k0 = t.ks * ph.kbs, k1 = min(ph.KB, k0 + ph.kbs);
-        if (t.p > 0) {
-          // every source tile covering this task's K range must be final
-          const DecPhase src = phase_of(a, t.p - 1);
-          const int lo = (k0 * kBK) / kBM, hi = (min(ph.K, k1 * kBK) - 1) / kBM;
-          bool ok = true;
-          int bad = -1;
-          for (int s = lo; s <= hi && ok; ++s) {
-            ok = wait_flag(&src.flags[s], g, abort_flag);
-            if (!ok) bad = s;
-          }
-          if (!ok) {
-            if (!*abort_flag)
-              note_timeout(a.status, 2, i, bad,
-                           static_cast<int>(ld_acquire_gpu(&src.flags[bad]) - g) * 1000 + t.p);
-            *abort_flag = 1;
-            break;
-          }
-        }
-        const CUtensorMap* tm = t.p == 0 ? &tmX : (t.p == 1 ? &tmZ : &tmU);
+    for (int s = 0; s < S_; ++s) last_par[s] = 0, used[s] = false;
+    for (int i = static_cast<int>(cid); i < a.total; i += static_cast<int>(ncl)) {
+      if (__shfl_sync(0xffffffffu, *abort_flag != 0, 0)) break;   // warp-uniform
+      const Task t = task_of(a, i);
+      const DecPhase ph = phase_of(a, t.p);
+      int k0, k1;
+      krange(ph, k0, k1);
+      if (t.p > 0 && k1 > k0) {
+        // every slice of the previous phase's output that this CTA's K range reads must be final
+        const DecPhase src = phase_of(a, t.p - 1);
+        const int sl0 = (k0 * kBK) / rows_per, sl1 = (min(ph.K, k1 * kBK) - 1) / rows_per;
         bool ok = true;
+        int bad = sl0;
+        for (int gs = sl0 + lane; gs <= sl1 && ok; gs += 32) {
+          ok = wait_flag(&src.flags[(gs / S) * kWsSlices + gs % S], g, abort_flag);
+          if (!ok) bad = gs;
+        }
+        const unsigned fails = __ballot_sync(0xffffffffu, !ok);
+        if (fails) {
+          if (lane == __ffs(fails) - 1 && !*abort_flag) {
+            const uint32_t* f = &src.flags[(bad / S) * kWsSlices + bad % S];
+            note_timeout(a.status, 2, i, bad, static_cast<int>(ld_acquire_gpu(f) - g) * 1000 + t.p);
+          }
+          __syncwarp();
+          if (lane == 0) *abort_flag = 1;
+          break;
+        }
+      }
+      bool ok = true;
+      if (lane == 0) {
+        const CUtensorMap* tm = t.p == 0 ? &tmX : (t.p == 1 ? &tmZ : &tmU);
         for (int kb = k0; kb < k1; ++kb) {
           if (!mbar_wait(&empty[stage], phase ^ 1, abort_flag)) {
             if (!*abort_flag) note_timeout(a.status, 3, i, stage, static_cast<int>(phase));
@@ -329,16 +374,14 @@ __global__ void __launch_bounds__(kThreads, 1)
           last_par[stage] = phase;
           if (++stage == S_) stage = 0, phase ^= 1;
         }
-        if (!ok) {
-          report(a.status, FQ_ERR_TIMEOUT);
-          *abort_flag = 1;
-          break;
-        }
+        if (!ok) *abort_flag = 1;
       }
+      if (!__shfl_sync(0xffffffffu, ok, 0)) break;
+    }
+    if (lane == 0)
       for (int s = 0; s < S_; ++s)
         if (used[s] && !mbar_wait(&fullB[s], last_par[s], nullptr))
           report(a.status, FQ_ERR_TIMEOUT);
-    }
   } else if (warp == 1) {
     // -------------------------------------------------------------- MMA issuer
     if (lane == 0) {
@@ -349,10 +392,11 @@ __global__ void __launch_bounds__(kThreads, 1)
       uint32_t acc_phase = 0;
       uint32_t apar = 0;     // bit s: parity of the next aready[s] phase
       bool issued_any = false;
-      for (int i = blockIdx.x; i < a.total && !*abort_flag; i += G) {
+      for (int i = static_cast<int>(cid); i < a.total && !*abort_flag; i += static_cast<int>(ncl)) {
         const Task t = task_of(a, i);
         const DecPhase ph = phase_of(a, t.p);
-        const int k0 = t.ks * ph.kbs, k1 = min(ph.KB, k0 + ph.kbs);
+        int k0, k1;
+        krange(ph, k0, k1);
         if (!mbar_wait(&tempty[buf], acc_phase ^ 1, abort_flag)) {
           if (!*abort_flag) note_timeout(a.status, 4, i, buf, static_cast<int>(acc_phase));
           *abort_flag = 1;
@@ -385,11 +429,10 @@ __global__ void __launch_bounds__(kThreads, 1)
           if (++stage == S_) stage = 0, phase ^= 1;
         }
         if (!ok) {
-          report(a.status, FQ_ERR_TIMEOUT);
           *abort_flag = 1;
           break;
         }
-        umma_commit(&tfull[buf]);
+        umma_commit(&tfull[buf]);      // with an empty K range this arrives at once
         if (++buf == 2) buf = 0, acc_phase ^= 1;
       }
       if (issued_any) {
@@ -404,10 +447,11 @@ __global__ void __launch_bounds__(kThreads, 1)
     uint32_t phase = 0;
     int it = 0;
     bool ok = true;
-    for (int i = blockIdx.x; i < a.total && ok && !*abort_flag; i += G) {
+    for (int i = static_cast<int>(cid); i < a.total && ok && !*abort_flag; i += static_cast<int>(ncl)) {
       const Task t = task_of(a, i);
       const DecPhase ph = phase_of(a, t.p);
-      const int k0 = t.ks * ph.kbs, k1 = min(ph.KB, k0 + ph.kbs);
+      int k0, k1;
+      krange(ph, k0, k1);
       for (int kb = k0; kb < k1; ++kb, ++it) {
         // every decoder warp follows every round of the ring (a parity wait is only exact
         // when the waiter is at most one phase ahead), and decodes the code rounds it owns
@@ -437,47 +481,70 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int quarter = warp & 3;                 // TMEM lanes 32 * quarter .. + 31
     const int r_in_tile = quarter * 32 + lane;
     const int et = threadIdx.x - 64;
+    const int rows_per = kBM / S;                 // rows of a tile per slice (one per CTA)
+    const int dest = r_in_tile / rows_per;        // CTA that reduces this thread's row
+    const int rl_own = r_in_tile % rows_per;
+    constexpr int kRow = Lo::kRecvRow;
+    const uint32_t recv_bytes = static_cast<uint32_t>((S - 1) * rows_per * BN * 4);
     pdl_wait();
     if (et == 0) *gen_s = ld_acquire_gpu(a.gen) + 1;
     named_barrier_sync(1, kEpi);
     const uint32_t g = *gen_s;
     int buf = 0;
     uint32_t acc_phase = 0;
-    for (int i = blockIdx.x; i < a.total; i += G) {
+    int j = 0;                                    // tasks finished by this CTA
+    for (int i = static_cast<int>(cid); i < a.total; i += static_cast<int>(ncl), ++j) {
       const Task t = task_of(a, i);
       const DecPhase ph = phase_of(a, t.p);
-      const int k0 = t.ks * ph.kbs, k1 = min(ph.KB, k0 + ph.kbs);
+      int k0, k1;
+      krange(ph, k0, k1);
+      const bool has_k = k1 > k0;
       const int row = t.tile * kBM + r_in_tile;
       const bool row_ok = row < ph.R;
-      float s_i = 0.f, z_i = 0.f, g_i = 1.f;
+      float s_i = 0.f, z_i = 0.f, g_row = 1.f;
+      if (t.p == 1 && row_ok) {
+        s_i = __half2float(a.scale[row]);
+        z_i = __half2float(a.zero[row]);
+        if (a.gamma) g_row = a.gamma[row];
+      }
       bool fail = false;
       if (t.p == 1) {
-        if (row_ok) {
-          s_i = __half2float(a.scale[row]);
-          z_i = __half2float(a.zero[row]);
-          if (a.gamma) g_i = a.gamma[row];
-        }
-        // sum of z over this split's K range, from the 64-column block sums of the analysis
-        if (et == 0) {
-          const int lo = (k0 * kBK) / kBM, hi = (min(ph.K, k1 * kBK) - 1) / kBM;
-          for (int s = lo; s <= hi && !fail; ++s) {
-            fail = !wait_flag(&a.ph[0].flags[s], g, abort_flag);
-            if (fail && !*abort_flag) note_timeout(a.status, 8, i, s, 0);
+        // sum of z over this CTA's K range, from the 16-row group sums of the slices it reads
+        if (has_k) {
+          const int sl0 = (k0 * kBK) / rows_per, sl1 = (min(ph.K, k1 * kBK) - 1) / rows_per;
+          for (int gs = sl0 + et; gs <= sl1 && !fail; gs += kEpi) {
+            fail = !wait_flag(&a.ph[0].flags[(gs / S) * kWsSlices + gs % S], g, abort_flag);
+            if (fail && !*abort_flag) note_timeout(a.status, 8, i, gs, 0);
           }
         }
-        named_barrier_sync(1, kEpi);
-        for (int q = et; q < BN; q += kEpi) {
-          float s = 0.f;
-          if (q < a.M)
-            for (int b = k0; b < k1 && b < a.nblk; ++b) s += ldcg_f32(a.zsum64 + b * a.M + q);
-          zs_s[q] = s;
+        if (bar_red_or_dec(1, kEpi, fail)) {
+          if (et == 0) *abort_flag = 1;
+          break;
+        }
+        {
+          // 128 / BN threads per token each add a strided share of the groups, then one
+          // thread per token adds the shares in a fixed order
+          constexpr int kPer = kEpi / BN;
+          const int q = et % BN, part = et / BN;
+          float sz = 0.f;
+          if (q < a.M && has_k) {
+            const int g0 = k0 * (kBK / kGroup), g1 = min(a.ngroups, k1 * (kBK / kGroup));
+            for (int gi = g0 + part; gi < g1; gi += kPer) sz += ldcg_f32(a.zsum + gi * a.M + q);
+          }
+          zs_part[part * BN + q] = sz;
+          named_barrier_sync(1, kEpi);
+          if (et < BN) {
+            float tot = 0.f;
+#pragma unroll
+            for (int r = 0; r < kPer; ++r) tot += zs_part[r * BN + et];
+            zs_s[et] = tot;
+          }
         }
       }
-      if (!fail && !mbar_wait(&tfull[buf], acc_phase, abort_flag)) {
+      if (!mbar_wait(&tfull[buf], acc_phase, abort_flag)) {
         fail = true;
         if (!*abort_flag && et == 0) note_timeout(a.status, 9, i, buf, static_cast<int>(acc_phase));
       }
-      if (fail) report(a.status, FQ_ERR_TIMEOUT);
       if (bar_red_or_dec(1, kEpi, fail || *abort_flag)) {
         if (et == 0) *abort_flag = 1;
         break;
@@ -485,109 +552,109 @@ __global__ void __launch_bounds__(kThreads, 1)
       tc_fence_after_sync();
       const uint32_t t_row = tmem_base + (static_cast<uint32_t>(quarter * 32) << 16) +
                              static_cast<uint32_t>(buf * BN);
-
-      // final values of this row for tokens c .. c + 15: store, and for the analysis the
-      // per-token sums over the tile's two 64-row blocks
-      auto finish = [&](int c, float (&v)[kChunk]) {
+      // this thread's row of the accumulator (for the core: gamma (s Q z + zero sum z) over the
+      // CTA's K range)
+      float vals[BN];
 #pragma unroll
-        for (int j = 0; j < kChunk; ++j) {
-          float val = v[j];
-          if (t.p == 1) val *= g_i;
-          const __nv_bfloat16 b = __float2bfloat16_rn(val);
-          if (row_ok && c + j < a.M) ph.out[static_cast<int64_t>(c + j) * ph.R + row] = b;
-          v[j] = row_ok ? __bfloat162float(b) : 0.f;
-        }
-        if (t.p == 0) {
-#pragma unroll
-          for (int j = 0; j < kChunk; ++j) {
-            float s = v[j];
-#pragma unroll
-            for (int off = 16; off > 0; off >>= 1) s += __shfl_xor_sync(0xffffffffu, s, off);
-            if (lane == 0) red[quarter * BN + c + j] = s;
-          }
-          named_barrier_sync(1, kEpi);
-          if (et < 2 * kChunk) {
-            const int blk = et / kChunk, tok = c + et % kChunk;
-            const float s = red[(2 * blk) * BN + tok] + red[(2 * blk + 1) * BN + tok];
-            const int gb = t.tile * 2 + blk;
-            if (gb < a.nblk && tok < a.M) a.zsum64[gb * a.M + tok] = s;
-          }
-          named_barrier_sync(1, kEpi);
-        }
-      };
-
-      if (ph.S == 1) {
-        float vals[BN];
-#pragma unroll
-        for (int c = 0; c < BN; c += kChunk) {
-          float v[kChunk];
+      for (int c = 0; c < BN; c += kChunk) {
+        float v[kChunk];
+        if (has_k) {
           tmem_ld16(t_row + c, v);
           tmem_wait_ld();
+        } else {
 #pragma unroll
-          for (int j = 0; j < kChunk; ++j)
-            vals[c + j] = t.p == 1 ? fmaf(s_i, v[j], z_i * zs_s[c + j]) : v[j];
+          for (int q = 0; q < kChunk; ++q) v[q] = 0.f;
         }
-        tc_fence_before_sync();
-        mbar_arrive(&tempty[buf]);
 #pragma unroll
-        for (int c = 0; c < BN; c += kChunk) {
-          float v[kChunk];
+        for (int q = 0; q < kChunk; ++q)
+          vals[c + q] = t.p == 1 ? g_row * fmaf(s_i, v[q], z_i * zs_s[c + q]) : v[q];
+      }
+      tc_fence_before_sync();
+      mbar_arrive(&tempty[buf]);
+
+      if (!clustered) {
+        // one CTA per task: this thread owns one row of the tile
 #pragma unroll
-          for (int j = 0; j < kChunk; ++j) v[j] = vals[c + j];
-          finish(c, v);
+        for (int c = 0; c < BN; ++c) {
+          const __nv_bfloat16 b = __float2bfloat16_rn(vals[c]);
+          if (row_ok && c < a.M) ph.out[static_cast<int64_t>(c) * ph.R + row] = b;
+          if (t.p == 0) {
+            // 16 consecutive rows = 16 consecutive lanes
+            float sv = row_ok ? __bfloat162float(b) : 0.f;
+#pragma unroll
+            for (int off = 8; off > 0; off >>= 1) sv += __shfl_xor_sync(0xffffffffu, sv, off);
+            const int grp = row / kGroup;
+            if ((lane & 15) == 0 && c < a.M && grp < a.ngroups) a.zsum[grp * a.M + c] = sv;
+          }
+        }
+        if (t.p < 2) {
+          named_barrier_sync(1, kEpi);
+          if (et == 0) st_release_gpu(&ph.flags[t.tile * kWsSlices], g);
         }
       } else {
-        float* part = ph.partial + static_cast<int64_t>(t.ks) * a.M * ph.R;
+        // ---- push this row into slot `ks` of the owning CTA's receive buffer
+        const int rb = j & 1;
+        float* recv = recv_buf + rb * (kBM * kRow);
+        const int slot_row = ks * rows_per + rl_own;
+        if (dest == ks) {
+          float4* dst = reinterpret_cast<float4*>(recv + slot_row * kRow);
 #pragma unroll
-        for (int c = 0; c < BN; c += kChunk) {
-          float v[kChunk];
-          tmem_ld16(t_row + c, v);
-          tmem_wait_ld();
+          for (int c4 = 0; c4 < BN / 4; ++c4)
+            dst[c4] = make_float4(vals[4 * c4], vals[4 * c4 + 1], vals[4 * c4 + 2], vals[4 * c4 + 3]);
+        } else {
+          const uint32_t rdst = mapa(smem_u32(recv + slot_row * kRow), static_cast<uint32_t>(dest));
+          const uint32_t rbar = mapa(smem_u32(&recv_bar[rb]), static_cast<uint32_t>(dest));
 #pragma unroll
-          for (int j = 0; j < kChunk; ++j) {
-            const float val = t.p == 1 ? fmaf(s_i, v[j], z_i * zs_s[c + j]) : v[j];
-            if (row_ok && c + j < a.M) part[static_cast<int64_t>(c + j) * ph.R + row] = val;
+          for (int c4 = 0; c4 < BN / 4; ++c4)
+            st_async_v4(rdst + 16 * c4, vals[4 * c4], vals[4 * c4 + 1], vals[4 * c4 + 2],
+                        vals[4 * c4 + 3], rbar);
+        }
+        // ---- the S - 1 peers' partials of this CTA's slice
+        const bool ok = mbar_wait(&recv_bar[rb], static_cast<uint32_t>(j >> 1) & 1u, abort_flag);
+        if (!ok && et == 0 && !*abort_flag) note_timeout(a.status, 11, i, j, 0);
+        if (bar_red_or_dec(1, kEpi, !ok)) {   // also orders this CTA's own slot writes
+          if (et == 0) *abort_flag = 1;
+          break;
+        }
+        // re-arm the buffer for this CTA's task after next; its peers write it only after
+        // this CTA has sent them the next task's partials, i.e. after the reads below
+        if (et == 0 && i + 2 * static_cast<int>(ncl) < a.total)
+          mbar_arrive_expect_tx(&recv_bar[rb], recv_bytes);
+        // ---- reduce the slice in rank order; item = (row of the slice, 4 tokens), so 16-row
+        // groups sit in 16 consecutive lanes (items per warp are all valid or all not)
+        const int items = rows_per * (BN / 4);
+        for (int w = et; w < items; w += kEpi) {
+          const int rl = w % rows_per, tg = w / rows_per;
+          float4 acc = *reinterpret_cast<const float4*>(recv + rl * kRow + 4 * tg);
+          for (int q = 1; q < S; ++q) {
+            const float4 v = *reinterpret_cast<const float4*>(recv + (q * rows_per + rl) * kRow + 4 * tg);
+            acc.x += v.x;
+            acc.y += v.y;
+            acc.z += v.z;
+            acc.w += v.w;
+          }
+          const int orow = t.tile * kBM + ks * rows_per + rl;
+          const bool ok_r = orow < ph.R;
+          const float o[4] = {acc.x, acc.y, acc.z, acc.w};
+#pragma unroll
+          for (int u = 0; u < 4; ++u) {
+            const int tok = 4 * tg + u;
+            const __nv_bfloat16 b = __float2bfloat16_rn(o[u]);
+            if (ok_r && tok < a.M) ph.out[static_cast<int64_t>(tok) * ph.R + orow] = b;
+            if (t.p == 0) {
+              float sv = ok_r ? __bfloat162float(b) : 0.f;
+#pragma unroll
+              for (int off = 8; off > 0; off >>= 1) sv += __shfl_xor_sync(0xffffffffu, sv, off);
+              const int grp = orow / kGroup;
+              if ((lane & 15) == 0 && tok < a.M && grp < a.ngroups) a.zsum[grp * a.M + tok] = sv;
+            }
           }
         }
-        tc_fence_before_sync();
-        mbar_arrive(&tempty[buf]);
-        __threadfence();
-        named_barrier_sync(1, kEpi);
-        if (et == 0) {
-          const unsigned old =
-              atomicInc(&ph.tickets[t.tile], static_cast<unsigned>(ph.S - 1));
-          *ticket_s = old == static_cast<unsigned>(ph.S - 1) ? 1 : 0;
+        if (t.p < 2) {
+          // the slice is stored: publish it
+          named_barrier_sync(1, kEpi);
+          if (et == 0) st_release_gpu(&ph.flags[t.tile * kWsSlices + ks], g);
         }
-        named_barrier_sync(1, kEpi);
-        if (*ticket_s == 0) {
-          if (++buf == 2) buf = 0, acc_phase ^= 1;
-          continue;                     // another CTA finishes this tile
-        }
-        __threadfence();
-#pragma unroll
-        for (int c = 0; c < BN; c += kChunk) {
-          float v[kChunk];
-#pragma unroll
-          for (int j = 0; j < kChunk; ++j) v[j] = 0.f;
-#pragma unroll 2
-          for (int q = 0; q < ph.S; ++q) {
-            const float* src = ph.partial + (static_cast<int64_t>(q) * a.M + c) * ph.R + row;
-            float w[kChunk];
-#pragma unroll
-            for (int j = 0; j < kChunk; ++j)
-              w[j] = (row_ok && c + j < a.M) ? ldcg_f32(src + static_cast<int64_t>(j) * ph.R)
-                                              : 0.f;
-#pragma unroll
-            for (int j = 0; j < kChunk; ++j) v[j] += w[j];
-          }
-          finish(c, v);
-        }
-      }
-      // the tile is final: publish it to dependent tasks
-      if (t.p < 2) {
-        __threadfence();
-        named_barrier_sync(1, kEpi);
-        if (et == 0) st_release_gpu(&ph.flags[t.tile], g);
       }
       if (++buf == 2) buf = 0, acc_phase ^= 1;
     }
@@ -598,8 +665,8 @@ __global__ void __launch_bounds__(kThreads, 1)
   if (threadIdx.x == 0) {
     // the last CTA to finish moves the workspace to the next call's generation
     __threadfence();
-    const unsigned old = atomicInc(a.done, static_cast<unsigned>(G - 1));
-    if (old == static_cast<unsigned>(G - 1)) {
+    const unsigned old = atomicInc(a.done, gridDim.x - 1);
+    if (old == gridDim.x - 1) {
       __threadfence();
       atomicAdd(a.gen, 1u);
     }
@@ -643,11 +710,10 @@ bool tmap_bf16(CUtensorMap* m, const void* base, int64_t rows, int64_t cols, int
 int decode_bn(int M) { return M <= 16 ? 16 : (M <= 32 ? 32 : 64); }
 
 struct DecWs {
-  size_t z, u, zsum, part[3], total;
+  size_t z, u, zsum, total;
 };
 
-DecWs dec_ws(int M, int d_in, int n_in, int n_out, int d_out) {
-  (void)d_in;
+DecWs dec_ws(int M, int n_in, int n_out) {
   DecWs L{};
   size_t off = kWsHeader;
   L.z = off;
@@ -655,12 +721,7 @@ DecWs dec_ws(int M, int d_in, int n_in, int n_out, int d_out) {
   L.u = off;
   off += round_up(static_cast<int64_t>(M) * n_out * 2, 256);
   L.zsum = off;
-  off += round_up(ceil_div(n_in, kBK) * M * 4, 256);
-  const int R[3] = {n_in, n_out, d_out};
-  for (int p = 0; p < 3; ++p) {
-    L.part[p] = off;
-    off += round_up(static_cast<int64_t>(kMaxSplit) * M * R[p] * 4, 256);
-  }
+  off += round_up(ceil_div(n_in, kGroup) * M * 4, 256);
   L.total = off;
   return L;
 }
@@ -678,40 +739,84 @@ cudaError_t prepare(int dev) {
   return e;
 }
 
-// K splits of one phase: the busiest CTA's K blocks plus a fixed cost per task (pipeline
-// fill, epilogue) and a small cost for a split's reduction, minimised over S.
-void plan(DecPhase& ph, int G) {
-  ph.RT = static_cast<int>(ceil_div(ph.R, kBM));
-  ph.KB = static_cast<int>(ceil_div(ph.K, kBK));
-  int best_s = 1;
-  double best = 1e30;
-  for (int s = 1; s <= std::min(kMaxSplit, ph.KB); ++s) {
-    const int kbs = static_cast<int>(ceil_div(ph.KB, s));
-    if (ceil_div(ph.KB, kbs) != s) continue;
-    const double per_cta = static_cast<double>(ceil_div(static_cast<int64_t>(ph.RT) * s, G));
-    const double cost = per_cta * (kbs + 3.0) + (s > 1 ? 2.0 : 0.0);
-    if (cost < best - 1e-9) best = cost, best_s = s;
+// Co-resident clusters of S CTAs of this kernel on the current device (0 if none).
+template <int BN>
+int max_clusters(int dev, int S) {
+  static std::mutex mu;
+  static std::map<std::pair<int, int>, int> cache;
+  std::lock_guard<std::mutex> g(mu);
+  const auto key = std::make_pair(dev, S);
+  const auto it = cache.find(key);
+  if (it != cache.end()) return it->second;
+  cudaLaunchConfig_t cfg{};
+  cfg.gridDim = dim3(static_cast<unsigned>(S * 64));
+  cfg.blockDim = dim3(kThreads);
+  cfg.dynamicSmemBytes = DecLayout<BN>::kBytes;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = static_cast<unsigned>(S);
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  int n = 0;
+  if (cudaOccupancyMaxActiveClusters(&n, decode_layer_kernel<BN>, &cfg) != cudaSuccess) {
+    cudaGetLastError();
+    n = 0;
   }
-  ph.S = best_s;
-  ph.kbs = static_cast<int>(ceil_div(ph.KB, best_s));
-  ph.tasks = ph.RT * ph.S;
+  cache[key] = n;
+  return n;
 }
 
 template <int BN>
-fq_status run(const CUtensorMap* m, DecArgs& a, int G, cudaStream_t s) {
+fq_status run(const CUtensorMap* m, DecArgs& a, const int* R, const int* K, int sms,
+              cudaStream_t s) {
   int dev = 0;
   cudaGetDevice(&dev);
   if (prepare<BN>(dev) != cudaSuccess) return FQ_ERR_CUDA;
+  // Cluster size: the busiest cluster's K blocks over the three phases, with a fixed cost per
+  // task (pipeline fill and drain, reduction), code blocks weighted by their smaller bytes.
+  int best_s = 1, best_ncl = 0;
+  double best = 1e30;
+  for (int S : {1, 2, 4, 8}) {
+    const int ncl = S == 1 ? sms : max_clusters<BN>(dev, S);
+    if (ncl <= 0) continue;
+    double cost = 0;
+    for (int p = 0; p < 3; ++p) {
+      const int RT = static_cast<int>(ceil_div(R[p], kBM));
+      const int KB = static_cast<int>(ceil_div(K[p], kBK));
+      const double w = p == 1 ? 0.35 : 1.0;
+      cost += static_cast<double>(ceil_div(RT, ncl)) * (w * ceil_div(KB, S) + 4.0);
+    }
+    if (cost < best - 1e-9) best = cost, best_s = S, best_ncl = ncl;
+  }
+  a.S = best_s;
+  int base = 0;
+  for (int p = 0; p < 3; ++p) {
+    DecPhase& ph = a.ph[p];
+    ph.RT = static_cast<int>(ceil_div(R[p], kBM));
+    if (ph.RT > kWsMaxTiles) return FQ_ERR_UNSUPPORTED;
+    ph.KB = static_cast<int>(ceil_div(K[p], kBK));
+    ph.kbs = static_cast<int>(ceil_div(ph.KB, best_s));
+    ph.base = base;
+    base += ph.RT;
+  }
+  a.total = base;
+  const int ncl = std::min(best_ncl, a.total);
   cudaLaunchConfig_t cfg{};
-  cfg.gridDim = dim3(static_cast<unsigned>(G));
+  cfg.gridDim = dim3(static_cast<unsigned>(ncl * best_s));
   cfg.blockDim = dim3(kThreads);
   cfg.dynamicSmemBytes = DecLayout<BN>::kBytes;
   cfg.stream = s;
-  cudaLaunchAttribute attr[1];
+  cudaLaunchAttribute attr[2];
   attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
   attr[0].val.programmaticStreamSerializationAllowed = 1;
+  attr[1].id = cudaLaunchAttributeClusterDimension;
+  attr[1].val.clusterDim.x = static_cast<unsigned>(best_s);
+  attr[1].val.clusterDim.y = 1;
+  attr[1].val.clusterDim.z = 1;
   cfg.attrs = attr;
-  cfg.numAttrs = 1;
+  cfg.numAttrs = best_s > 1 ? 2 : 1;
   return cudaLaunchKernelEx(&cfg, decode_layer_kernel<BN>, m[0], m[1], m[2], m[3], m[4], a) ==
                  cudaSuccess
              ? FQ_OK
@@ -721,7 +826,9 @@ fq_status run(const CUtensorMap* m, DecArgs& a, int G, cudaStream_t s) {
 }  // namespace
 
 size_t decode_workspace_bytes(int M, int d_in, int n_in, int n_out, int d_out) {
-  return dec_ws(M, d_in, n_in, n_out, d_out).total;
+  (void)d_in;
+  (void)d_out;
+  return dec_ws(M, n_in, n_out).total;
 }
 
 fq_status launch_decode_forward(const void* x, int M, int d_in, const void* T_in,
@@ -729,7 +836,7 @@ fq_status launch_decode_forward(const void* x, int M, int d_in, const void* T_in
                                 const float* gamma, void* y, char* ws, size_t ws_bytes,
                                 cudaStream_t s) {
   const int n_in = Cq.n_in, n_out = Cq.n_out;
-  const DecWs L = dec_ws(M, d_in, n_in, n_out, d_out);
+  const DecWs L = dec_ws(M, n_in, n_out);
   if (ws_bytes < L.total) return FQ_ERR_WORKSPACE;
   const int BN = decode_bn(M);
   int dev = 0, sms = 0;
@@ -742,27 +849,18 @@ fq_status launch_decode_forward(const void* x, int M, int d_in, const void* T_in
   const int R[3] = {n_in, n_out, d_out};
   const int K[3] = {d_in, n_in, n_out};
   void* outs[3] = {ws + L.z, ws + L.u, y};
-  int base = 0;
   for (int p = 0; p < 3; ++p) {
-    DecPhase& ph = a.ph[p];
-    ph.R = R[p];
-    ph.K = K[p];
-    plan(ph, sms);
-    if (ph.RT > kWsMaxTiles) return FQ_ERR_UNSUPPORTED;
-    ph.base = base;
-    base += ph.tasks;
-    ph.out = static_cast<__nv_bfloat16*>(outs[p]);
-    ph.partial = reinterpret_cast<float*>(ws + L.part[p]);
-    ph.flags = reinterpret_cast<uint32_t*>(ws + kWsFlags) + p * kWsMaxTiles;
-    ph.tickets = reinterpret_cast<uint32_t*>(ws + kWsTickets) + p * kWsMaxTiles;
+    a.ph[p].R = R[p];
+    a.ph[p].K = K[p];
+    a.ph[p].out = static_cast<__nv_bfloat16*>(outs[p]);
+    a.ph[p].flags = reinterpret_cast<uint32_t*>(ws + kWsFlags) + p * kWsMaxTiles * kWsSlices;
   }
-  a.total = base;
   a.words = Cq.words;
   a.scale = reinterpret_cast<const __half*>(Cq.scale);
   a.zero = reinterpret_cast<const __half*>(Cq.zero);
   a.gamma = gamma;
-  a.zsum64 = reinterpret_cast<float*>(ws + L.zsum);
-  a.nblk = static_cast<int>(ceil_div(n_in, kBK));
+  a.zsum = reinterpret_cast<float*>(ws + L.zsum);
+  a.ngroups = static_cast<int>(ceil_div(n_in, kGroup));
   a.status = reinterpret_cast<int32_t*>(ws);
   a.gen = reinterpret_cast<uint32_t*>(ws + kWsGen);
   a.done = reinterpret_cast<uint32_t*>(ws + kWsDone);
@@ -776,11 +874,10 @@ fq_status launch_decode_forward(const void* x, int M, int d_in, const void* T_in
       !tmap_bf16(&m[2], ws + L.z, M, n_in, BN) ||
       !tmap_bf16(&m[3], T_out_t, d_out, n_out, kBM) || !tmap_bf16(&m[4], ws + L.u, M, n_out, BN))
     return FQ_ERR_CUDA;
-  const int G = std::min(sms, a.total);
   switch (BN) {
-    case 16: return run<16>(m, a, G, s);
-    case 32: return run<32>(m, a, G, s);
-    default: return run<64>(m, a, G, s);
+    case 16: return run<16>(m, a, R, K, sms, s);
+    case 32: return run<32>(m, a, R, K, sms, s);
+    default: return run<64>(m, a, R, K, sms, s);
   }
 }
 

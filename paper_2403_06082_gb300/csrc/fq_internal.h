@@ -17,15 +17,16 @@ inline int64_t round_up(int64_t a, int64_t b) { return ceil_div(a, b) * b; }
 
 // Workspace header (64 KiB, at fixed offsets whatever the layer's sizes, so that one workspace
 // can serve layers of different shapes): [0] device status word, [4] generation counter,
-// [8] end-of-call ticket, [1024] ready flags and [kWsTickets] split tickets of up to
-// kWsMaxTiles row tiles per phase.  A zero-filled header is a valid initial state and every
-// completed call leaves it valid for the next one.
+// [8] end-of-call ticket, [kWsFlags] ready flags, kWsSlices per row tile of up to kWsMaxTiles
+// row tiles per phase.  A zero-filled header is a valid initial state and every completed call
+// leaves it valid for the next one.
 constexpr size_t kWsHeader = 64 * 1024;
 constexpr size_t kWsGen = 4;
 constexpr size_t kWsDone = 8;
-constexpr int kWsMaxTiles = 2048;
 constexpr size_t kWsFlags = 1024;
-constexpr size_t kWsTickets = kWsFlags + 3 * kWsMaxTiles * 4;
+constexpr int kWsSlices = 8;
+constexpr int kWsMaxTiles = 640;
+static_assert(kWsFlags + 3 * kWsMaxTiles * kWsSlices * 4 <= kWsHeader, "flags fit the header");
 constexpr int kDecodeMaxM = 64;   // batches up to this size take the fused decode kernel
 
 // ---- fq_api.cu
