@@ -541,9 +541,10 @@ __global__ void __launch_bounds__(kThreads, 1)
           }
         }
       }
-      if (!mbar_wait(&tfull[buf], acc_phase, abort_flag)) {
+      // one thread waits, the others block in the named barrier below
+      if (et == 0 && !mbar_wait(&tfull[buf], acc_phase, abort_flag)) {
         fail = true;
-        if (!*abort_flag && et == 0) note_timeout(a.status, 9, i, buf, static_cast<int>(acc_phase));
+        if (!*abort_flag) note_timeout(a.status, 9, i, buf, static_cast<int>(acc_phase));
       }
       if (bar_red_or_dec(1, kEpi, fail || *abort_flag)) {
         if (et == 0) *abort_flag = 1;
@@ -610,8 +611,11 @@ __global__ void __launch_bounds__(kThreads, 1)
                         vals[4 * c4 + 3], rbar);
         }
         // ---- the S - 1 peers' partials of this CTA's slice
-        const bool ok = mbar_wait(&recv_bar[rb], static_cast<uint32_t>(j >> 1) & 1u, abort_flag);
-        if (!ok && et == 0 && !*abort_flag) note_timeout(a.status, 11, i, j, 0);
+        bool ok = true;
+        if (et == 0) {
+          ok = mbar_wait(&recv_bar[rb], static_cast<uint32_t>(j >> 1) & 1u, abort_flag);
+          if (!ok && !*abort_flag) note_timeout(a.status, 11, i, j, 0);
+        }
         if (bar_red_or_dec(1, kEpi, !ok)) {   // also orders this CTA's own slot writes
           if (et == 0) *abort_flag = 1;
           break;
@@ -662,6 +666,9 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   tc_fence_before_sync();
   __syncthreads();
+  // No CTA leaves while a peer may still write into its shared memory (after a wait that gave
+  // up, the exchange can be cut short); every wait above is bounded, so all CTAs get here.
+  if (clustered) cluster_sync();
   if (threadIdx.x == 0) {
     // the last CTA to finish moves the workspace to the next call's generation
     __threadfence();
