@@ -56,7 +56,7 @@ static_assert(kMaxSplit <= kWsSlices, "one ready flag per slice");
 constexpr int kEpi = 128;
 constexpr int kChunk = 16;
 constexpr int kGroup = 16;                 // columns of z per partial sum
-constexpr int kThreads = 352;
+constexpr int kThreads = 384;
 constexpr int64_t kL2PrefetchBudget = 64ll << 20;
 
 struct DecPhase {
@@ -338,44 +338,64 @@ __global__ void __launch_bounds__(kThreads, 1)
       const DecPhase ph = phase_of(a, t.p);
       int k0, k1;
       krange(ph, k0, k1);
-      if (t.p > 0 && k1 > k0) {
-        // every slice of the previous phase's output that this CTA's K range reads must be final
-        const DecPhase src = phase_of(a, t.p - 1);
-        const int sl0 = (k0 * kBK) / rows_per, sl1 = (min(ph.K, k1 * kBK) - 1) / rows_per;
-        bool ok = true;
-        int bad = sl0;
-        for (int gs = sl0 + lane; gs <= sl1 && ok; gs += 32) {
-          ok = wait_flag(&src.flags[(gs / S) * kWsSlices + gs % S], g, abort_flag);
-          if (!ok) bad = gs;
-        }
-        const unsigned fails = __ballot_sync(0xffffffffu, !ok);
-        if (fails) {
-          if (lane == __ffs(fails) - 1 && !*abort_flag) {
-            const uint32_t* f = &src.flags[(bad / S) * kWsSlices + bad % S];
-            note_timeout(a.status, 2, i, bad, static_cast<int>(ld_acquire_gpu(f) - g) * 1000 + t.p);
-          }
-          __syncwarp();
-          if (lane == 0) *abort_flag = 1;
-          break;
-        }
-      }
+      // Loads go out in K order as soon as the slices of the previous phase's output that a K
+      // block reads are final: the lanes poll the not-yet-final slices of the K range, and
+      // the ready prefix decides how far lane 0 may issue.
+      const DecPhase src = phase_of(a, t.p > 0 ? t.p - 1 : 0);
+      const int sl1 = k1 > k0 ? (min(ph.K, k1 * kBK) - 1) / rows_per : 0;
+      int ready = k1 > k0 ? (k0 * kBK) / rows_per : 0;   // slices below `ready` are final
+      const long long t_start = clock64();
       bool ok = true;
-      if (lane == 0) {
-        const CUtensorMap* tm = t.p == 0 ? &tmX : (t.p == 1 ? &tmZ : &tmU);
-        for (int kb = k0; kb < k1; ++kb) {
-          if (!mbar_wait(&empty[stage], phase ^ 1, abort_flag)) {
-            if (!*abort_flag) note_timeout(a.status, 3, i, stage, static_cast<int>(phase));
-            ok = false;
-            break;
+      int kb = k0;
+      const CUtensorMap* tm = t.p == 0 ? &tmX : (t.p == 1 ? &tmZ : &tmU);
+      while (kb < k1 && ok) {
+        int kb_end = k1;
+        if (t.p > 0 && ready <= sl1) {
+          // first slice (from `ready`) that is not final yet, over the whole warp
+          int first_missing = sl1 + 1;
+          for (int gs = ready + lane; gs <= sl1; gs += 32)
+            if (ld_acquire_gpu(&src.flags[(gs / S) * kWsSlices + gs % S]) != g) {
+              first_missing = gs;
+              break;
+            }
+#pragma unroll
+          for (int off = 16; off > 0; off >>= 1)
+            first_missing = min(first_missing, __shfl_xor_sync(0xffffffffu, first_missing, off));
+          ready = first_missing;
+          // K blocks whose rows all lie below the first missing slice
+          kb_end = ready > sl1 ? k1 : min(k1, (ready * rows_per) / kBK);
+          if (kb_end <= kb) {
+            if (clock64() - t_start > kWaitLimitCycles || *abort_flag) {
+              if (lane == 0 && !*abort_flag) {
+                const uint32_t* f = &src.flags[(ready / S) * kWsSlices + ready % S];
+                note_timeout(a.status, 2, i, ready, static_cast<int>(ld_acquire_gpu(f) - g) * 1000 + t.p);
+              }
+              ok = false;
+              break;
+            }
+            __nanosleep(64);
+            continue;
           }
-          mbar_arrive_expect_tx(&fullB[stage], kBTile);
-          tma_load_2d(sB + stage * kBTile, tm, &fullB[stage], kb * kBK, 0, pol_x);
-          used[stage] = true;
-          last_par[stage] = phase;
-          if (++stage == S_) stage = 0, phase ^= 1;
         }
-        if (!ok) *abort_flag = 1;
+        if (lane == 0) {
+          for (; kb < kb_end; ++kb) {
+            if (!mbar_wait(&empty[stage], phase ^ 1, abort_flag)) {
+              if (!*abort_flag) note_timeout(a.status, 3, i, stage, static_cast<int>(phase));
+              ok = false;
+              break;
+            }
+            mbar_arrive_expect_tx(&fullB[stage], kBTile);
+            tma_load_2d(sB + stage * kBTile, tm, &fullB[stage], kb * kBK, 0, pol_x);
+            used[stage] = true;
+            last_par[stage] = phase;
+            if (++stage == S_) stage = 0, phase ^= 1;
+          }
+        }
+        ok = __shfl_sync(0xffffffffu, ok, 0);
+        kb = __shfl_sync(0xffffffffu, kb, 0);
+        // stage / phase / used / last_par live in lane 0 only
       }
+      if (!ok && lane == 0) *abort_flag = 1;
       if (!__shfl_sync(0xffffffffu, ok, 0)) break;
     }
     if (lane == 0)
@@ -440,9 +460,9 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (!mbar_wait(mma_done, 0, nullptr)) report(a.status, FQ_ERR_TIMEOUT);
       }
     }
-  } else if (warp >= 7) {
+  } else if (warp >= 7 && warp != 9) {
     // -------------------------------------------------------------- code decoders
-    const int dw = warp - 7;
+    const int dw = warp <= 8 ? warp - 7 : warp - 8;   // warps 7, 8, 10, 11
     int stage = 0;
     uint32_t phase = 0;
     int it = 0;
@@ -476,7 +496,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       report(a.status, FQ_ERR_TIMEOUT);
       *abort_flag = 1;
     }
-  } else {
+  } else if (warp >= 2 && warp <= 5) {
     // -------------------------------------------------------------- epilogue (warps 2-5)
     const int quarter = warp & 3;                 // TMEM lanes 32 * quarter .. + 31
     const int r_in_tile = quarter * 32 + lane;
