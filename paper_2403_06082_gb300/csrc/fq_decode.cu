@@ -13,10 +13,11 @@
 // CTA adds the S partials of its slice in rank order (deterministic; no global partials, no
 // atomics, no remote arrivals).  Receive buffers alternate between consecutive tasks; a buffer
 // is only written again after its owner has sent the next task's partials, which it does only
-// after reading the buffer, so no back-pressure signal is needed.  Cluster c runs tasks c,
-// c + C, ... in order; task indices grow with the phase, so every cluster finishes its
-// analysis tasks before its core tasks and those before its synthesis tasks, and no cluster
-// waits on work queued behind a wait.  Each CTA stamps the ready flag of its slice with this
+// after reading the buffer, so no back-pressure signal is needed.  Each cluster runs its own
+// list of tasks, in phase order (so no cluster waits on work queued behind a wait); the
+// lists are built on the host (tiles dealt round-robin, each phase's tiles ordered by where
+// they fall in the next phase's K splits, so that every consumer's first K blocks are
+// produced first).  Each CTA stamps the ready flag of its slice with this
 // call's generation (release) once the slice is stored, and the activation producer of a
 // dependent task waits for exactly the slices its K range reads (acquire, bounded, one lane
 // per flag).  No phase waits for the whole grid, and the weight producer runs ahead into the
@@ -37,9 +38,11 @@
 #include <cudaTypedefs.h>
 
 #include <algorithm>
+#include <array>
 #include <map>
 #include <mutex>
 #include <utility>
+#include <vector>
 
 #include "fq_device.cuh"
 #include "fq_internal.h"
@@ -60,7 +63,7 @@ constexpr int kThreads = 384;
 constexpr int64_t kL2PrefetchBudget = 64ll << 20;
 
 struct DecPhase {
-  int R, K, RT, KB, kbs, base;
+  int R, K, RT, KB, kbs;
   __nv_bfloat16* out;     // [M][R]
   uint32_t* flags;        // [RT][kWsSlices] slice final in this call when == generation + 1
 };
@@ -78,6 +81,14 @@ struct DecArgs {
   uint32_t* gen;
   uint32_t* done;
   int prefetch_later;     // 0: none, 1: codes, 2: codes and T_out^T tiles
+};
+
+// Per-cluster task lists, a kernel parameter: cluster c runs task[off[c]] .. task[off[c+1]-1].
+constexpr int kMaxClusters = 160;
+constexpr int kMaxSched = 3 * kWsMaxTiles;
+struct DecSched {
+  uint16_t off[kMaxClusters + 1];
+  uint16_t task[kMaxSched];          // phase << 14 | row tile
 };
 
 template <int BN>
@@ -110,9 +121,9 @@ __device__ __forceinline__ DecPhase phase_of(const DecArgs& a, int p) {
   return p == 0 ? a.ph[0] : (p == 1 ? a.ph[1] : a.ph[2]);
 }
 
-__device__ __forceinline__ Task task_of(const DecArgs& a, int i) {
-  const int p = (i >= a.ph[1].base) + (i >= a.ph[2].base);
-  return {p, i - phase_of(a, p).base};
+__device__ __forceinline__ Task task_at(const DecSched& sc, int ti) {
+  const uint32_t e = sc.task[ti];
+  return {static_cast<int>(e >> 14), static_cast<int>(e & 0x3FFFu)};
 }
 
 // q -> bf16(128 + q) - 128 (exact), one 128-byte row of a K-major tile with the 128-byte
@@ -171,7 +182,8 @@ __global__ void __launch_bounds__(kThreads, 1)
                         const __grid_constant__ CUtensorMap tmX,
                         const __grid_constant__ CUtensorMap tmZ,
                         const __grid_constant__ CUtensorMap tmTout,
-                        const __grid_constant__ CUtensorMap tmU, const DecArgs a) {
+                        const __grid_constant__ CUtensorMap tmU, const DecArgs a,
+                        const __grid_constant__ DecSched sched) {
   using Lo = DecLayout<BN>;
   constexpr int S_ = Lo::kStages;
   constexpr int kBTile = Lo::kBTile;
@@ -209,6 +221,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     ncl = cluster_count_x();
   }
   const int ks = static_cast<int>(rank);
+  const int t_lo = sched.off[cid], t_hi = sched.off[cid + 1];   // this cluster's tasks
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < S_; ++s) {
@@ -230,7 +243,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       // arm the receive buffers for this CTA's first two tasks (later tasks re-arm them)
       const uint32_t bytes = static_cast<uint32_t>((S - 1) * (kBM / S) * BN * 4);
       for (int b = 0; b < 2; ++b)
-        if (static_cast<int>(cid) + b * static_cast<int>(ncl) < a.total)
+        if (t_lo + b < t_hi)
           mbar_arrive_expect_tx(&recv_bar[b], bytes);
     }
     prefetch_tmap(&tmTin);
@@ -264,8 +277,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       bool used[S_];
 #pragma unroll
       for (int s = 0; s < S_; ++s) last_par[s] = 0, used[s] = false;
-      for (int i = static_cast<int>(cid); i < a.total && !*abort_flag; i += static_cast<int>(ncl)) {
-        const Task t = task_of(a, i);
+      for (int i = t_lo; i < t_hi && !*abort_flag; ++i) {
+        const Task t = task_at(sched, i);
         const DecPhase ph = phase_of(a, t.p);
         int k0, k1;
         krange(ph, k0, k1);
@@ -292,9 +305,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (first) {
           first = false;
           // warm L2 with the weight tiles of this CTA's later tasks
-          for (int j = i + static_cast<int>(ncl); j < a.total && a.prefetch_later > 0;
-               j += static_cast<int>(ncl)) {
-            const Task u = task_of(a, j);
+          for (int j = i + 1; j < t_hi && a.prefetch_later > 0; ++j) {
+            const Task u = task_at(sched, j);
             const DecPhase q = phase_of(a, u.p);
             int u0, u1;
             krange(q, u0, u1);
@@ -332,9 +344,9 @@ __global__ void __launch_bounds__(kThreads, 1)
     bool used[S_];
 #pragma unroll
     for (int s = 0; s < S_; ++s) last_par[s] = 0, used[s] = false;
-    for (int i = static_cast<int>(cid); i < a.total; i += static_cast<int>(ncl)) {
+    for (int i = t_lo; i < t_hi; ++i) {
       if (__shfl_sync(0xffffffffu, *abort_flag != 0, 0)) break;   // warp-uniform
-      const Task t = task_of(a, i);
+      const Task t = task_at(sched, i);
       const DecPhase ph = phase_of(a, t.p);
       int k0, k1;
       krange(ph, k0, k1);
@@ -412,8 +424,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       uint32_t acc_phase = 0;
       uint32_t apar = 0;     // bit s: parity of the next aready[s] phase
       bool issued_any = false;
-      for (int i = static_cast<int>(cid); i < a.total && !*abort_flag; i += static_cast<int>(ncl)) {
-        const Task t = task_of(a, i);
+      for (int i = t_lo; i < t_hi && !*abort_flag; ++i) {
+        const Task t = task_at(sched, i);
         const DecPhase ph = phase_of(a, t.p);
         int k0, k1;
         krange(ph, k0, k1);
@@ -467,8 +479,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     uint32_t phase = 0;
     int it = 0;
     bool ok = true;
-    for (int i = static_cast<int>(cid); i < a.total && ok && !*abort_flag; i += static_cast<int>(ncl)) {
-      const Task t = task_of(a, i);
+    for (int i = t_lo; i < t_hi && ok && !*abort_flag; ++i) {
+      const Task t = task_at(sched, i);
       const DecPhase ph = phase_of(a, t.p);
       int k0, k1;
       krange(ph, k0, k1);
@@ -513,8 +525,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     int buf = 0;
     uint32_t acc_phase = 0;
     int j = 0;                                    // tasks finished by this CTA
-    for (int i = static_cast<int>(cid); i < a.total; i += static_cast<int>(ncl), ++j) {
-      const Task t = task_of(a, i);
+    for (int i = t_lo; i < t_hi; ++i, ++j) {
+      const Task t = task_at(sched, i);
       const DecPhase ph = phase_of(a, t.p);
       int k0, k1;
       krange(ph, k0, k1);
@@ -642,7 +654,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         // re-arm the buffer for this CTA's task after next; its peers write it only after
         // this CTA has sent them the next task's partials, i.e. after the reads below
-        if (et == 0 && i + 2 * static_cast<int>(ncl) < a.total)
+        if (et == 0 && i + 2 < t_hi)
           mbar_arrive_expect_tx(&recv_bar[rb], recv_bytes);
         // ---- reduce the slice in rank order; item = (row of the slice, 4 tokens), so 16-row
         // groups sit in 16 consecutive lanes (items per warp are all valid or all not)
@@ -795,18 +807,63 @@ int max_clusters(int dev, int S) {
   return n;
 }
 
+// Task lists for `ncl` clusters of S CTAs: the three phases' tiles, concatenated in phase order,
+// dealt round-robin (each phase spreads evenly and starts on the clusters the previous one
+// left least busy).  Within the analysis and the core phase, tiles are ordered by their offset
+// inside the next phase's K splits, so that every split of the next phase finds its first K
+// blocks among the first tiles produced.
+void build_schedule(const int* R, const int* K, int S, int ncl, DecSched* out) {
+  int RT[3], kbs[3];
+  for (int p = 0; p < 3; ++p) {
+    RT[p] = static_cast<int>(ceil_div(R[p], kBM));
+    kbs[p] = static_cast<int>(ceil_div(ceil_div(K[p], kBK), S));
+  }
+  std::vector<std::vector<uint16_t>> lists(ncl);
+  std::vector<int> order;
+  int pos = 0;
+  for (int p = 0; p < 3; ++p) {
+    order.resize(RT[p]);
+    for (int t = 0; t < RT[p]; ++t) order[t] = t;
+    if (p < 2) {
+      const int64_t split_rows = static_cast<int64_t>(kbs[p + 1]) * kBK;
+      std::stable_sort(order.begin(), order.end(), [&](int x, int y) {
+        return (static_cast<int64_t>(x) * kBM) % split_rows <
+               (static_cast<int64_t>(y) * kBM) % split_rows;
+      });
+    }
+    for (int t : order) lists[pos++ % ncl].push_back(static_cast<uint16_t>((p << 14) | t));
+  }
+  int n = 0;
+  for (int c = 0; c < ncl; ++c) {
+    out->off[c] = static_cast<uint16_t>(n);
+    for (uint16_t e : lists[c]) out->task[n++] = e;
+  }
+  out->off[ncl] = static_cast<uint16_t>(n);
+}
+
+struct Plan {
+  int S = 0, ncl = 0;
+  DecSched sched{};
+};
+
+// Cluster size and task lists for a layer shape, cached.  Cluster size: the busiest cluster's
+// K blocks over the three phases, with a fixed cost per task (pipeline fill and drain,
+// reduction) and code blocks weighted by their smaller bytes.
 template <int BN>
-fq_status run(const CUtensorMap* m, DecArgs& a, const int* R, const int* K, int sms,
-              cudaStream_t s) {
-  int dev = 0;
-  cudaGetDevice(&dev);
-  if (prepare<BN>(dev) != cudaSuccess) return FQ_ERR_CUDA;
-  // Cluster size: the busiest cluster's K blocks over the three phases, with a fixed cost per
-  // task (pipeline fill and drain, reduction), code blocks weighted by their smaller bytes.
-  int best_s = 1, best_ncl = 0;
-  double best = 1e30;
+const Plan* plan_for(int dev, int sms, const int* R, const int* K) {
+  static std::mutex mu;
+  static std::map<std::array<int, 7>, Plan> cache;
+  const std::array<int, 7> key{dev, R[0], R[1], R[2], K[0], K[1], K[2]};
+  std::lock_guard<std::mutex> g(mu);
+  const auto it = cache.find(key);
+  if (it != cache.end()) return &it->second;
+  int total = 0;
+  for (int p = 0; p < 3; ++p) total += static_cast<int>(ceil_div(R[p], kBM));
+  Plan best;
+  double best_cost = 1e30;
   for (int S : {1, 2, 4, 8}) {
-    const int ncl = S == 1 ? sms : max_clusters<BN>(dev, S);
+    int ncl = S == 1 ? sms : max_clusters<BN>(dev, S);
+    ncl = std::min({ncl, total, kMaxClusters});
     if (ncl <= 0) continue;
     double cost = 0;
     for (int p = 0; p < 3; ++p) {
@@ -815,23 +872,42 @@ fq_status run(const CUtensorMap* m, DecArgs& a, const int* R, const int* K, int 
       const double w = p == 1 ? 0.35 : 1.0;
       cost += static_cast<double>(ceil_div(RT, ncl)) * (w * ceil_div(KB, S) + 4.0);
     }
-    if (cost < best - 1e-9) best = cost, best_s = S, best_ncl = ncl;
+    if (cost < best_cost - 1e-9) {
+      best_cost = cost;
+      best.S = S;
+      best.ncl = ncl;
+    }
   }
-  a.S = best_s;
-  int base = 0;
+  if (best.S == 0) return nullptr;
+  build_schedule(R, K, best.S, best.ncl, &best.sched);
+  return &(cache[key] = best);
+}
+
+template <int BN>
+fq_status run(const CUtensorMap* m, DecArgs& a, const int* R, const int* K, int sms,
+              cudaStream_t s) {
+  int dev = 0;
+  cudaGetDevice(&dev);
+  if (prepare<BN>(dev) != cudaSuccess) return FQ_ERR_CUDA;
+  int total = 0;
+  for (int p = 0; p < 3; ++p) {
+    const int RT = static_cast<int>(ceil_div(R[p], kBM));
+    if (RT > kWsMaxTiles || RT > 0x3FFF) return FQ_ERR_UNSUPPORTED;
+    total += RT;
+  }
+  if (total > kMaxSched) return FQ_ERR_UNSUPPORTED;
+  const Plan* plan = plan_for<BN>(dev, sms, R, K);
+  if (!plan) return FQ_ERR_CUDA;
+  a.S = plan->S;
   for (int p = 0; p < 3; ++p) {
     DecPhase& ph = a.ph[p];
     ph.RT = static_cast<int>(ceil_div(R[p], kBM));
-    if (ph.RT > kWsMaxTiles) return FQ_ERR_UNSUPPORTED;
     ph.KB = static_cast<int>(ceil_div(K[p], kBK));
-    ph.kbs = static_cast<int>(ceil_div(ph.KB, best_s));
-    ph.base = base;
-    base += ph.RT;
+    ph.kbs = static_cast<int>(ceil_div(ph.KB, plan->S));
   }
-  a.total = base;
-  const int ncl = std::min(best_ncl, a.total);
+  a.total = total;
   cudaLaunchConfig_t cfg{};
-  cfg.gridDim = dim3(static_cast<unsigned>(ncl * best_s));
+  cfg.gridDim = dim3(static_cast<unsigned>(plan->ncl * plan->S));
   cfg.blockDim = dim3(kThreads);
   cfg.dynamicSmemBytes = DecLayout<BN>::kBytes;
   cfg.stream = s;
@@ -839,13 +915,13 @@ fq_status run(const CUtensorMap* m, DecArgs& a, const int* R, const int* K, int 
   attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
   attr[0].val.programmaticStreamSerializationAllowed = 1;
   attr[1].id = cudaLaunchAttributeClusterDimension;
-  attr[1].val.clusterDim.x = static_cast<unsigned>(best_s);
+  attr[1].val.clusterDim.x = static_cast<unsigned>(plan->S);
   attr[1].val.clusterDim.y = 1;
   attr[1].val.clusterDim.z = 1;
   cfg.attrs = attr;
-  cfg.numAttrs = best_s > 1 ? 2 : 1;
-  return cudaLaunchKernelEx(&cfg, decode_layer_kernel<BN>, m[0], m[1], m[2], m[3], m[4], a) ==
-                 cudaSuccess
+  cfg.numAttrs = plan->S > 1 ? 2 : 1;
+  return cudaLaunchKernelEx(&cfg, decode_layer_kernel<BN>, m[0], m[1], m[2], m[3], m[4], a,
+                            plan->sched) == cudaSuccess
              ? FQ_OK
              : FQ_ERR_CUDA;
 }
