@@ -223,39 +223,38 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int ks = static_cast<int>(rank);
   const int t_lo = sched.off[cid], t_hi = sched.off[cid + 1];   // this cluster's tasks
 
-  if (threadIdx.x == 0) {
-    for (int s = 0; s < S_; ++s) {
-      mbar_init(&fullA[s], 1);
-      mbar_init(&fullB[s], 1);
-      mbar_init(&empty[s], 1);
-      mbar_init(&aready[s], 32);
+  if (warp == 0) {
+    // the barriers, initialised lane-parallel: fullA, fullB, empty (count 1), aready (32),
+    // tfull[2] (1), tempty[2] (kEpi), mma_done (1), recv_bar[2] (1)
+    for (int b = lane; b < Lo::kBars; b += 32) {
+      const int r = b - 4 * S_;
+      const uint32_t cnt = b < 3 * S_ ? 1u : (b < 4 * S_ ? 32u : ((r == 2 || r == 3) ? kEpi : 1u));
+      mbar_init(&fullA[b], cnt);
     }
-    for (int b = 0; b < 2; ++b) {
-      mbar_init(&tfull[b], 1);
-      mbar_init(&tempty[b], kEpi);
-    }
-    mbar_init(mma_done, 1);
-    mbar_init(&recv_bar[0], 1);
-    mbar_init(&recv_bar[1], 1);
-    *abort_flag = 0;
     fence_barrier_init();
-    if (clustered) {
-      // arm the receive buffers for this CTA's first two tasks (later tasks re-arm them)
-      const uint32_t bytes = static_cast<uint32_t>((S - 1) * (kBM / S) * BN * 4);
-      for (int b = 0; b < 2; ++b)
-        if (t_lo + b < t_hi)
-          mbar_arrive_expect_tx(&recv_bar[b], bytes);
+    __syncwarp();
+    if (lane == 0) {
+      *abort_flag = 0;
+      if (clustered) {
+        // arm the receive buffers for this CTA's first two tasks (later tasks re-arm them)
+        const uint32_t bytes = static_cast<uint32_t>((S - 1) * (kBM / S) * BN * 4);
+        for (int b = 0; b < 2; ++b)
+          if (t_lo + b < t_hi) mbar_arrive_expect_tx(&recv_bar[b], bytes);
+      }
+      prefetch_tmap(&tmTin);
+      prefetch_tmap(&tmX);
+      prefetch_tmap(&tmZ);
+      prefetch_tmap(&tmTout);
+      prefetch_tmap(&tmU);
     }
-    prefetch_tmap(&tmTin);
-    prefetch_tmap(&tmX);
-    prefetch_tmap(&tmZ);
-    prefetch_tmap(&tmTout);
-    prefetch_tmap(&tmU);
   }
   if (warp == 1) tmem_alloc(tmem_slot, Lo::kTmemCols);
   tc_fence_before_sync();
   __syncthreads();
-  if (clustered) cluster_sync();   // every CTA's barriers exist before any remote arrival
+  // Every CTA's barriers must exist before a peer pushes partial sums into it: all threads
+  // arrive here, and the epilogue (the only role that writes into other CTAs) waits before its
+  // first push; the other roles wait at the end.
+  if (clustered) cluster_arrive();
   tc_fence_after_sync();
   const uint32_t tmem_base = *tmem_slot;
   pdl_launch_dependents();
@@ -521,6 +520,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     pdl_wait();
     if (et == 0) *gen_s = ld_acquire_gpu(a.gen) + 1;
     named_barrier_sync(1, kEpi);
+    if (clustered) cluster_wait();
     const uint32_t g = *gen_s;
     int buf = 0;
     uint32_t acc_phase = 0;
@@ -700,7 +700,10 @@ __global__ void __launch_bounds__(kThreads, 1)
   __syncthreads();
   // No CTA leaves while a peer may still write into its shared memory (after a wait that gave
   // up, the exchange can be cut short); every wait above is bounded, so all CTAs get here.
-  if (clustered) cluster_sync();
+  if (clustered) {
+    if (warp < 2 || warp > 5) cluster_wait();    // the epilogue waited before its first push
+    cluster_sync();
+  }
   if (threadIdx.x == 0) {
     // the last CTA to finish moves the workspace to the next call's generation
     __threadfence();

@@ -234,6 +234,16 @@ __device__ __forceinline__ uint32_t cluster_count_x() {
 
 // All threads of all CTAs of the cluster (hardware cluster barrier; the CTAs of a cluster are
 // co-scheduled, so every one of them reaches it).
+// Split cluster barrier: every thread arrives; a thread waits (once) before it relies on the
+// other CTAs having arrived, and before it arrives again.
+__device__ __forceinline__ void cluster_arrive() {
+  asm volatile("barrier.cluster.arrive.release.aligned;" ::: "memory");
+}
+
+__device__ __forceinline__ void cluster_wait() {
+  asm volatile("barrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
+
 __device__ __forceinline__ void cluster_sync() {
   asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;"
                ::: "memory");
