@@ -164,6 +164,81 @@ def rotate_rows(T: np.ndarray, draws) -> np.ndarray:
     return np.ascontiguousarray(Y[:, draws.perm])
 
 
+def unrotate_rows(Y: np.ndarray, draws) -> np.ndarray:
+    """Y R without forming R: each row y becomes R^T y = D (Q_a kron Q_b)^T Pi^T y, with
+    (Q_a kron Q_b)^T v = vec(Q_a^T X Q_b) for X the a x b row-major reshape of v."""
+    Qa, Qb = haar_orthogonal(draws.ga), haar_orthogonal(draws.gb)
+    m, d = Y.shape
+    Z = np.empty((m, d))
+    Z[:, draws.perm] = Y
+    X = Z.reshape(m, draws.a, draws.b)
+    V = np.matmul(np.matmul(Qa.T[None, :, :], X), Qb[None, :, :]).reshape(m, d)
+    return V * draws.signs[None, :]
+
+
+def run_width(k: int, rho: int, d: int):
+    """w = d / rho when spectral tetris gives rho/2 disjoint runs of w ones (F_j = 1 on
+    complex coordinates j w .. (j+1) w - 1, App. J with an integer d/rho), else None."""
+    if rho % 2 or d % 2 or d % rho:
+        return None
+    w = d // rho
+    F = spectral_tetris(rho // 2, d // 2)
+    if not np.array_equal(F, np.kron(np.eye(rho // 2), np.ones((1, w)))):
+        return None
+    if not modulation_is_tight(F, k):
+        raise ValueError(f"(k={k}, rho={rho}, d={d}) is not a valid TFF for this construction")
+    return w
+
+
+def _run_dft(k: int, j: int, w: int) -> np.ndarray:
+    """k x w matrix with entries w^(-ki n) / sqrt(k), n = j w .. (j+1) w - 1 the absolute complex
+    coordinates of run j (the conjugated modulation of App. J)."""
+    n = np.arange(j * w, (j + 1) * w)
+    ki = np.arange(k)
+    return np.exp(-2j * np.pi * ((ki[:, None] * n[None, :]) % k) / k) / math.sqrt(k)
+
+
+def analysis_apply(k: int, rho: int, d: int, draws, X: np.ndarray) -> np.ndarray:
+    """X T^T (M x n) for T = frame(k, rho, d, draws) without forming T, when d/rho is an
+    integer.  T = T_u R^T, so each token is first taken to R^T x; then, with x_c[n] =
+    x[2n] + i x[2n+1], the complex coefficient of frame vector (j, ki) is the inner product
+    with F_j * w^(ki n) / sqrt(k), i.e. k^-1/2 sum over run j of w^(-ki n) x_c[n]; its real and
+    imaginary parts are rows 2 (j k + ki) and 2 (j k + ki) + 1 of the realified operator."""
+    X = np.asarray(X, dtype=np.float64)
+    if k == 1 and rho == d:
+        return X if draws is None else unrotate_rows(X, draws)
+    w = run_width(k, rho, d)
+    if w is None:
+        raise ValueError("structured application needs d / rho to be an integer")
+    Xr = X if draws is None else unrotate_rows(X, draws)
+    xc = Xr[:, 0::2] + 1j * Xr[:, 1::2]
+    Z = np.empty((X.shape[0], k * rho))
+    for j in range(rho // 2):
+        zc = xc[:, j * w:(j + 1) * w] @ _run_dft(k, j, w).T
+        Z[:, 2 * j * k:2 * (j + 1) * k:2] = zc.real
+        Z[:, 2 * j * k + 1:2 * (j + 1) * k:2] = zc.imag
+    return Z
+
+
+def synthesis_apply(k: int, rho: int, d: int, draws, U: np.ndarray) -> np.ndarray:
+    """U T (M x d), the adjoint of analysis_apply: per run j the complex coordinates are
+    sum over ki of u_(j,ki) w^(ki n) / sqrt(k) with u_c = u[2c] + i u[2c+1], written back as
+    (Re, Im) pairs, then each token is taken to R y."""
+    U = np.asarray(U, dtype=np.float64)
+    if k == 1 and rho == d:
+        return U if draws is None else rotate_rows(U, draws)
+    w = run_width(k, rho, d)
+    if w is None:
+        raise ValueError("structured application needs d / rho to be an integer")
+    uc = U[:, 0::2] + 1j * U[:, 1::2]
+    Y = np.empty((U.shape[0], d))
+    for j in range(rho // 2):
+        yc = uc[:, j * k:(j + 1) * k] @ np.conj(_run_dft(k, j, w))
+        Y[:, 2 * j * w:2 * (j + 1) * w:2] = yc.real
+        Y[:, 2 * j * w + 1:2 * (j + 1) * w:2] = yc.imag
+    return Y if draws is None else rotate_rows(Y, draws)
+
+
 def frame(k: int, rho: int, d: int, draws=None) -> np.ndarray:
     """Analysis operator P^T (n x d) of the TFF, rotated when rotation draws are given."""
     T = tff_analysis(k, rho, d)

@@ -83,8 +83,12 @@ struct Layout {
   static constexpr int kStageBytes = kATileBytes + kBTileBytes + kCodesStage;
   static constexpr int kRedBytes = kSplit ? BN * kBM * 4 : 0;
   static constexpr int kOnesBytes = kOnesZsum ? kATileBytes : 0;
-  static constexpr int kStages =
+  // Code rounds are decoded by warp (round mod 4), which waits for a stage's codes only in the
+  // rounds it owns; that is exact only when every phase of a stage's barrier belongs to the
+  // same warp, i.e. when the ring depth is a multiple of 4.
+  static constexpr int kStagesRaw =
       std::min(12, (kSmemBudget - kRedBytes - kOnesBytes) / kStageBytes);
+  static constexpr int kStages = kCodes ? (kStagesRaw & ~3) : kStagesRaw;
   // accumulators [0, 2 BN); sum(z) accumulators [2 BN, 4 BN)
   static constexpr int kAccCols = kOnesZsum ? 4 * BN : 2 * BN;
   static constexpr uint32_t kTmemCols = kAccCols <= 32 ? 32 : (kAccCols <= 64 ? 64 : (kAccCols <= 128 ? 128 : (kAccCols <= 256 ? 256 : 512)));
@@ -102,6 +106,7 @@ struct Layout {
   static constexpr int kBytes = oZsum + 2 * BN * 4 + 1024;          // + alignment slack
   static_assert(kBTileBytes % 1024 == 0, "B tiles must keep 1024-byte alignment");
   static_assert(kBytes <= 227 * 1024, "shared memory");
+  static_assert(kStages >= 2 && (!kCodes || kStages % 4 == 0), "ring depth");
 };
 
 template <int PHASE>

@@ -62,6 +62,14 @@ def test_llama7b_prefill_sampled(name, use_gamma):
     _check(L, X, BF16, use_gamma, sample)
 
 
+def test_llama7b_prefill_m4096_sampled():
+    # the largest prefill batch of the workload: 4096 tokens, filter off, 32 tokens checked
+    L = oracle_layer("llama2_7b_prefill", "gate")
+    X = activations("llama2_7b_prefill", "gate", 4096)
+    sample = np.sort(wl.rng(3, "sample-4096", "gate").choice(4096, 32, replace=False))
+    _check(L, X, BF16, False, sample)
+
+
 @pytest.mark.parametrize("name", ["fc1", "fc2"])
 def test_vit_mlp_full_sampled(name):
     L = oracle_layer("vit_b16_mlp", name)

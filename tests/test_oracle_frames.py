@@ -186,3 +186,46 @@ def test_invalid_triple_rejected():
     # k smaller than the support width w = d/rho breaks tightness
     with pytest.raises(ValueError):
         frames.tff_analysis(10, 16, 256)
+
+
+# ---- structured application (no dense T), for layers whose dense T does not fit in fp64
+@pytest.mark.parametrize("k,rho,d", [(18, 16, 256), (53, 16, 768), (5, 8, 40), (7, 8, 48),
+                                     (1, 48, 48), (20, 16, 256)])
+@pytest.mark.parametrize("rotate", [False, True])
+def test_structured_application_equals_the_dense_frame(k, rho, d, rotate):
+    draws = wl.rotation_draws(5, "structured", str(k), d=d) if rotate else None
+    T = frames.frame(k, rho, d, draws)
+    g = wl.rng(5, "structured-x", str(k), str(d))
+    X = g.standard_normal((6, d))
+    U = g.standard_normal((6, T.shape[0]))
+    np.testing.assert_allclose(frames.analysis_apply(k, rho, d, draws, X), X @ T.T, atol=1e-12)
+    np.testing.assert_allclose(frames.synthesis_apply(k, rho, d, draws, U), U @ T, atol=1e-12)
+
+
+def test_unrotate_is_the_transpose_rotation():
+    d = 96
+    draws = wl.rotation_draws(9, "unrotate", d=d)
+    R = frames.rotation_matrix(draws)
+    Y = wl.rng(9, "unrotate-y").standard_normal((4, d))
+    np.testing.assert_allclose(frames.unrotate_rows(Y, draws), Y @ R, atol=1e-13)
+    np.testing.assert_allclose(frames.unrotate_rows(frames.rotate_rows(Y, draws), draws), Y,
+                               atol=1e-13)
+
+
+@pytest.mark.parametrize("d", [8192, 28672])
+def test_structured_frame_is_tight_at_llama70b_widths(d):
+    # Parseval at full width, without the dense operator: synthesis(analysis(x)) = x
+    k, rho = frames.choose_k(Fraction(11, 10), d, 16)
+    draws = wl.rotation_draws(4, "tight", d=d)
+    X = wl.rng(4, "tight-x", str(d)).standard_normal((2, d))
+    Z = frames.analysis_apply(k, rho, d, draws, X)
+    assert Z.shape == (2, k * rho)
+    np.testing.assert_allclose(frames.synthesis_apply(k, rho, d, draws, Z), X, atol=1e-10)
+    # and the energy is kept (T^T T = I means |T x| = |x|)
+    np.testing.assert_allclose(np.linalg.norm(Z, axis=1), np.linalg.norm(X, axis=1), rtol=1e-12)
+
+
+def test_structured_application_needs_integer_runs():
+    # d / rho not an integer: spectral tetris places T(x) blocks, no runs of ones
+    with pytest.raises(ValueError):
+        frames.analysis_apply(5, 4, 22, None, np.zeros((1, 22)))
