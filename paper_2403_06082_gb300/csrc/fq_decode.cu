@@ -32,8 +32,9 @@
 // header is a valid start and every call leaves it valid for the next (flags keep
 // generations that are all in the past; the last CTA to finish advances the generation).
 //
-// Warps: 0 weight (A) producer, 1 TMEM owner + MMA issuer, 2-5 epilogue (thread = tile row),
-// 6 activation (B) producer, 7-10 code decoders (core stages, stage i -> warp i mod 4).
+// Warps: 0 weight (A) producer, 1 TMEM owner + MMA issuer 0, 2-5 epilogue (thread = tile row),
+// 6 activation (B) producer, 7, 8, 10, 11 code decoders (round i -> decoder i mod 4), and for
+// 16 or 32 tokens 12, 14, 15 MMA issuers 1-3 (one issuer per SM sub-partition).
 #include <cuda.h>
 #include <cudaTypedefs.h>
 
@@ -59,7 +60,22 @@ static_assert(kMaxSplit <= kWsSlices, "one ready flag per slice");
 constexpr int kEpi = 128;
 constexpr int kChunk = 16;
 constexpr int kGroup = 16;                 // columns of z per partial sum
-constexpr int kThreads = 384;
+// MMA issuers per CTA.  A tcgen05.mma with N = 16 or 32 tokens is short, and one thread cannot
+// issue K blocks (waits, MMAs, commit) as fast as the tensor core retires them; NI issuers, one
+// per SM sub-partition, each own the ring stages s = q (mod NI) and accumulate their K blocks
+// into their own accumulator, which the epilogue adds.  Owning stages (not K blocks) keeps
+// every barrier of a stage waited for by one thread, in phase order.  With 64 tokens the
+// epilogue's registers do not leave room for the extra warps: one issuer.
+template <int BN>
+struct DecCfg {
+  static constexpr int NI = BN <= 32 ? 4 : 1;
+  static constexpr int kThreads = NI == 4 ? 512 : 384;
+};
+// warp -> issuer index (warps 1, 12, 14, 15: sub-partitions 1, 0, 2, 3), -1 for other roles
+__host__ __device__ constexpr int issuer_of(int warp, int ni) {
+  return warp == 1 ? 0
+                   : (ni == 4 ? (warp == 12 ? 1 : (warp == 14 ? 2 : (warp == 15 ? 3 : -1))) : -1);
+}
 constexpr int64_t kL2PrefetchBudget = 64ll << 20;
 
 struct DecPhase {
@@ -97,20 +113,27 @@ struct DecLayout {
   static constexpr int kStage = kATile + kBTile + kCodeBytes;
   static constexpr int kRecvRow = BN + 4;                     // floats per received row
   static constexpr int kRecv = kBM * kRecvRow * 4;            // [S][128/S][BN + 4] fp32
-  static constexpr int kStages = std::min(12, (200 * 1024 - 4096 - 2 * kRecv) / kStage);
-  static constexpr uint32_t kTmemCols = 2 * BN < 32 ? 32 : 2 * BN;
+  static constexpr int NI = DecCfg<BN>::NI;
+  // a multiple of NI: issuer q owns stages q, q + NI, ...
+  static constexpr int kStages =
+      std::min(12, (216 * 1024 - 4096 - 2 * kRecv) / kStage) / NI * NI;
+  static constexpr int kAccCols = 2 * NI * BN;               // [2 buffers][NI issuers][BN]
+  static constexpr uint32_t kTmemCols =
+      kAccCols <= 32 ? 32 : (kAccCols <= 64 ? 64 : (kAccCols <= 128 ? 128 : 256));
   static constexpr int oA = 0;
   static constexpr int oB = oA + kStages * kATile;
   static constexpr int oC = oB + kStages * kBTile;
   static constexpr int oRecv = oC + kStages * kCodeBytes;    // two receive buffers
   static constexpr int oBar = oRecv + 2 * kRecv;
-  static constexpr int kBars = 4 * kStages + 7;
+  static constexpr int kBars = 4 * kStages + 10;
   static constexpr int oMisc = oBar + kBars * 8;
   static constexpr int oZs = oMisc + 32;                     // [BN] floats
   static constexpr int oZsPart = oZs + BN * 4;               // [128] floats
   static constexpr int kBytes = oZsPart + kEpi * 4 + 1024;
   static_assert(kBTile % 1024 == 0, "B tiles keep 1024-byte alignment");
-  static_assert(kStages >= 3, "pipeline depth");
+  static_assert(kStages >= 3 && kStages % NI == 0, "pipeline depth, stage ownership");
+  static_assert(kAccCols <= 256, "accumulator columns");
+  static_assert(kBytes <= 227 * 1024, "shared memory per CTA");
 };
 
 struct Task {
@@ -177,7 +200,7 @@ __device__ __forceinline__ void note_timeout(int32_t* status, int role, int task
 }
 
 template <int BN>
-__global__ void __launch_bounds__(kThreads, 1)
+__global__ void __launch_bounds__(DecCfg<BN>::kThreads, 1)
     decode_layer_kernel(const __grid_constant__ CUtensorMap tmTin,
                         const __grid_constant__ CUtensorMap tmX,
                         const __grid_constant__ CUtensorMap tmZ,
@@ -187,6 +210,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   using Lo = DecLayout<BN>;
   constexpr int S_ = Lo::kStages;
   constexpr int kBTile = Lo::kBTile;
+  constexpr int NI = Lo::NI;
 
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>(
@@ -203,8 +227,8 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint64_t* aready = empty + S_;
   uint64_t* tfull = aready + S_;
   uint64_t* tempty = tfull + 2;
-  uint64_t* mma_done = tempty + 2;
-  uint64_t* recv_bar = mma_done + 1;   // [2] the peers' partials of this CTA's slice arrived
+  uint64_t* mma_done = tempty + 2;     // [4] one per issuer
+  uint64_t* recv_bar = mma_done + 4;   // [2] the peers' partials of this CTA's slice arrived
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + Lo::oMisc);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
   uint32_t* gen_s = tmem_slot + 2;
@@ -225,10 +249,13 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   if (warp == 0) {
     // the barriers, initialised lane-parallel: fullA, fullB, empty (count 1), aready (32),
-    // tfull[2] (1), tempty[2] (kEpi), mma_done (1), recv_bar[2] (1)
+    // tfull[2] (one commit per issuer), tempty[2] (kEpi), mma_done[4] (1), recv_bar[2] (1)
     for (int b = lane; b < Lo::kBars; b += 32) {
       const int r = b - 4 * S_;
-      const uint32_t cnt = b < 3 * S_ ? 1u : (b < 4 * S_ ? 32u : ((r == 2 || r == 3) ? kEpi : 1u));
+      const uint32_t cnt = b < 3 * S_ ? 1u
+                           : (b < 4 * S_ ? 32u
+                                         : (r < 2 ? static_cast<uint32_t>(NI)
+                                                  : (r < 4 ? static_cast<uint32_t>(kEpi) : 1u)));
       mbar_init(&fullA[b], cnt);
     }
     fence_barrier_init();
@@ -413,8 +440,11 @@ __global__ void __launch_bounds__(kThreads, 1)
       for (int s = 0; s < S_; ++s)
         if (used[s] && !mbar_wait(&fullB[s], last_par[s], nullptr))
           report(a.status, FQ_ERR_TIMEOUT);
-  } else if (warp == 1) {
-    // -------------------------------------------------------------- MMA issuer
+  } else if (issuer_of(warp, NI) >= 0) {
+    // -------------------------------------------------------------- MMA issuers
+    // issuer q: the K blocks that land in ring stages s = q (mod NI), into accumulator q of
+    // the task's buffer; every issuer walks every round to follow the ring
+    const int q = issuer_of(warp, NI);
     if (lane == 0) {
       constexpr uint32_t idesc = umma_idesc_bf16(kBM, BN);
       int stage = 0;
@@ -434,44 +464,48 @@ __global__ void __launch_bounds__(kThreads, 1)
           break;
         }
         tc_fence_after_sync();
-        const uint32_t d_tmem = tmem_base + static_cast<uint32_t>(buf * BN);
+        const uint32_t d_tmem = tmem_base + static_cast<uint32_t>((buf * NI + q) * BN);
         bool ok = true;
+        bool acc = false;      // this issuer has accumulated a K block of the task
         for (int kb = k0; kb < k1; ++kb) {
-          if (t.p == 1) {
-            ok = mbar_wait(&aready[stage], (apar >> stage) & 1u, abort_flag);
-            apar ^= 1u << stage;
-          } else {
-            ok = mbar_wait(&fullA[stage], phase, abort_flag);
-          }
-          if (!ok && !*abort_flag) note_timeout(a.status, 5, i, stage, kb * 2 + static_cast<int>(phase));
-          if (ok) {
-            ok = mbar_wait(&fullB[stage], phase, abort_flag);
-            if (!ok && !*abort_flag) note_timeout(a.status, 6, i, stage, kb * 2 + static_cast<int>(phase));
-          }
-          if (!ok) break;
-          tc_fence_after_sync();
-          const uint64_t adesc = umma_desc_sw128(smem_u32(sA + stage * kATile));
-          const uint64_t bdesc = umma_desc_sw128(smem_u32(sB + stage * kBTile));
+          if (stage % NI == q) {
+            if (t.p == 1) {
+              ok = mbar_wait(&aready[stage], (apar >> stage) & 1u, abort_flag);
+              apar ^= 1u << stage;
+            } else {
+              ok = mbar_wait(&fullA[stage], phase, abort_flag);
+            }
+            if (!ok && !*abort_flag) note_timeout(a.status, 5, i, stage, kb * 2 + static_cast<int>(phase));
+            if (ok) {
+              ok = mbar_wait(&fullB[stage], phase, abort_flag);
+              if (!ok && !*abort_flag) note_timeout(a.status, 6, i, stage, kb * 2 + static_cast<int>(phase));
+            }
+            if (!ok) break;
+            tc_fence_after_sync();
+            const uint64_t adesc = umma_desc_sw128(smem_u32(sA + stage * kATile));
+            const uint64_t bdesc = umma_desc_sw128(smem_u32(sB + stage * kBTile));
 #pragma unroll
-          for (int k = 0; k < kBK / 16; ++k)
-            umma_bf16(d_tmem, adesc + 2 * k, bdesc + 2 * k, idesc, (kb > k0 || k > 0) ? 1u : 0u);
-          issued_any = true;
-          umma_commit(&empty[stage]);
+            for (int k = 0; k < kBK / 16; ++k)
+              umma_bf16(d_tmem, adesc + 2 * k, bdesc + 2 * k, idesc, (acc || k > 0) ? 1u : 0u);
+            acc = true;
+            issued_any = true;
+            umma_commit(&empty[stage]);
+          }
           if (++stage == S_) stage = 0, phase ^= 1;
         }
         if (!ok) {
           *abort_flag = 1;
           break;
         }
-        umma_commit(&tfull[buf]);      // with an empty K range this arrives at once
+        umma_commit(&tfull[buf]);      // with no K block of its own this arrives at once
         if (++buf == 2) buf = 0, acc_phase ^= 1;
       }
       if (issued_any) {
-        umma_commit(mma_done);
-        if (!mbar_wait(mma_done, 0, nullptr)) report(a.status, FQ_ERR_TIMEOUT);
+        umma_commit(&mma_done[q]);
+        if (!mbar_wait(&mma_done[q], 0, nullptr)) report(a.status, FQ_ERR_TIMEOUT);
       }
     }
-  } else if (warp >= 7 && warp != 9) {
+  } else if (warp >= 7 && warp <= 11 && warp != 9) {
     // -------------------------------------------------------------- code decoders
     const int dw = warp <= 8 ? warp - 7 : warp - 8;   // warps 7, 8, 10, 11
     int stage = 0;
@@ -524,6 +558,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     const uint32_t g = *gen_s;
     int buf = 0;
     uint32_t acc_phase = 0;
+    int ring_pos = 0;                             // ring stage of the next task's first K block
     int j = 0;                                    // tasks finished by this CTA
     for (int i = t_lo; i < t_hi; ++i, ++j) {
       const Task t = task_at(sched, i);
@@ -584,19 +619,27 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
       tc_fence_after_sync();
       const uint32_t t_row = tmem_base + (static_cast<uint32_t>(quarter * 32) << 16) +
-                             static_cast<uint32_t>(buf * BN);
+                             static_cast<uint32_t>(buf * NI * BN);
+      // issuers that accumulated K blocks of this task: those owning the task's first
+      // min(NI, K blocks) ring stages
+      const int nkb = max(0, k1 - k0);
+      const int ring0 = ring_pos % NI;
+      ring_pos = (ring_pos + nkb) % S_;
       // this thread's row of the accumulator (for the core: gamma (s Q z + zero sum z) over the
-      // CTA's K range)
+      // CTA's K range), the issuers' accumulators added in issuer order
       float vals[BN];
 #pragma unroll
       for (int c = 0; c < BN; c += kChunk) {
         float v[kChunk];
-        if (has_k) {
-          tmem_ld16(t_row + c, v);
-          tmem_wait_ld();
-        } else {
 #pragma unroll
-          for (int q = 0; q < kChunk; ++q) v[q] = 0.f;
+        for (int q = 0; q < kChunk; ++q) v[q] = 0.f;
+        for (int qa = 0; qa < NI; ++qa) {
+          if ((qa - ring0 + NI) % NI >= nkb) continue;       // uniform across the warp
+          float w[kChunk];
+          tmem_ld16(t_row + static_cast<uint32_t>(qa * BN + c), w);
+          tmem_wait_ld();
+#pragma unroll
+          for (int q = 0; q < kChunk; ++q) v[q] += w[q];
         }
 #pragma unroll
         for (int q = 0; q < kChunk; ++q)
@@ -792,7 +835,7 @@ int max_clusters(int dev, int S) {
   if (it != cache.end()) return it->second;
   cudaLaunchConfig_t cfg{};
   cfg.gridDim = dim3(static_cast<unsigned>(S * 64));
-  cfg.blockDim = dim3(kThreads);
+  cfg.blockDim = dim3(DecCfg<BN>::kThreads);
   cfg.dynamicSmemBytes = DecLayout<BN>::kBytes;
   cudaLaunchAttribute attr[1];
   attr[0].id = cudaLaunchAttributeClusterDimension;
@@ -911,7 +954,7 @@ fq_status run(const CUtensorMap* m, DecArgs& a, const int* R, const int* K, int 
   a.total = total;
   cudaLaunchConfig_t cfg{};
   cfg.gridDim = dim3(static_cast<unsigned>(plan->ncl * plan->S));
-  cfg.blockDim = dim3(kThreads);
+  cfg.blockDim = dim3(DecCfg<BN>::kThreads);
   cfg.dynamicSmemBytes = DecLayout<BN>::kBytes;
   cfg.stream = s;
   cudaLaunchAttribute attr[2];
