@@ -33,8 +33,18 @@
 // generations that are all in the past; the last CTA to finish advances the generation).
 //
 // Warps: 0 weight (A) producer, 1 TMEM owner + MMA issuer 0, 2-5 epilogue (thread = tile row),
-// 6 activation (B) producer, 7, 8, 10, 11 code decoders (round i -> decoder i mod 4), and for
-// 16 or 32 tokens 12, 14, 15 MMA issuers 1-3 (one issuer per SM sub-partition).
+// 6 activation (B) producer, 7, 8, 10, 11 code decoders (ring stage s -> decoder s mod 4), and
+// for 16 or 32 tokens 12, 14, 15 MMA issuers 1-3 (one issuer per SM sub-partition).
+//
+// Ring protocol.  A parity wait on an mbarrier is only exact when its waiter is neither ahead
+// of the barrier nor two or more phases behind it, so each barrier's waiters take part in
+// every one of its phases that follows a phase they wait for:
+//   empty[s]  (the round's MMAs completed)  the weight and the activation producers, which
+//             both fill every round of the stage;
+//   cfull[s]  (a core round's code block landed)  decoder s mod 4, whose arrival on fullA[s]
+//             the round's MMAs (and so the next code load into the stage) wait for;
+//   fullA[s]  (the A tile is in place: the weight tile's bytes, or the decoder's arrival in
+//             core rounds), fullB[s]  the issuer that owns s, which commits empty[s].
 #include <cuda.h>
 #include <cudaTypedefs.h>
 
@@ -219,13 +229,13 @@ __global__ void __launch_bounds__(DecCfg<BN>::kThreads, 1)
   uint8_t* sB = smem + Lo::oB;
   uint8_t* sC = smem + Lo::oC;
   float* recv_buf = reinterpret_cast<float*>(smem + Lo::oRecv);
-  // fullA completes every round of a stage (a weight tile or, for core tasks, its codes);
-  // aready only in core rounds, so the MMA tracks its parity per stage
+  // fullA, fullB and empty complete once in every round of their stage, cfull[s] in core
+  // rounds only (its waiters keep one parity bit per stage)
   uint64_t* fullA = reinterpret_cast<uint64_t*>(smem + Lo::oBar);
   uint64_t* fullB = fullA + S_;
   uint64_t* empty = fullB + S_;
-  uint64_t* aready = empty + S_;
-  uint64_t* tfull = aready + S_;
+  uint64_t* cfull = empty + S_;
+  uint64_t* tfull = cfull + S_;
   uint64_t* tempty = tfull + 2;
   uint64_t* mma_done = tempty + 2;     // [4] one per issuer
   uint64_t* recv_bar = mma_done + 4;   // [2] the peers' partials of this CTA's slice arrived
@@ -248,14 +258,13 @@ __global__ void __launch_bounds__(DecCfg<BN>::kThreads, 1)
   const int t_lo = sched.off[cid], t_hi = sched.off[cid + 1];   // this cluster's tasks
 
   if (warp == 0) {
-    // the barriers, initialised lane-parallel: fullA, fullB, empty (count 1), aready (32),
-    // tfull[2] (one commit per issuer), tempty[2] (kEpi), mma_done[4] (1), recv_bar[2] (1)
+    // the barriers, initialised lane-parallel: fullA, fullB, empty, cfull (count 1), tfull[2]
+    // (one commit per issuer), tempty[2] (kEpi), mma_done[4] (1), recv_bar[2] (1)
     for (int b = lane; b < Lo::kBars; b += 32) {
       const int r = b - 4 * S_;
-      const uint32_t cnt = b < 3 * S_ ? 1u
-                           : (b < 4 * S_ ? 32u
-                                         : (r < 2 ? static_cast<uint32_t>(NI)
-                                                  : (r < 4 ? static_cast<uint32_t>(kEpi) : 1u)));
+      const uint32_t cnt = r < 0 ? 1u
+                                 : (r < 2 ? static_cast<uint32_t>(NI)
+                                          : (r < 4 ? static_cast<uint32_t>(kEpi) : 1u));
       mbar_init(&fullA[b], cnt);
     }
     fence_barrier_init();
@@ -299,10 +308,9 @@ __global__ void __launch_bounds__(DecCfg<BN>::kThreads, 1)
       int stage = 0;
       uint32_t phase = 0;
       bool first = true;
-      uint32_t last_par[S_];
-      bool used[S_];
-#pragma unroll
-      for (int s = 0; s < S_; ++s) last_par[s] = 0, used[s] = false;
+      // bit s: stage s filled / its last fill a code block / parity of that fill's phase of
+      // fullA (weight tile) or cfull (code block)
+      uint32_t used = 0, last_code = 0, last_par = 0, cpar = 0;
       for (int i = t_lo; i < t_hi && !*abort_flag; ++i) {
         const Task t = task_at(sched, i);
         const DecPhase ph = phase_of(a, t.p);
@@ -314,18 +322,23 @@ __global__ void __launch_bounds__(DecCfg<BN>::kThreads, 1)
             *abort_flag = 1;
             break;
           }
+          const uint32_t bit = 1u << stage;
+          used |= bit;
           if (t.p == 1) {
-            mbar_arrive_expect_tx(&fullA[stage], kCodeBytes);
+            mbar_arrive_expect_tx(&cfull[stage], kCodeBytes);
             bulk_load(sC + stage * kCodeBytes,
                       a.words + (static_cast<int64_t>(t.tile) * ph.KB + kb) * 512, kCodeBytes,
-                      &fullA[stage], pol_w);
+                      &cfull[stage], pol_w);
+            last_code |= bit;
+            last_par = (last_par & ~bit) | (cpar & bit);
+            cpar ^= bit;
           } else {
             mbar_arrive_expect_tx(&fullA[stage], kATile);
             tma_load_2d(sA + stage * kATile, t.p == 0 ? &tmTin : &tmTout, &fullA[stage],
                         kb * kBK, t.tile * kBM, pol_w);
+            last_code &= ~bit;
+            last_par = (last_par & ~bit) | (phase << stage);
           }
-          used[stage] = true;
-          last_par[stage] = phase;
           if (++stage == S_) stage = 0, phase ^= 1;
         }
         if (first) {
@@ -352,8 +365,12 @@ __global__ void __launch_bounds__(DecCfg<BN>::kThreads, 1)
           }
         }
       }
+      // no copy may still be landing when the CTA leaves: the last fill of every stage (no
+      // later phase of its barrier exists, so the parity wait is exact)
       for (int s = 0; s < S_; ++s)
-        if (used[s] && !mbar_wait(&fullA[s], last_par[s], nullptr))
+        if (((used >> s) & 1u) &&
+            !mbar_wait(((last_code >> s) & 1u) ? &cfull[s] : &fullA[s], (last_par >> s) & 1u,
+                       nullptr))
           report(a.status, FQ_ERR_TIMEOUT);
     }
   } else if (warp == 6) {
@@ -451,7 +468,6 @@ __global__ void __launch_bounds__(DecCfg<BN>::kThreads, 1)
       uint32_t phase = 0;
       int buf = 0;
       uint32_t acc_phase = 0;
-      uint32_t apar = 0;     // bit s: parity of the next aready[s] phase
       bool issued_any = false;
       for (int i = t_lo; i < t_hi && !*abort_flag; ++i) {
         const Task t = task_at(sched, i);
@@ -469,12 +485,7 @@ __global__ void __launch_bounds__(DecCfg<BN>::kThreads, 1)
         bool acc = false;      // this issuer has accumulated a K block of the task
         for (int kb = k0; kb < k1; ++kb) {
           if (stage % NI == q) {
-            if (t.p == 1) {
-              ok = mbar_wait(&aready[stage], (apar >> stage) & 1u, abort_flag);
-              apar ^= 1u << stage;
-            } else {
-              ok = mbar_wait(&fullA[stage], phase, abort_flag);
-            }
+            ok = mbar_wait(&fullA[stage], phase, abort_flag);
             if (!ok && !*abort_flag) note_timeout(a.status, 5, i, stage, kb * 2 + static_cast<int>(phase));
             if (ok) {
               ok = mbar_wait(&fullB[stage], phase, abort_flag);
@@ -507,37 +518,46 @@ __global__ void __launch_bounds__(DecCfg<BN>::kThreads, 1)
     }
   } else if (warp >= 7 && warp <= 11 && warp != 9) {
     // -------------------------------------------------------------- code decoders
-    const int dw = warp <= 8 ? warp - 7 : warp - 8;   // warps 7, 8, 10, 11
+    // Decoder d (warps 7, 8, 10, 11) expands the code blocks of the core rounds that land in
+    // ring stages s = d (mod 4) into the stage's A slot; it waits for nothing else.  All lanes
+    // wait (measured: one polling lane with the others parked in a shuffle wakes later).
+    const int dw = warp <= 8 ? warp - 7 : warp - 8;
     int stage = 0;
-    uint32_t phase = 0;
-    int it = 0;
+    uint32_t cpar = 0;     // bit s: parity of the next cfull[s] phase
     bool ok = true;
-    for (int i = t_lo; i < t_hi && ok && !*abort_flag; ++i) {
+    for (int i = t_lo; i < t_hi && ok; ++i) {
+      if (__shfl_sync(0xffffffffu, *abort_flag != 0, 0)) break;   // warp-uniform
       const Task t = task_at(sched, i);
       const DecPhase ph = phase_of(a, t.p);
       int k0, k1;
       krange(ph, k0, k1);
-      for (int kb = k0; kb < k1; ++kb, ++it) {
-        // every decoder warp follows every round of the ring (a parity wait is only exact
-        // when the waiter is at most one phase ahead), and decodes the code rounds it owns
-        if (!mbar_wait(&fullA[stage], phase, abort_flag)) {
-          if (!*abort_flag && lane == 0) note_timeout(a.status, 7, i, stage, static_cast<int>(phase));
-          ok = false;
-          break;
-        }
-        if (t.p == 1 && (it & 3) == dw) {
+      const int n = max(0, k1 - k0);
+      if (t.p != 1) {
+        stage = (stage + n) % S_;
+        continue;
+      }
+      for (int kb = 0; kb < n; ++kb) {
+        if ((stage & 3) == dw) {
+          const bool got = mbar_wait(&cfull[stage], (cpar >> stage) & 1u, abort_flag);
+          if (!got && lane == 0 && !*abort_flag) note_timeout(a.status, 7, i, stage, static_cast<int>(cpar));
+          cpar ^= 1u << stage;
+          if (!__all_sync(0xffffffffu, got)) {
+            ok = false;
+            break;
+          }
           const uint4* codes = reinterpret_cast<const uint4*>(sC + stage * kCodeBytes);
           uint8_t* tile_a = sA + stage * kATile;
 #pragma unroll
           for (int rr = 0; rr < 4; ++rr)
             decode_row_dec(codes[lane + 32 * rr], tile_a, lane + 32 * rr);
           fence_proxy_async_smem();
-          mbar_arrive(&aready[stage]);
+          __syncwarp();
+          if (lane == 0) mbar_arrive(&fullA[stage]);
         }
-        if (++stage == S_) stage = 0, phase ^= 1;
+        if (++stage == S_) stage = 0;
       }
     }
-    if (!ok) {
+    if (!ok && lane == 0) {
       report(a.status, FQ_ERR_TIMEOUT);
       *abort_flag = 1;
     }
