@@ -303,7 +303,7 @@ __global__ void __launch_bounds__(DecCfg<BN>::kThreads, 1)
 
   if (warp == 0) {
     // -------------------------------------------------------------- weight (A) producer
-    if (lane == 0) {
+    {
       const uint64_t pol_w = policy_evict_first();
       int stage = 0;
       uint32_t phase = 0;
@@ -311,40 +311,50 @@ __global__ void __launch_bounds__(DecCfg<BN>::kThreads, 1)
       // bit s: stage s filled / its last fill a code block / parity of that fill's phase of
       // fullA (weight tile) or cfull (code block)
       uint32_t used = 0, last_code = 0, last_par = 0, cpar = 0;
-      for (int i = t_lo; i < t_hi && !*abort_flag; ++i) {
+      bool wok = true;
+      for (int i = t_lo; i < t_hi && wok; ++i) {
+        if (__any_sync(0xffffffffu, *abort_flag != 0)) break;
         const Task t = task_at(sched, i);
         const DecPhase ph = phase_of(a, t.p);
         int k0, k1;
         krange(ph, k0, k1);
         for (int kb = k0; kb < k1; ++kb) {
-          if (!mbar_wait(&empty[stage], phase ^ 1, abort_flag)) {
-            if (!*abort_flag) note_timeout(a.status, 1, i, stage, static_cast<int>(phase));
-            *abort_flag = 1;
+          const bool got = mbar_wait(&empty[stage], phase ^ 1, abort_flag);
+          if (!__all_sync(0xffffffffu, got)) {
+            if (lane == 0) {
+              if (!*abort_flag) note_timeout(a.status, 1, i, stage, static_cast<int>(phase));
+              *abort_flag = 1;
+            }
+            wok = false;
             break;
           }
           const uint32_t bit = 1u << stage;
           used |= bit;
           if (t.p == 1) {
-            mbar_arrive_expect_tx(&cfull[stage], kCodeBytes);
-            bulk_load(sC + stage * kCodeBytes,
-                      a.words + (static_cast<int64_t>(t.tile) * ph.KB + kb) * 512, kCodeBytes,
-                      &cfull[stage], pol_w);
+            if (lane == 0) {
+              mbar_arrive_expect_tx(&cfull[stage], kCodeBytes);
+              bulk_load(sC + stage * kCodeBytes,
+                        a.words + (static_cast<int64_t>(t.tile) * ph.KB + kb) * 512, kCodeBytes,
+                        &cfull[stage], pol_w);
+            }
             last_code |= bit;
             last_par = (last_par & ~bit) | (cpar & bit);
             cpar ^= bit;
           } else {
-            mbar_arrive_expect_tx(&fullA[stage], kATile);
-            tma_load_2d(sA + stage * kATile, t.p == 0 ? &tmTin : &tmTout, &fullA[stage],
-                        kb * kBK, t.tile * kBM, pol_w);
+            if (lane == 0) {
+              mbar_arrive_expect_tx(&fullA[stage], kATile);
+              tma_load_2d(sA + stage * kATile, t.p == 0 ? &tmTin : &tmTout, &fullA[stage],
+                          kb * kBK, t.tile * kBM, pol_w);
+            }
             last_code &= ~bit;
             last_par = (last_par & ~bit) | (phase << stage);
           }
           if (++stage == S_) stage = 0, phase ^= 1;
         }
-        if (first) {
+        if (first && wok) {
           first = false;
           // warm L2 with the weight tiles of this CTA's later tasks
-          for (int j = i + 1; j < t_hi && a.prefetch_later > 0; ++j) {
+          for (int j = i + 1; j < t_hi && a.prefetch_later > 0 && lane == 0; ++j) {
             const Task u = task_at(sched, j);
             const DecPhase q = phase_of(a, u.p);
             int u0, u1;
@@ -367,7 +377,7 @@ __global__ void __launch_bounds__(DecCfg<BN>::kThreads, 1)
       }
       // no copy may still be landing when the CTA leaves: the last fill of every stage (no
       // later phase of its barrier exists, so the parity wait is exact)
-      for (int s = 0; s < S_; ++s)
+      for (int s = 0; s < S_ && lane == 0; ++s)
         if (((used >> s) & 1u) &&
             !mbar_wait(((last_code >> s) & 1u) ? &cfull[s] : &fullA[s], (last_par >> s) & 1u,
                        nullptr))
@@ -383,10 +393,7 @@ __global__ void __launch_bounds__(DecCfg<BN>::kThreads, 1)
     const int rows_per = kBM / S;
     int stage = 0;
     uint32_t phase = 0;
-    uint32_t last_par[S_];
-    bool used[S_];
-#pragma unroll
-    for (int s = 0; s < S_; ++s) last_par[s] = 0, used[s] = false;
+    uint32_t used = 0, last_par = 0;   // bit s: stage s filled, parity of its last fill
     for (int i = t_lo; i < t_hi; ++i) {
       if (__shfl_sync(0xffffffffu, *abort_flag != 0, 0)) break;   // warp-uniform
       const Task t = task_at(sched, i);
@@ -432,30 +439,28 @@ __global__ void __launch_bounds__(DecCfg<BN>::kThreads, 1)
             continue;
           }
         }
-        if (lane == 0) {
-          for (; kb < kb_end; ++kb) {
-            if (!mbar_wait(&empty[stage], phase ^ 1, abort_flag)) {
-              if (!*abort_flag) note_timeout(a.status, 3, i, stage, static_cast<int>(phase));
-              ok = false;
-              break;
-            }
+        for (; kb < kb_end; ++kb) {
+          const bool got = mbar_wait(&empty[stage], phase ^ 1, abort_flag);
+          if (!__all_sync(0xffffffffu, got)) {
+            if (lane == 0 && !*abort_flag) note_timeout(a.status, 3, i, stage, static_cast<int>(phase));
+            ok = false;
+            break;
+          }
+          if (lane == 0) {
             mbar_arrive_expect_tx(&fullB[stage], kBTile);
             tma_load_2d(sB + stage * kBTile, tm, &fullB[stage], kb * kBK, 0, pol_x);
-            used[stage] = true;
-            last_par[stage] = phase;
-            if (++stage == S_) stage = 0, phase ^= 1;
           }
+          used |= 1u << stage;
+          last_par = (last_par & ~(1u << stage)) | (phase << stage);
+          if (++stage == S_) stage = 0, phase ^= 1;
         }
-        ok = __shfl_sync(0xffffffffu, ok, 0);
-        kb = __shfl_sync(0xffffffffu, kb, 0);
-        // stage / phase / used / last_par live in lane 0 only
       }
       if (!ok && lane == 0) *abort_flag = 1;
       if (!__shfl_sync(0xffffffffu, ok, 0)) break;
     }
     if (lane == 0)
       for (int s = 0; s < S_; ++s)
-        if (used[s] && !mbar_wait(&fullB[s], last_par[s], nullptr))
+        if (((used >> s) & 1u) && !mbar_wait(&fullB[s], (last_par >> s) & 1u, nullptr))
           report(a.status, FQ_ERR_TIMEOUT);
   } else if (issuer_of(warp, NI) >= 0) {
     // -------------------------------------------------------------- MMA issuers
