@@ -3,8 +3,8 @@
 // Every phase is one persistent, warp-specialised kernel computing
 //     out[t][i] = epilogue( sum_k A[i][k] * B[t][k] )      (i < R rows, t < M tokens)
 // with the weight-side operand A as the 128-row MMA operand and the tokens as the N operand
-// (N = BN in {16, ..., 256}), so one kernel serves decode (M <= 16) and prefill (M in the
-// thousands).  Phases (Sec. 3.2):
+// (N = BN = 128 or 256).  It serves batches of more than 64 tokens (prefill); smaller ones take
+// the fused decode kernel.  Phases (Sec. 3.2):
 //   analysis   A = T_in (n_in x d_in),  B = x,  out = z (bf16)
 //   core       A = 2-bit codes of C_hat (n_out x n_in) decoded to bf16 in shared memory,
 //              B = z, out = u = gamma * (s * acc + zero * sum(z))   (bf16)
@@ -16,17 +16,9 @@
 // of shared-memory stages guarded by mbarriers; accumulators are double-buffered in TMEM so
 // the epilogue of one tile overlaps the MMAs of the next.
 //
-// Small batches (BN <= 64) leave too few row tiles to occupy the GPU, so the K range of a
-// tile is split over the S CTAs of a thread-block cluster.  Each CTA writes its fp32 partial
-// tile to its own shared memory, the CTAs signal one another through cluster-scope mbarrier
-// arrivals, and each reduces a slice of the tile's rows by reading all S partials through
-// distributed shared memory in a fixed order (deterministic, no global partials, no atomics).
-// In the core phase with small batches, sum(z) comes from the tensor cores: every K step also
-// multiplies the z tile by a constant all-ones A tile into a second accumulator, so each split
-// carries its own share of sum(z), accumulated in fp32 from exactly the bf16 values its MMAs
-// consumed.  With larger batches (one split) the analysis epilogue produces per-tile sums of z
-// instead, which costs no tensor time.  Decoder warps take whole stages in turn (stage i goes
-// to warp i mod 4), so four stages are decoded at once.
+// sum(z), needed by the core's zero term, comes from the analysis epilogue as one sum per
+// 128-row tile of z and token, taken over the bf16 values stored.  Decoder warps take whole
+// stages in turn (stage i goes to warp i mod 4), so four stages are decoded at once.
 //
 // The three phases are chained with programmatic dependent launch (the analysis kernel too,
 // so consecutive layers chain as well): a kernel's CTAs start on SMs as they free up, load
@@ -52,58 +44,48 @@ constexpr int kBM = 128;                    // MMA M (rows of A per tile)
 constexpr int kBK = 64;                     // K per stage (one 128-byte swizzle atom of bf16)
 constexpr int kATileBytes = kBM * kBK * 2;  // 16 KiB
 constexpr int kCodeBytes = kBM * kBK / 4;   // 2 KiB of packed codes per stage
-constexpr int kMaxSplits = 8;               // portable cluster size
 constexpr int kSmemBudget = 200 * 1024;
-constexpr int64_t kL2PrefetchBudget = 64ll << 20;   // bytes of later-phase weights warmed in L2
 constexpr int kEpi = 128;                   // epilogue threads
 constexpr int kChunk = 16;                  // accumulator columns per TMEM load
 
 struct PhaseArgs {
   int R, K, M;
-  int RT, TT, S, KB, kb_per_split, tiles;
+  int RT, TT, KB, tiles;
   const uint32_t* words;     // core: packed codes
   __nv_bfloat16* out;        // [M][R]
-  float* zsum_part;          // BN >= 128: analysis writes [RT][M] sums of z; core reads them
+  float* zsum_part;          // analysis writes [RT][M] sums of z; the core reads them
   int zsum_tiles;
   const __half* scale;
   const __half* zero;
   const float* gamma;
   int32_t* status;
-  const char* pf_base[2];    // analysis: later phases' weights to warm in L2 (or null)
-  int64_t pf_bytes[2];
 };
 
 template <int PHASE, int BN>
 struct Layout {
   static constexpr bool kCodes = PHASE == kCore;
-  static constexpr bool kSplit = BN <= 64;              // cluster split-K allowed
-  static constexpr bool kOnesZsum = kCodes && BN <= 64;   // sum(z) by an all-ones MMA
   static constexpr int kBTileBytes = BN * kBK * 2;
   static constexpr int kCodesStage = kCodes ? kCodeBytes : 0;
   static constexpr int kStageBytes = kATileBytes + kBTileBytes + kCodesStage;
-  static constexpr int kRedBytes = kSplit ? BN * kBM * 4 : 0;
-  static constexpr int kOnesBytes = kOnesZsum ? kATileBytes : 0;
   // Code rounds are decoded by warp (round mod 4), which waits for a stage's codes only in the
   // rounds it owns; that is exact only when every phase of a stage's barrier belongs to the
   // same warp, i.e. when the ring depth is a multiple of 4.
-  static constexpr int kStagesRaw =
-      std::min(12, (kSmemBudget - kRedBytes - kOnesBytes) / kStageBytes);
+  static constexpr int kStagesRaw = std::min(12, kSmemBudget / kStageBytes);
   static constexpr int kStages = kCodes ? (kStagesRaw & ~3) : kStagesRaw;
-  // accumulators [0, 2 BN); sum(z) accumulators [2 BN, 4 BN)
-  static constexpr int kAccCols = kOnesZsum ? 4 * BN : 2 * BN;
-  static constexpr uint32_t kTmemCols = kAccCols <= 32 ? 32 : (kAccCols <= 64 ? 64 : (kAccCols <= 128 ? 128 : (kAccCols <= 256 ? 256 : 512)));
+  // double-buffered accumulators [0, 2 BN)
+  static constexpr int kAccCols = 2 * BN;
+  static constexpr uint32_t kTmemCols = kAccCols <= 256 ? 256 : 512;
   // byte offsets from the 1024-aligned base
-  static constexpr int oOnes = 0;
-  static constexpr int oA = oOnes + kOnesBytes;
+  static constexpr int oA = 0;
   static constexpr int oB = oA + kStages * kATileBytes;
   static constexpr int oCodes = oB + kStages * kBTileBytes;
-  static constexpr int oRed = oCodes + kStages * kCodesStage;
-  static constexpr int oBar = oRed + kRedBytes;
-  static constexpr int kNumBars = 4 * kStages + 2 + 2 + 1 + 2;
+  static constexpr int oBar = oCodes + kStages * kCodesStage;
+  static constexpr int kNumBars = 4 * kStages + 2 + 2 + 1;
   static constexpr int oMisc = oBar + kNumBars * 8;
   static constexpr int oRedSmall = oMisc + 16;                      // [4][kChunk] floats
   static constexpr int oZsum = oRedSmall + 4 * kChunk * 4;          // [2][BN] floats
   static constexpr int kBytes = oZsum + 2 * BN * 4 + 1024;          // + alignment slack
+  static_assert(BN == 128 || BN == 256, "prefill tile widths");
   static_assert(kBTileBytes % 1024 == 0, "B tiles must keep 1024-byte alignment");
   static_assert(kBytes <= 227 * 1024, "shared memory");
   static_assert(kStages >= 2 && (!kCodes || kStages % 4 == 0), "ring depth");
@@ -168,7 +150,6 @@ __global__ void __launch_bounds__(threads_for<PHASE>(), 1)
   uint8_t* sA = smem + Lo::oA;
   uint8_t* sB = smem + Lo::oB;
   uint8_t* sCodes = smem + Lo::oCodes;
-  float* red_buf = reinterpret_cast<float*>(smem + Lo::oRed);      // [BN][128] partial tile
   uint64_t* full = reinterpret_cast<uint64_t*>(smem + Lo::oBar);   // A (+B) landed / B landed
   uint64_t* empty = full + S_;      // stage consumed by the MMAs
   uint64_t* aready = empty + S_;    // decoded A tile written (core)
@@ -176,25 +157,14 @@ __global__ void __launch_bounds__(threads_for<PHASE>(), 1)
   uint64_t* tfull = cfull + S_;     // accumulator ready
   uint64_t* tempty = tfull + 2;     // accumulator drained
   uint64_t* mma_done = tempty + 2;
-  uint64_t* rdy = mma_done + 1;     // cluster: partials of every CTA written
-  uint64_t* cons = rdy + 1;         // cluster: every CTA done reading partials
-  uint8_t* sOnes = smem + Lo::oOnes;                               // all-ones A tile
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + Lo::oMisc);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
   float* red = reinterpret_cast<float*>(smem + Lo::oRedSmall);     // [4][kChunk]
-  float* zsum_s = reinterpret_cast<float*>(smem + Lo::oZsum);      // [2][BN] (BN >= 128)
+  float* zsum_s = reinterpret_cast<float*>(smem + Lo::oZsum);      // [2][BN]
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const bool clustered = p.S > 1;
-  uint32_t rank = 0, cid = blockIdx.x, ncl = gridDim.x;
-  if (clustered) {
-    rank = cluster_ctarank();
-    cid = cluster_id_x();
-    ncl = cluster_count_x();
-  }
-  const int ks = static_cast<int>(rank);
-  const int k0 = ks * p.kb_per_split;
-  const int k1 = min(p.KB, k0 + p.kb_per_split);
+  const uint32_t cid = blockIdx.x, ncl = gridDim.x;
+  const int k0 = 0, k1 = p.KB;
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < S_; ++s) {
@@ -208,24 +178,14 @@ __global__ void __launch_bounds__(threads_for<PHASE>(), 1)
       mbar_init(&tempty[b], kEpi);
     }
     mbar_init(mma_done, 1);
-    mbar_init(rdy, static_cast<uint32_t>(p.S));
-    mbar_init(cons, static_cast<uint32_t>(p.S));
     *abort_flag = 0;
     fence_barrier_init();
     if (!kCodes) prefetch_tmap(&tmA);
     prefetch_tmap(&tmB);
   }
-  if (Lo::kOnesZsum) {
-    // bf16 1.0 everywhere (the swizzle permutes identical chunks, so no layout is needed)
-    for (int i = threadIdx.x; i < kATileBytes / 16; i += blockDim.x)
-      reinterpret_cast<uint4*>(sOnes)[i] = make_uint4(0x3F803F80u, 0x3F803F80u, 0x3F803F80u,
-                                                      0x3F803F80u);
-    fence_proxy_async_smem();
-  }
   if (warp == 1) tmem_alloc(tmem_slot, Lo::kTmemCols);
   tc_fence_before_sync();
   __syncthreads();
-  if (clustered) cluster_sync();   // every CTA's barriers exist before any remote arrival
   tc_fence_after_sync();
   const uint32_t tmem_base = *tmem_slot;
 
@@ -306,24 +266,6 @@ __global__ void __launch_bounds__(threads_for<PHASE>(), 1)
           issued[stage] = true;
           issued_parity[stage] = phase;
           if (++stage == S_) stage = 0, phase ^= 1;
-          if (PHASE == kAnalysis && it + 1 == pre) {
-            // this CTA's share of the later phases' weights, into L2 while T_in streams
-            for (int r = 0; r < 2; ++r) {
-              if (!p.pf_base[r]) continue;
-              const int64_t share =
-                  ((p.pf_bytes[r] + gridDim.x - 1) / gridDim.x + 255) & ~255LL;
-              const int64_t beg = static_cast<int64_t>(blockIdx.x) * share;
-              const int64_t end = p.pf_bytes[r] < beg + share ? p.pf_bytes[r] : beg + share;
-              for (int64_t off = beg; off < end; off += 32768) {
-                const uint32_t len =
-                    static_cast<uint32_t>(end - off < 32768 ? end - off : 32768);
-                asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(
-                                 p.pf_base[r] + off),
-                             "r"(len)
-                             : "memory");
-              }
-            }
-          }
         }
       }
       // Never leave with copies in flight: wait (bounded) for the last round of each stage.
@@ -352,8 +294,6 @@ __global__ void __launch_bounds__(threads_for<PHASE>(), 1)
         }
         tc_fence_after_sync();
         const uint32_t d_tmem = tmem_base + static_cast<uint32_t>(buf * BN);
-        const uint32_t d_ones = tmem_base + static_cast<uint32_t>(2 * BN + buf * BN);
-        const uint64_t odesc = umma_desc_sw128(smem_u32(sOnes));
         bool ok = true;
         for (int kb = k0; kb < k1; ++kb) {
           ok = mbar_wait(&full[stage], phase, abort_flag) &&
@@ -363,14 +303,8 @@ __global__ void __launch_bounds__(threads_for<PHASE>(), 1)
           const uint64_t adesc = umma_desc_sw128(smem_u32(sA + stage * kATileBytes));
           const uint64_t bdesc = umma_desc_sw128(smem_u32(sB + stage * kBTile));
 #pragma unroll
-          for (int k = 0; k < kBK / 16; ++k) {
-            // advance 16 bf16 = 32 bytes along K inside the swizzle atom
-            umma_bf16(d_tmem, adesc + 2 * k, bdesc + 2 * k, idesc,
-                      (kb > k0 || k > 0) ? 1u : 0u);
-            if (Lo::kOnesZsum)
-              umma_bf16(d_ones, odesc + 2 * k, bdesc + 2 * k, idesc,
-                        (kb > k0 || k > 0) ? 1u : 0u);
-          }
+          for (int k = 0; k < kBK / 16; ++k)   // 16 bf16 = 32 bytes along K per step
+            umma_bf16(d_tmem, adesc + 2 * k, bdesc + 2 * k, idesc, (kb > k0 || k > 0) ? 1u : 0u);
           issued_any = true;
           umma_commit(&empty[stage]);
           if (++stage == S_) stage = 0, phase ^= 1;
@@ -398,13 +332,7 @@ __global__ void __launch_bounds__(threads_for<PHASE>(), 1)
     pdl_wait();
     int buf = 0;
     uint32_t acc_phase = 0;
-    int j = 0;                                    // tiles finished by this CTA
-    // the slice of each tile's rows this CTA reduces when the tile's K range is split
-    const int rows_per = (kBM + p.S - 1) / p.S;
-    const int r0 = ks * rows_per;
-    const int rcnt = max(0, min(kBM - r0, rows_per));
-    const uint32_t red_addr = smem_u32(red_buf);
-    for (int tile = static_cast<int>(cid); tile < p.tiles; tile += static_cast<int>(ncl), ++j) {
+    for (int tile = static_cast<int>(cid); tile < p.tiles; tile += static_cast<int>(ncl)) {
       const int rt = tile % p.RT, tt = tile / p.RT;
       const int row = rt * kBM + r_in_tile;
       const int t0 = tt * BN;
@@ -414,7 +342,7 @@ __global__ void __launch_bounds__(threads_for<PHASE>(), 1)
         s_i = __half2float(p.scale[row]);
         z_i = __half2float(p.zero[row]);
       }
-      if (PHASE == kCore && !Lo::kOnesZsum) {
+      if (PHASE == kCore) {
         // sum_j z[t][j] for the tile's tokens, from the analysis phase's per-tile sums
         named_barrier_sync(1, kEpi);
         for (int q = et; q < BN; q += kEpi) {
@@ -427,8 +355,7 @@ __global__ void __launch_bounds__(threads_for<PHASE>(), 1)
         }
         named_barrier_sync(1, kEpi);
       }
-      bool fail = !mbar_wait(&tfull[buf], acc_phase, abort_flag);
-      if (clustered && j > 0 && !fail) fail = !mbar_wait_cluster(cons, (j - 1) & 1);
+      const bool fail = !mbar_wait(&tfull[buf], acc_phase, abort_flag);
       if (fail) report(p.status, FQ_ERR_TIMEOUT);
       if (bar_red_or(1, kEpi, fail || *abort_flag)) {
         if (et == 0) *abort_flag = 1;
@@ -438,26 +365,22 @@ __global__ void __launch_bounds__(threads_for<PHASE>(), 1)
       const uint32_t t_row = tmem_base + (static_cast<uint32_t>(quarter * 32) << 16) +
                              static_cast<uint32_t>(buf * BN);
       const float* zs = zsum_s + buf * BN;
-      const uint32_t t_ones = t_row + static_cast<uint32_t>(2 * BN);
-
-      if (!clustered) {
+      {
         const float g_i = (PHASE == kCore && row_ok && p.gamma) ? p.gamma[row] : 1.f;
 #pragma unroll 1
         for (int c = 0; c < BN; c += kChunk) {
-          float v[kChunk], zv[kChunk];
+          float v[kChunk];
           tmem_ld16(t_row + c, v);
-          if (Lo::kOnesZsum) tmem_ld16(t_ones + c, zv);
           tmem_wait_ld();
 #pragma unroll
           for (int q = 0; q < kChunk; ++q) {
-            const float zsq = Lo::kOnesZsum ? zv[q] : zs[c + q];
-            if (PHASE == kCore) v[q] = g_i * fmaf(s_i, v[q], z_i * zsq);
+            if (PHASE == kCore) v[q] = g_i * fmaf(s_i, v[q], z_i * zs[c + q]);
             const __nv_bfloat16 b = __float2bfloat16_rn(v[q]);
             v[q] = __bfloat162float(b);
             const int t = t0 + c + q;
             if (row_ok && t < p.M) p.out[static_cast<int64_t>(t) * p.R + row] = b;
           }
-          if (PHASE == kAnalysis && !Lo::kSplit) {
+          if (PHASE == kAnalysis) {
             // per-token sum over the tile's 128 rows of the bf16 z actually stored
 #pragma unroll
             for (int q = 0; q < kChunk; ++q) {
@@ -483,72 +406,9 @@ __global__ void __launch_bounds__(threads_for<PHASE>(), 1)
         }
         tc_fence_before_sync();
         mbar_arrive(&tempty[buf]);
-      } else if (Lo::kSplit) {
-        // ---- cluster split-K: partial tile -> own shared memory, token-major [BN][128]
-#pragma unroll 1
-        for (int c = 0; c < BN; c += kChunk) {
-          float v[kChunk], zv[kChunk];
-          tmem_ld16(t_row + c, v);
-          if (Lo::kOnesZsum) tmem_ld16(t_ones + c, zv);
-          tmem_wait_ld();
-#pragma unroll
-          for (int q = 0; q < kChunk; ++q) {
-            const float zsq = Lo::kOnesZsum ? zv[q] : zs[c + q];
-            if (PHASE == kCore) v[q] = fmaf(s_i, v[q], z_i * zsq);
-            red_buf[(c + q) * kBM + r_in_tile] = v[q];
-          }
-        }
-        tc_fence_before_sync();
-        mbar_arrive(&tempty[buf]);
-        fence_acq_rel_cluster();
-        named_barrier_sync(1, kEpi);
-        if (et == 0)
-          for (int q = 0; q < p.S; ++q) mbar_arrive_cluster(mapa(smem_u32(rdy), q));
-        const bool ok = mbar_wait_cluster(rdy, j & 1);
-        if (!ok) report(p.status, FQ_ERR_TIMEOUT);
-        if (bar_red_or(1, kEpi, !ok)) {
-          if (et == 0) *abort_flag = 1;
-          break;
-        }
-        // reduce rows r0 .. r0 + rcnt of the tile over the S partials, in rank order; the
-        // loads of four elements are issued together
-        const int total = rcnt * BN;
-        for (int base = et; base < total; base += 4 * kEpi) {
-          float part[4][kMaxSplits];
-#pragma unroll
-          for (int g = 0; g < 4; ++g) {
-            const int idx = base + g * kEpi;
-            const int tok = idx / rcnt, rl = r0 + idx % rcnt;
-            const uint32_t off = red_addr + static_cast<uint32_t>((tok * kBM + rl) * 4);
-#pragma unroll
-            for (int q = 0; q < kMaxSplits; ++q)
-              part[g][q] = (idx < total && q < p.S) ? ld_dsmem_f32(mapa(off, q)) : 0.f;
-          }
-#pragma unroll
-          for (int g = 0; g < 4; ++g) {
-            const int idx = base + g * kEpi;
-            if (idx >= total) break;
-            const int tok = idx / rcnt, rl = r0 + idx % rcnt;
-            float sum = part[g][0];
-#pragma unroll
-            for (int q = 1; q < kMaxSplits; ++q)
-              if (q < p.S) sum += part[g][q];
-            const int orow = rt * kBM + rl, t = t0 + tok;
-            if (orow < p.R && t < p.M) {
-              if (PHASE == kCore && p.gamma) sum *= p.gamma[orow];
-              p.out[static_cast<int64_t>(t) * p.R + orow] = __float2bfloat16_rn(sum);
-            }
-          }
-        }
-        named_barrier_sync(1, kEpi);    // this CTA's reads of every partial are done
-        if (et == 0)
-          for (int q = 0; q < p.S; ++q) mbar_arrive_cluster(mapa(smem_u32(cons), q));
       }
       if (++buf == 2) buf = 0, acc_phase ^= 1;
     }
-    // Peers may still be reading this CTA's partial tile: do not exit before they are done.
-    if (clustered && j > 0 && !mbar_wait_cluster(cons, (j - 1) & 1))
-      report(p.status, FQ_ERR_TIMEOUT);
   } else {
     // ---------------------------------------------------------------- code decoders (core)
     if (kCodes) {
@@ -622,13 +482,7 @@ bool make_tmap(CUtensorMap* m, const void* base, int64_t rows, int64_t cols, int
              CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
-int pick_bn(int M) {
-  if (M <= 16) return 16;
-  if (M <= 32) return 32;
-  if (M <= 64) return 64;
-  if (M <= 128) return 128;
-  return 256;
-}
+int pick_bn(int M) { return M <= 128 ? 128 : 256; }
 
 struct DeviceInfo {
   int dev = -1;
@@ -656,58 +510,14 @@ cudaError_t prepare_kernel(int dev) {
   return e;
 }
 
-// Largest number of co-resident clusters of `S` CTAs for this kernel (0 if none).
-template <int PHASE, int BN>
-int max_clusters(int dev, int S) {
-  static std::mutex mu;
-  static std::map<std::pair<int, int>, int> cache;
-  std::lock_guard<std::mutex> g(mu);
-  const auto key = std::make_pair(dev, S);
-  const auto it = cache.find(key);
-  if (it != cache.end()) return it->second;
-  cudaLaunchConfig_t cfg{};
-  cfg.gridDim = dim3(static_cast<unsigned>(S * 64));
-  cfg.blockDim = dim3(threads_for<PHASE>());
-  cfg.dynamicSmemBytes = Layout<PHASE, BN>::kBytes;
-  cudaLaunchAttribute attr[1];
-  attr[0].id = cudaLaunchAttributeClusterDimension;
-  attr[0].val.clusterDim.x = static_cast<unsigned>(S);
-  attr[0].val.clusterDim.y = 1;
-  attr[0].val.clusterDim.z = 1;
-  cfg.attrs = attr;
-  cfg.numAttrs = 1;
-  int n = 0;
-  if (cudaOccupancyMaxActiveClusters(&n, tc_phase_kernel<PHASE, BN>, &cfg) != cudaSuccess) {
-    cudaGetLastError();
-    n = 0;
-  }
-  cache[key] = n;
-  return n;
-}
-
-// Split K over clusters of S CTAs so that the tiles' K blocks spread evenly over the
-// co-resident clusters: minimise waves * (K blocks per split + fixed per-tile cost).
+// One tile per CTA and round: as many CTAs as tiles, at most one per SM.
 template <int PHASE, int BN>
 void plan_phase(PhaseArgs& a, const DeviceInfo& d, int& grid) {
   a.RT = static_cast<int>(ceil_div(a.R, kBM));
   a.TT = static_cast<int>(ceil_div(a.M, BN));
   a.KB = static_cast<int>(ceil_div(a.K, kBK));
   a.tiles = a.RT * a.TT;
-  int best_s = 1, best_par = std::min(a.tiles, d.sms);
-  double best = static_cast<double>(ceil_div(a.tiles, best_par)) * (a.KB + 3.0);
-  if (Layout<PHASE, BN>::kSplit) {
-    for (int s = 2; s <= std::min(kMaxSplits, a.KB); ++s) {
-      const int kbs = static_cast<int>(ceil_div(a.KB, s));
-      if (ceil_div(a.KB, kbs) != s) continue;
-      const int cl = std::min(max_clusters<PHASE, BN>(d.dev, s), a.tiles);
-      if (cl <= 0) continue;
-      const double cost = static_cast<double>(ceil_div(a.tiles, cl)) * (kbs + 3.0) + 1.0;
-      if (cost < best - 1e-9) best = cost, best_s = s, best_par = cl;
-    }
-  }
-  a.S = best_s;
-  a.kb_per_split = static_cast<int>(ceil_div(a.KB, best_s));
-  grid = best_par * best_s;
+  grid = std::min(a.tiles, d.sms);
 }
 
 struct WsLayout {
@@ -735,15 +545,11 @@ cudaError_t launch_phase(const CUtensorMap& tmA, const CUtensorMap& tmB, const P
   cfg.blockDim = dim3(threads_for<PHASE>());
   cfg.dynamicSmemBytes = Layout<PHASE, BN>::kBytes;
   cfg.stream = s;
-  cudaLaunchAttribute attr[2];
+  cudaLaunchAttribute attr[1];
   attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
   attr[0].val.programmaticStreamSerializationAllowed = 1;
-  attr[1].id = cudaLaunchAttributeClusterDimension;
-  attr[1].val.clusterDim.x = static_cast<unsigned>(a.S);
-  attr[1].val.clusterDim.y = 1;
-  attr[1].val.clusterDim.z = 1;
   cfg.attrs = attr;
-  cfg.numAttrs = a.S > 1 ? 2 : 1;
+  cfg.numAttrs = 1;
   return cudaLaunchKernelEx(&cfg, tc_phase_kernel<PHASE, BN>, tmA, tmB, a);
 }
 
@@ -760,8 +566,6 @@ fq_status run_forward(const CUtensorMap* maps, PhaseArgs* a, cudaStream_t s) {
   plan_phase<kAnalysis, BN>(a[0], d, g[0]);
   plan_phase<kCore, BN>(a[1], d, g[1]);
   plan_phase<kSynthesis, BN>(a[2], d, g[2]);
-  // the per-tile sums of z come from the analysis epilogue only when it is not split
-  if (!Layout<kCore, BN>::kOnesZsum && a[0].S != 1) return FQ_ERR_UNSUPPORTED;
   a[1].zsum_tiles = a[0].RT;
   if (launch_phase<kAnalysis, BN>(maps[0], maps[1], a[0], g[0], s) != cudaSuccess ||
       launch_phase<kCore, BN>(maps[1], maps[2], a[1], g[1], s) != cudaSuccess ||
@@ -804,18 +608,6 @@ fq_status launch_tc_forward(const void* x, int M, int d_in, const void* T_in,
     a[ph].zsum_part = zsum;
     a[ph].status = status;
   }
-  // Warm L2 with the code words, and with T_out^T when both fit comfortably, while the
-  // analysis phase streams T_in (small batches only: there the phases are HBM-bound).
-  const int64_t code_bytes = static_cast<int64_t>(fq_packed_words(n_out, n_in)) * 4;
-  const int64_t tout_bytes = static_cast<int64_t>(d_out) * n_out * 2;
-  if (M <= 64 && code_bytes <= kL2PrefetchBudget) {
-    a[0].pf_base[0] = reinterpret_cast<const char*>(Cq.words);
-    a[0].pf_bytes[0] = code_bytes;
-    if (code_bytes + tout_bytes <= kL2PrefetchBudget) {
-      a[0].pf_base[1] = static_cast<const char*>(T_out_t);
-      a[0].pf_bytes[1] = tout_bytes;
-    }
-  }
   a[1].words = Cq.words;
   a[1].scale = reinterpret_cast<const __half*>(Cq.scale);
   a[1].zero = reinterpret_cast<const __half*>(Cq.zero);
@@ -828,13 +620,7 @@ fq_status launch_tc_forward(const void* x, int M, int d_in, const void* T_in,
       !make_tmap(&maps[4], u, M, n_out, BN))
     return FQ_ERR_CUDA;
 
-  switch (BN) {
-    case 16: return run_forward<16>(maps, a, s);
-    case 32: return run_forward<32>(maps, a, s);
-    case 64: return run_forward<64>(maps, a, s);
-    case 128: return run_forward<128>(maps, a, s);
-    default: return run_forward<256>(maps, a, s);
-  }
+  return BN == 128 ? run_forward<128>(maps, a, s) : run_forward<256>(maps, a, s);
 }
 
 }  // namespace fq
