@@ -33,8 +33,9 @@
 // generations that are all in the past; the last CTA to finish advances the generation).
 //
 // Warps: 0 weight (A) producer, 1 TMEM owner + MMA issuer 0, 2-5 epilogue (thread = tile row),
-// 6 activation (B) producer, 7, 8, 10, 11 code decoders (ring stage s -> decoder s mod 4), and
-// for 16 or 32 tokens 12, 14, 15 MMA issuers 1-3 (one issuer per SM sub-partition).
+// 6 activation (B) producer, 7-10 code decoders (ring stage s -> decoder s mod 4; one per SM
+// sub-partition, since the decode is issue-bound), and for 16 or 32 tokens 12, 14, 15 MMA
+// issuers 1-3 (one issuer per SM sub-partition).
 //
 // Ring protocol.  A parity wait on an mbarrier is only exact when its waiter is neither ahead
 // of the barrier nor two or more phases behind it, so each barrier's waiters take part in
@@ -159,28 +160,29 @@ __device__ __forceinline__ Task task_at(const DecSched& sc, int ti) {
   return {static_cast<int>(e >> 14), static_cast<int>(e & 0x3FFFu)};
 }
 
-// q -> bf16(128 + q) - 128 (exact), one 128-byte row of a K-major tile with the 128-byte
-// swizzle (16-byte chunk c of row r lands at chunk c ^ (r mod 8)).
+// q -> bf16(4 + q) (exact: 4 .. 7 need 3 significant bits), one 128-byte row of a K-major tile
+// with the 128-byte swizzle (16-byte chunk c of row r lands at chunk c ^ (r mod 8)).  Columns
+// 2p and 2p + 1 of a word sit at bits 2p and 2p + 16; one shift puts them at bits 5 and 21, the
+// two mantissa bits below the leading one of 4.0 (0x4080), and one AND-OR adds the exponent.
+// The MMA then yields sum_j (4 + q_j) z_j, and the epilogue subtracts 4 sum_j z_j.
+template <int P>
+__device__ __forceinline__ uint32_t code_pair_bf16(uint32_t w) {
+  const uint32_t x = P <= 2 ? (w << (5 - 2 * P)) : (w >> (2 * P - 5));
+  return (x & 0x00600060u) | 0x40804080u;
+}
+
 __device__ __forceinline__ void decode_row_dec(const uint4 w4, uint8_t* tile, int r) {
   const uint32_t wv[4] = {w4.x, w4.y, w4.z, w4.w};
-  const __nv_bfloat162 bias = __floats2bfloat162_rn(128.f, 128.f);
   uint8_t* row = tile + r * 128;
 #pragma unroll
   for (int wi = 0; wi < 4; ++wi) {
-    uint32_t h[8];
-#pragma unroll
-    for (int p = 0; p < 8; ++p) {
-      const uint32_t bits = ((wv[wi] >> (2 * p)) & 0x00030003u) | 0x43004300u;
-      __nv_bfloat162 v = *reinterpret_cast<const __nv_bfloat162*>(&bits);
-      v = __hsub2(v, bias);
-      h[p] = *reinterpret_cast<const uint32_t*>(&v);
-    }
-#pragma unroll
-    for (int half = 0; half < 2; ++half) {
-      const int c = 2 * wi + half;
-      *reinterpret_cast<uint4*>(row + ((c ^ (r & 7)) << 4)) =
-          make_uint4(h[4 * half], h[4 * half + 1], h[4 * half + 2], h[4 * half + 3]);
-    }
+    const uint32_t w = wv[wi];
+    const uint4 lo = make_uint4(code_pair_bf16<0>(w), code_pair_bf16<1>(w), code_pair_bf16<2>(w),
+                                code_pair_bf16<3>(w));
+    const uint4 hi = make_uint4(code_pair_bf16<4>(w), code_pair_bf16<5>(w), code_pair_bf16<6>(w),
+                                code_pair_bf16<7>(w));
+    *reinterpret_cast<uint4*>(row + (((2 * wi) ^ (r & 7)) << 4)) = lo;
+    *reinterpret_cast<uint4*>(row + (((2 * wi + 1) ^ (r & 7)) << 4)) = hi;
   }
 }
 
@@ -521,12 +523,12 @@ __global__ void __launch_bounds__(DecCfg<BN>::kThreads, 1)
         if (!mbar_wait(&mma_done[q], 0, nullptr)) report(a.status, FQ_ERR_TIMEOUT);
       }
     }
-  } else if (warp >= 7 && warp <= 11 && warp != 9) {
+  } else if (warp >= 7 && warp <= 10) {
     // -------------------------------------------------------------- code decoders
-    // Decoder d (warps 7, 8, 10, 11) expands the code blocks of the core rounds that land in
+    // Decoder d (warps 7-10) expands the code blocks of the core rounds that land in
     // ring stages s = d (mod 4) into the stage's A slot; it waits for nothing else.  All lanes
     // wait (measured: one polling lane with the others parked in a shuffle wakes later).
-    const int dw = warp <= 8 ? warp - 7 : warp - 8;
+    const int dw = warp - 7;
     int stage = 0;
     uint32_t cpar = 0;     // bit s: parity of the next cfull[s] phase
     bool ok = true;
@@ -599,6 +601,7 @@ __global__ void __launch_bounds__(DecCfg<BN>::kThreads, 1)
         z_i = __half2float(a.zero[row]);
         if (a.gamma) g_row = a.gamma[row];
       }
+      const float zb_i = z_i - 4.f * s_i;          // the decoded codes carry an offset of 4
       bool fail = false;
       if (t.p == 1) {
         // sum of z over this CTA's K range, from the 16-row group sums of the slices it reads
@@ -668,7 +671,7 @@ __global__ void __launch_bounds__(DecCfg<BN>::kThreads, 1)
         }
 #pragma unroll
         for (int q = 0; q < kChunk; ++q)
-          vals[c + q] = t.p == 1 ? g_row * fmaf(s_i, v[q], z_i * zs_s[c + q]) : v[q];
+          vals[c + q] = t.p == 1 ? g_row * fmaf(s_i, v[q], zb_i * zs_s[c + q]) : v[q];
       }
       tc_fence_before_sync();
       mbar_arrive(&tempty[buf]);
