@@ -87,6 +87,12 @@ __host__ __device__ constexpr int issuer_of(int warp, int ni) {
   return warp == 1 ? 0
                    : (ni == 4 ? (warp == 12 ? 1 : (warp == 14 ? 2 : (warp == 15 ? 3 : -1))) : -1);
 }
+// L2 warming.  When a layer's code blocks fit kL2PrefetchBudget, each CTA prefetches the code
+// blocks of its later tasks after issuing its first task's loads.  When the code blocks and
+// T_out^T fit together, it also prefetches the T_out^T tiles of its synthesis tasks, once it
+// reaches its first code-product task: by then its analysis loads are out, and the code
+// product, bounded by the decode, leaves HBM mostly idle (prefetching them earlier competes with
+// the analysis stream; prefetching part of a larger layer's T_out^T measured no faster).
 constexpr int64_t kL2PrefetchBudget = 64ll << 20;
 
 struct DecPhase {
@@ -107,7 +113,8 @@ struct DecArgs {
   int32_t* status;
   uint32_t* gen;
   uint32_t* done;
-  int prefetch_later;     // 0: none, 1: codes, 2: codes and T_out^T tiles
+  int pf_codes;           // prefetch this CTA's later code blocks into L2
+  int pf_tout;            // prefetch the T_out^T tiles of its synthesis tasks into L2
 };
 
 // Per-cluster task lists, a kernel parameter: cluster c runs task[off[c]] .. task[off[c+1]-1].
@@ -309,7 +316,7 @@ __global__ void __launch_bounds__(DecCfg<BN>::kThreads, 1)
       const uint64_t pol_w = policy_evict_first();
       int stage = 0;
       uint32_t phase = 0;
-      bool first = true;
+      bool first = true, tout_pf = a.pf_tout > 0;
       // bit s: stage s filled / its last fill a code block / parity of that fill's phase of
       // fullA (weight tile) or cfull (code block)
       uint32_t used = 0, last_code = 0, last_par = 0, cpar = 0;
@@ -320,6 +327,23 @@ __global__ void __launch_bounds__(DecCfg<BN>::kThreads, 1)
         const DecPhase ph = phase_of(a, t.p);
         int k0, k1;
         krange(ph, k0, k1);
+        if (tout_pf && t.p >= 1) {
+          tout_pf = false;
+          // this CTA's synthesis tiles, in the order they will be read, into L2
+          for (int j = i; j < t_hi && lane == 0; ++j) {
+            const Task u = task_at(sched, j);
+            if (u.p != 2) continue;
+            const DecPhase q = phase_of(a, u.p);
+            int u0, u1;
+            krange(q, u0, u1);
+            for (int kb = u0; kb < u1; ++kb)
+              asm volatile(
+                  "cp.async.bulk.prefetch.tensor.2d.L2.global.tile [%0, {%1, %2}];" ::"l"(
+                      reinterpret_cast<uint64_t>(&tmTout)),
+                  "r"(kb * kBK), "r"(u.tile * kBM)
+                  : "memory");
+          }
+        }
         for (int kb = k0; kb < k1; ++kb) {
           const bool got = mbar_wait(&empty[stage], phase ^ 1, abort_flag);
           if (!__all_sync(0xffffffffu, got)) {
@@ -355,8 +379,8 @@ __global__ void __launch_bounds__(DecCfg<BN>::kThreads, 1)
         }
         if (first && wok) {
           first = false;
-          // warm L2 with the weight tiles of this CTA's later tasks
-          for (int j = i + 1; j < t_hi && a.prefetch_later > 0 && lane == 0; ++j) {
+          // warm L2 with the code blocks of this CTA's later tasks
+          for (int j = i + 1; j < t_hi && a.pf_codes && lane == 0; ++j) {
             const Task u = task_at(sched, j);
             const DecPhase q = phase_of(a, u.p);
             int u0, u1;
@@ -366,13 +390,6 @@ __global__ void __launch_bounds__(DecCfg<BN>::kThreads, 1)
               asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(src),
                            "r"(static_cast<uint32_t>((u1 - u0) * kCodeBytes))
                            : "memory");
-            } else if (u.p == 2 && a.prefetch_later > 1) {
-              for (int kb = u0; kb < u1; ++kb)
-                asm volatile(
-                    "cp.async.bulk.prefetch.tensor.2d.L2.global.tile [%0, {%1, %2}];" ::"l"(
-                        reinterpret_cast<uint64_t>(&tmTout)),
-                    "r"(kb * kBK), "r"(u.tile * kBM)
-                    : "memory");
             }
           }
         }
@@ -980,6 +997,12 @@ fq_status run(const CUtensorMap* m, DecArgs& a, const int* R, const int* K, int 
     ph.kbs = static_cast<int>(ceil_div(ph.KB, plan->S));
   }
   a.total = total;
+  {
+    const int64_t code_bytes = static_cast<int64_t>(R[1]) * K[1] / 4;
+    const int64_t tout_bytes = static_cast<int64_t>(R[2]) * K[2] * 2;
+    a.pf_codes = code_bytes <= kL2PrefetchBudget;
+    a.pf_tout = code_bytes + tout_bytes <= kL2PrefetchBudget;
+  }
   cudaLaunchConfig_t cfg{};
   cfg.gridDim = dim3(static_cast<unsigned>(plan->ncl * plan->S));
   cfg.blockDim = dim3(DecCfg<BN>::kThreads);
@@ -1041,10 +1064,6 @@ fq_status launch_decode_forward(const void* x, int M, int d_in, const void* T_in
   a.status = reinterpret_cast<int32_t*>(ws);
   a.gen = reinterpret_cast<uint32_t*>(ws + kWsGen);
   a.done = reinterpret_cast<uint32_t*>(ws + kWsDone);
-  const int64_t code_bytes = static_cast<int64_t>(fq_packed_words(n_out, n_in)) * 4;
-  const int64_t tout_bytes = static_cast<int64_t>(d_out) * n_out * 2;
-  a.prefetch_later = code_bytes + tout_bytes <= kL2PrefetchBudget ? 2
-                     : (code_bytes <= kL2PrefetchBudget ? 1 : 0);
 
   CUtensorMap m[5];
   if (!tmap_bf16(&m[0], T_in, n_in, d_in, kBM) || !tmap_bf16(&m[1], x, M, d_in, BN) ||
