@@ -36,11 +36,9 @@ def gpu_frame(k, d, draws):
     return out
 
 
-@pytest.mark.parametrize("name,r,M", [
-    ("q", "1", 16), ("q", "11/10", 1), ("q", "11/10", 16), ("q", "6/5", 16),
-    ("q", "11/10", 128), ("gate", "11/10", 16), ("down", "11/10", 1), ("down", "6/5", 16),
-])
-def test_llama70b_layer(name, r, M):
+def run_layer(name, r, M):
+    """The layer through the C ABI on M tokens: (y on the host, X, the oracle as a function of
+    the tokens it is given)."""
     layer = next(l for l in WK.layers if l.name == name)
     k_in, _ = frames.choose_k(Fraction(r), layer.d_in, RHO)
     k_out, _ = frames.choose_k(Fraction(r), layer.d_out, RHO)
@@ -65,9 +63,35 @@ def test_llama70b_layer(name, r, M):
     fq.fq_linear_forward(x, M, layer.d_in, T_in, C, T_out_t, layer.d_out, None, y, ws, nb)
     assert fq.fq_check(ws) == 0
     got = y.double().cpu().numpy()
+    del T_in, T_out_t, words, x, y, ws
+    torch.cuda.empty_cache()
 
-    Z = frames.analysis_apply(k_in, RHO, layer.d_in, draws_in, X)
-    U = forward.core(Z, codes, scale, zero)
-    ref = frames.synthesis_apply(k_out, RHO, layer.d_out, draws_out, U)
-    err = rel_frobenius(got, ref)
+    def ref(Xs):
+        Z = frames.analysis_apply(k_in, RHO, layer.d_in, draws_in, Xs)
+        U = forward.core(Z, codes, scale, zero)
+        return frames.synthesis_apply(k_out, RHO, layer.d_out, draws_out, U)
+
+    return got, X, ref
+
+
+@pytest.mark.parametrize("name,r,M", [
+    ("q", "1", 16), ("q", "11/10", 1), ("q", "11/10", 16), ("q", "6/5", 16),
+    ("q", "11/10", 128), ("gate", "11/10", 16), ("down", "11/10", 1), ("down", "6/5", 16),
+])
+def test_llama70b_layer(name, r, M):
+    got, X, ref = run_layer(name, r, M)
+    err = rel_frobenius(got, ref(X))
     assert err <= 1e-2, err
+
+
+@pytest.mark.parametrize("name,r,M", [
+    ("q", "11/10", 1024), ("q", "1", 4096), ("gate", "11/10", 4096), ("down", "6/5", 1024),
+])
+def test_llama70b_large_batch_sampled(name, r, M):
+    """The whole batch runs on the GPU (the tensor-core path, 256-token tiles); the oracle
+    checks eight tokens: the first and last of the batch and of token tiles, and the middle."""
+    got, X, ref = run_layer(name, r, M)
+    rows = sorted({0, 1, 255, 256, M // 2, M // 2 + 1, M - 2, M - 1})
+    err = rel_frobenius(got[rows], ref(X[rows]))
+    assert err <= 1e-2, err
+    assert np.isfinite(got).all()
