@@ -21,8 +21,8 @@
 // call's generation (release) once the slice is stored, and the activation producer of a
 // dependent task waits for exactly the slices its K range reads (acquire, bounded, one lane
 // per flag).  No phase waits for the whole grid, and the weight producer runs ahead into the
-// next tasks (and warms L2 with this CTA's later weight tiles) while activations are still
-// being produced.
+// next tasks (and warms L2 with this CTA's later code blocks, and with its synthesis tiles when
+// the layer is small enough) while activations are still being produced.
 //
 // sum(z), needed by the core's zero term, is produced with the analysis output as one sum per
 // 16 columns of z and token, from the bf16 values stored; a core split adds the groups of its
