@@ -24,9 +24,10 @@
 // next tasks (and warms L2 with this CTA's later code blocks, and with its synthesis tiles when
 // the layer is small enough) while activations are still being produced.
 //
-// sum(z), needed by the core's zero term, is produced with the analysis output as one sum per
-// 16 columns of z and token, from the bf16 values stored; a core split adds the groups of its
-// own K range.
+// sum(z), needed by the core's zero term, is taken by the core's epilogue over the bf16 z of its
+// own K range, read from global memory once the slices' ready flags are seen (this runs while
+// the task's MMAs are in flight, and keeps the analysis epilogue, which every core task waits
+// for, short).
 //
 // The workspace header holds the generation counter and the tiles' ready flags; a zero-filled
 // header is a valid start and every call leaves it valid for the next (flags keep
@@ -70,7 +71,6 @@ constexpr int kMaxSplit = 8;
 static_assert(kMaxSplit <= kWsSlices, "one ready flag per slice");
 constexpr int kEpi = 128;
 constexpr int kChunk = 16;
-constexpr int kGroup = 16;                 // columns of z per partial sum
 // MMA issuers per CTA.  A tcgen05.mma with N = 16 or 32 tokens is short, and one thread cannot
 // issue K blocks (waits, MMAs, commit) as fast as the tensor core retires them; NI issuers, one
 // per SM sub-partition, each own the ring stages s = q (mod NI) and accumulate their K blocks
@@ -108,8 +108,6 @@ struct DecArgs {
   const __half* scale;
   const __half* zero;
   const float* gamma;
-  float* zsum;            // [ngroups][M] sums of z over groups of 16 columns
-  int ngroups;
   int32_t* status;
   uint32_t* gen;
   uint32_t* done;
@@ -153,6 +151,10 @@ struct DecLayout {
   static_assert(kAccCols <= 256, "accumulator columns");
   static_assert(kBytes <= 227 * 1024, "shared memory per CTA");
 };
+
+__device__ __forceinline__ uint4 ldcg_u4(const __nv_bfloat16* p) {
+  return __ldcg(reinterpret_cast<const uint4*>(p));
+}
 
 struct Task {
   int p, tile;
@@ -621,7 +623,7 @@ __global__ void __launch_bounds__(DecCfg<BN>::kThreads, 1)
       const float zb_i = z_i - 4.f * s_i;          // the decoded codes carry an offset of 4
       bool fail = false;
       if (t.p == 1) {
-        // sum of z over this CTA's K range, from the 16-row group sums of the slices it reads
+        // sum of z over this CTA's K range: first the ready flags of the slices it reads
         if (has_k) {
           const int sl0 = (k0 * kBK) / rows_per, sl1 = (min(ph.K, k1 * kBK) - 1) / rows_per;
           for (int gs = sl0 + et; gs <= sl1 && !fail; gs += kEpi) {
@@ -634,14 +636,25 @@ __global__ void __launch_bounds__(DecCfg<BN>::kThreads, 1)
           break;
         }
         {
-          // 128 / BN threads per token each add a strided share of the groups, then one
+          // 128 / BN threads per token each add a strided share of the token's z, then one
           // thread per token adds the shares in a fixed order
           constexpr int kPer = kEpi / BN;
           const int q = et % BN, part = et / BN;
           float sz = 0.f;
           if (q < a.M && has_k) {
-            const int g0 = k0 * (kBK / kGroup), g1 = min(a.ngroups, k1 * (kBK / kGroup));
-            for (int gi = g0 + part; gi < g1; gi += kPer) sz += ldcg_f32(a.zsum + gi * a.M + q);
+            // z columns k0 * 64 .. of token q: multiples of 8 (n_in is a multiple of 16), so
+            // 16-byte loads from L2, each thread a strided share
+            const int c0 = k0 * kBK, c1 = min(ph.K, k1 * kBK);
+            const __nv_bfloat16* zr = a.ph[0].out + static_cast<int64_t>(q) * ph.K;
+            for (int c = c0 + 8 * part; c < c1; c += 8 * kPer) {
+              const uint4 w = ldcg_u4(zr + c);
+              const uint32_t wv[4] = {w.x, w.y, w.z, w.w};
+#pragma unroll
+              for (int e = 0; e < 4; ++e) {
+                const float2 f = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&wv[e]));
+                sz += f.x + f.y;
+              }
+            }
           }
           zs_part[part * BN + q] = sz;
           named_barrier_sync(1, kEpi);
@@ -699,14 +712,6 @@ __global__ void __launch_bounds__(DecCfg<BN>::kThreads, 1)
         for (int c = 0; c < BN; ++c) {
           const __nv_bfloat16 b = __float2bfloat16_rn(vals[c]);
           if (row_ok && c < a.M) ph.out[static_cast<int64_t>(c) * ph.R + row] = b;
-          if (t.p == 0) {
-            // 16 consecutive rows = 16 consecutive lanes
-            float sv = row_ok ? __bfloat162float(b) : 0.f;
-#pragma unroll
-            for (int off = 8; off > 0; off >>= 1) sv += __shfl_xor_sync(0xffffffffu, sv, off);
-            const int grp = row / kGroup;
-            if ((lane & 15) == 0 && c < a.M && grp < a.ngroups) a.zsum[grp * a.M + c] = sv;
-          }
         }
         if (t.p < 2) {
           named_barrier_sync(1, kEpi);
@@ -765,13 +770,6 @@ __global__ void __launch_bounds__(DecCfg<BN>::kThreads, 1)
             const int tok = 4 * tg + u;
             const __nv_bfloat16 b = __float2bfloat16_rn(o[u]);
             if (ok_r && tok < a.M) ph.out[static_cast<int64_t>(tok) * ph.R + orow] = b;
-            if (t.p == 0) {
-              float sv = ok_r ? __bfloat162float(b) : 0.f;
-#pragma unroll
-              for (int off = 8; off > 0; off >>= 1) sv += __shfl_xor_sync(0xffffffffu, sv, off);
-              const int grp = orow / kGroup;
-              if ((lane & 15) == 0 && tok < a.M && grp < a.ngroups) a.zsum[grp * a.M + tok] = sv;
-            }
           }
         }
         if (t.p < 2) {
@@ -840,7 +838,7 @@ bool tmap_bf16(CUtensorMap* m, const void* base, int64_t rows, int64_t cols, int
 int decode_bn(int M) { return M <= 16 ? 16 : (M <= 32 ? 32 : 64); }
 
 struct DecWs {
-  size_t z, u, zsum, total;
+  size_t z, u, total;
 };
 
 DecWs dec_ws(int M, int n_in, int n_out) {
@@ -850,8 +848,6 @@ DecWs dec_ws(int M, int n_in, int n_out) {
   off += round_up(static_cast<int64_t>(M) * n_in * 2, 256);
   L.u = off;
   off += round_up(static_cast<int64_t>(M) * n_out * 2, 256);
-  L.zsum = off;
-  off += round_up(ceil_div(n_in, kGroup) * M * 4, 256);
   L.total = off;
   return L;
 }
@@ -1059,8 +1055,6 @@ fq_status launch_decode_forward(const void* x, int M, int d_in, const void* T_in
   a.scale = reinterpret_cast<const __half*>(Cq.scale);
   a.zero = reinterpret_cast<const __half*>(Cq.zero);
   a.gamma = gamma;
-  a.zsum = reinterpret_cast<float*>(ws + L.zsum);
-  a.ngroups = static_cast<int>(ceil_div(n_in, kGroup));
   a.status = reinterpret_cast<int32_t*>(ws);
   a.gen = reinterpret_cast<uint32_t*>(ws + kWsGen);
   a.done = reinterpret_cast<uint32_t*>(ws + kWsDone);
