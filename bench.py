@@ -195,14 +195,31 @@ class Regime:
                        for L in self.layers)
         self.ws_bytes = ws_bytes
         self.ws = torch.zeros(ws_bytes, dtype=torch.uint8, device=dev)
-        for L, layer in zip(self.layers, self.wk.layers):
+        # The step's activations and outputs live in one device buffer each (every layer a
+        # 256-byte aligned slice), mirrored by one pinned host buffer each, so a step moves its
+        # inputs in one host-to-device copy and its results in one device-to-host copy.
+        def offsets(sizes):
+            offs, tot = [], 0
+            for n in sizes:
+                offs.append(tot)
+                tot += -(-n // 128) * 128
+            return offs, tot
+        xo, xt = offsets([M * L["d_in"] for L in self.layers])
+        yo, yt = offsets([M * L["d_out"] for L in self.layers])
+        self.x_all = torch.zeros(xt, dtype=torch.bfloat16, device=dev)
+        self.y_all = torch.zeros(yt, dtype=torch.bfloat16, device=dev)
+        self.x_host_all = torch.zeros(xt, dtype=torch.bfloat16).pin_memory()
+        self.y_host_all = torch.zeros(yt, dtype=torch.bfloat16).pin_memory()
+        for L, layer, x0, y0 in zip(self.layers, self.wk.layers, xo, yo):
             X = wl.activations(self.wk, layer, M)
             if rank:
                 X = wl.round_bf16(wl.rng(rank, wl_key, layer.name, "X-rank").standard_normal(X.shape))
-            L["x"] = torch.from_numpy(X).to(dev, torch.bfloat16)
-            L["y"] = torch.empty(M, L["d_out"], dtype=torch.bfloat16, device=dev)
-            L["x_host"] = torch.from_numpy(X).to(torch.bfloat16).pin_memory()
-            L["y_host"] = torch.empty(M, L["d_out"], dtype=torch.bfloat16).pin_memory()
+            L["x_host"] = self.x_host_all[x0:x0 + M * L["d_in"]].view(M, L["d_in"])
+            L["x_host"].copy_(torch.from_numpy(X).to(torch.bfloat16))
+            L["x"] = self.x_all[x0:x0 + M * L["d_in"]].view(M, L["d_in"])
+            L["x"].copy_(L["x_host"])
+            L["y"] = self.y_all[y0:y0 + M * L["d_out"]].view(M, L["d_out"])
+            L["y_host"] = self.y_host_all[y0:y0 + M * L["d_out"]].view(M, L["d_out"])
         # one eager call per layer before any capture (sets kernel attributes, checks status)
         for L in self.layers:
             self.forward(L, torch.cuda.current_stream(dev).cuda_stream)
@@ -211,23 +228,30 @@ class Regime:
                 raise RuntimeError(f"{L['name']}: {fq.fq_status_str(st)}")
         torch.cuda.synchronize()
 
-    def forward(self, L, stream, host=False):
-        fq, torch = self.fq, self.torch
-        if host:
-            L["x"].copy_(L["x_host"], non_blocking=True)
+    def forward(self, L, stream):
+        fq = self.fq
         fq.fq_linear_forward(L["x"], self.M, L["d_in"], L["T_in"], L["C"], L["T_out_t"],
                              L["d_out"], L["gamma"] if self.use_gamma else None, L["y"],
                              self.ws, self.ws_bytes, fq.FQ_BF16, stream)
-        if host:
-            L["y_host"].copy_(L["y"], non_blocking=True)
 
     def capture(self, layers, stream, host=False):
+        """One graph: the layers' forwards in order; with host=True (all layers) the step's
+        inputs come from pinned host memory first and its results go back at the end."""
         torch = self.torch
+        assert not host or layers is self.layers
         g = torch.cuda.CUDAGraph()
         with torch.cuda.graph(g, stream=stream):
+            if host:
+                self.x_all.copy_(self.x_host_all, non_blocking=True)
             for L in layers:
-                self.forward(L, stream.cuda_stream, host)
+                self.forward(L, stream.cuda_stream)
+            if host:
+                self.y_host_all.copy_(self.y_all, non_blocking=True)
         return g
+
+    def host_bytes(self):
+        """Bytes one host-backed step copies in and out."""
+        return self.x_all.numel() * 2, self.y_all.numel() * 2
 
     def bytes_flops(self, L):
         args = (L["d_in"], L["d_out"], L["n_in"], L["n_out"], self.M)
@@ -527,8 +551,7 @@ def main(argv=None):
                               args.warmup)
     e2e_ms = max_over_ranks(e2e_ms, dist, dev)
     e2e_us = aggregate(e2e_ms, max(100, args.steps // 4), nL, world)
-    h2d = sum(L["x"].numel() * 2 for L in dec.layers)
-    d2h = sum(L["y"].numel() * 2 for L in dec.layers)
+    h2d, d2h = dec.host_bytes()
 
     per_layer = {L["name"]: {"us": round(per_ms[i] * 1e3, 2),
                              "GBps": round(bytes_fl[i][0] / (per_ms[i] * 1e-3) / 1e9, 1),
@@ -583,7 +606,9 @@ def main(argv=None):
             "per_layer": per_layer,
         },
         "e2e": {"value": round(e2e_us, 3), "unit": UNIT, "h2d_bytes_per_step": h2d,
-                "d2h_bytes_per_step": d2h},
+                "d2h_bytes_per_step": d2h,
+                "copies": ("per step: one host-to-device copy of the 7 layers' inputs from pinned "
+                           "memory, the 7 forwards, one device-to-host copy of their outputs")},
         "gpu_launches": nL * args.steps,      # one fused kernel per layer forward (M <= 64)
         "clocks": clocks,
         "prefill": prefill,
