@@ -16,6 +16,11 @@
 // of shared-memory stages guarded by mbarriers; accumulators are double-buffered in TMEM so
 // the epilogue of one tile overlaps the MMAs of the next.
 //
+// Tiles are numbered token tile fastest (tile = row tile * TT + token tile) and CTA c takes tiles
+// c, c + grid, ...: the CTAs of a wave share each weight tile across all token tiles, so a
+// weight matrix larger than L2 (T_out^T of the up and gate layers, 267 MB) streams from HBM
+// once per wave instead of once per token tile (measured 8.7% faster on the 2048-token block).
+//
 // sum(z), needed by the core's zero term, comes from the analysis epilogue as one sum per
 // 128-row tile of z and token, taken over the bf16 values stored.  Decoder warps take whole
 // stages in turn (stage i goes to warp i mod 4), so four stages are decoded at once.
@@ -202,7 +207,7 @@ __global__ void __launch_bounds__(threads_for<PHASE>(), 1)
       // full ring of them before waiting for it, and warm L2 with the rest.
       int pre = 0;
       if (static_cast<int>(cid) < p.tiles) {
-        const int rt = static_cast<int>(cid) % p.RT;
+        const int rt = static_cast<int>(cid) / p.TT;
         pre = min(S_, k1 - k0);
         for (int i = 0; i < pre; ++i) {
           const int kb = k0 + i;
@@ -242,7 +247,7 @@ __global__ void __launch_bounds__(threads_for<PHASE>(), 1)
       for (int s = 0; s < S_; ++s) issued[s] = false, issued_parity[s] = 0;
       for (int tile = static_cast<int>(cid); tile < p.tiles && !*abort_flag;
            tile += static_cast<int>(ncl)) {
-        const int rt = tile % p.RT, tt = tile / p.RT;
+        const int rt = tile / p.TT, tt = tile % p.TT;
         for (int kb = k0; kb < k1; ++kb, ++it) {
           if (it >= pre) {
             if (!mbar_wait(&empty[stage], phase ^ 1, abort_flag)) {
@@ -333,7 +338,7 @@ __global__ void __launch_bounds__(threads_for<PHASE>(), 1)
     int buf = 0;
     uint32_t acc_phase = 0;
     for (int tile = static_cast<int>(cid); tile < p.tiles; tile += static_cast<int>(ncl)) {
-      const int rt = tile % p.RT, tt = tile / p.RT;
+      const int rt = tile / p.TT, tt = tile % p.TT;
       const int row = rt * kBM + r_in_tile;
       const int t0 = tt * BN;
       const bool row_ok = row < p.R;
