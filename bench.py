@@ -252,6 +252,47 @@ class Regime:
                 self.y_host_all.copy_(self.y_all, non_blocking=True)
         return g
 
+    def capture_grouped(self, groups, stream):
+        """One graph of all layers with the independent layers of a group side by side: group
+        members run on their own streams and workspaces, each on `budget` SMs
+        (fq_linear_forward_sms); the groups run in order."""
+        torch, fq = self.torch, self.fq
+        by_name = {L["name"]: L for L in self.layers}
+        width = max(len(names) for names, _ in groups)
+        if not hasattr(self, "group_ws"):
+            self.group_ws = [self.ws] + [torch.zeros(self.ws_bytes, dtype=torch.uint8,
+                                                     device=self.dev) for _ in range(width - 1)]
+        side = [torch.cuda.Stream(device=self.dev) for _ in range(width - 1)]
+
+        def launch(names, budget, streams):
+            for name, st, ws in zip(names, streams, self.group_ws):
+                L = by_name[name]
+                fq.fq_linear_forward_sms(L["x"], self.M, L["d_in"], L["T_in"], L["C"],
+                                         L["T_out_t"], L["d_out"],
+                                         L["gamma"] if self.use_gamma else None, L["y"], ws,
+                                         self.ws_bytes, budget, fq.FQ_BF16, st.cuda_stream)
+
+        for names, budget in groups:             # eager calls: plans for each budget, status
+            launch(names, budget, [stream] + side)
+            torch.cuda.synchronize()
+            for ws in self.group_ws[:len(names)]:
+                st = fq.fq_check(ws)
+                if st != 0:
+                    raise RuntimeError(f"group {names}: {fq.fq_status_str(st)}")
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, stream=stream):
+            for names, budget in groups:
+                fork = torch.cuda.Event()
+                fork.record(stream)
+                for st in side[:len(names) - 1]:
+                    st.wait_event(fork)
+                launch(names, budget, [stream] + side)
+                for st in side[:len(names) - 1]:
+                    join = torch.cuda.Event()
+                    join.record(st)
+                    stream.wait_event(join)
+        return g
+
     def host_bytes(self):
         """Bytes one host-backed step copies in and out."""
         return self.x_all.numel() * 2, self.y_all.numel() * 2
@@ -548,6 +589,24 @@ def main(argv=None):
     achieved = dom_bytes / (per_ms[dom] * 1e-3) / 1e9
     step_bytes = sum(b for b, _ in bytes_fl)
 
+    # the same block with independent layers side by side (q|k|v, o, gate|up, down)
+    sms = torch.cuda.get_device_properties(dev).multi_processor_count
+    groups = [(["q", "k", "v"], sms // 3), (["o"], 0), (["gate", "up"], sms // 2),
+              (["down"], 0)]
+    grouped_graph = dec.capture_grouped(groups, stream)
+    barrier()
+    grp_ms, _ = timed_replays(torch, [grouped_graph], stream, args.steps, args.warmup)
+    grp_ms = max_over_ranks(grp_ms, dist, dev)
+    grp_us = aggregate(grp_ms, args.steps, nL, world)
+    grouped = {
+        "value": round(grp_us, 3), "unit": UNIT, "ms_per_step": round(grp_ms / args.steps, 4),
+        "groups": " ; ".join(f"{'|'.join(n)}@{b or sms} SMs" for n, b in groups),
+        "how": ("fq_linear_forward_sms: the layers of a group run on parallel streams, each "
+                "with its own workspace and SM budget; groups run in order; one CUDA graph "
+                "per step"),
+    }
+    del grouped_graph
+
     # end to end through the C ABI with host buffers
     barrier()
     e2e_ms, _ = timed_replays(torch, [e2e_graph], stream, max(100, args.steps // 4),
@@ -608,6 +667,7 @@ def main(argv=None):
             "step_frac": round(roof_us / us_layer, 3),
             "per_layer": per_layer,
         },
+        "grouped": grouped,
         "e2e": {"value": round(e2e_us, 3), "unit": UNIT, "h2d_bytes_per_step": h2d,
                 "d2h_bytes_per_step": d2h,
                 "copies": ("per step: one host-to-device copy of the 7 layers' inputs from pinned "

@@ -124,6 +124,23 @@ fq_status fq_linear_forward(const void* x, int M, int d_in, const void* T_in,
                             const float* gamma, void* y, void* ws, size_t ws_bytes, int mode,
                             fq_stream_t stream);
 
+/* fq_linear_forward on at most max_sms SMs (0: all of them), so that independent layers
+ * (q, k and v of an attention block, or gate and up of an MLP, which read the same input) can
+ * run side by side on different streams, each with its own workspace.  The grid and the plan
+ * of the FQ_BF16 kernels are sized for the budget (one CTA per SM); FQ_FP32_DEBUG ignores it.
+ * For M <= 64 the CTAs of one call wait on one another's partial results, so every CTA of the
+ * call must be resident at once.  Such a call takes clusters of CTAs in proportion to its
+ * budget's share of the SM count (a GPC holds a whole number of clusters), so that calls whose
+ * budgets add up to no more than the device's SM count are resident together.  Calls whose
+ * budgets overcommit the device, or that share it with other work holding SMs, can stall one
+ * another until a bounded wait runs out (FQ_ERR_TIMEOUT through fq_check).
+ * Errors: those of fq_linear_forward, and FQ_ERR_INVALID_ARG for max_sms < 0.  This entry
+ * point has no counterpart in the paper. */
+fq_status fq_linear_forward_sms(const void* x, int M, int d_in, const void* T_in,
+                                const fq_packed* C, const void* T_out_t, int d_out,
+                                const float* gamma, void* y, void* ws, size_t ws_bytes, int mode,
+                                int max_sms, fq_stream_t stream);
+
 /* ------------------------------------------------------------------------------------------
  * Offline preparation of a layer (not on the inference path).  These produce the inputs of
  * fq_linear_forward on the device from a weight matrix W and the frame parameters.

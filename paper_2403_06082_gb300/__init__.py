@@ -15,7 +15,8 @@ from dataclasses import dataclass
 
 __all__ = [
     "FQ_BF16", "FQ_FP32_DEBUG", "FrameQuantError", "Packed", "lib", "lib_path",
-    "fq_packed_words", "fq_pack", "fq_workspace_bytes", "fq_linear_forward", "fq_check",
+    "fq_packed_words", "fq_pack", "fq_workspace_bytes", "fq_linear_forward",
+    "fq_linear_forward_sms", "fq_check",
     "fq_status_str", "EXPORTED", "fq_frame_workspace_bytes", "fq_frame_build",
     "fq_coefficients_workspace_bytes", "fq_coefficients", "fq_quantize_rtn",
     "fq_linear_forward_static", "FQ_STATIC_SCRATCH_BYTES",
@@ -28,6 +29,7 @@ STATUS = {0: "FQ_OK", 1: "FQ_ERR_INVALID_ARG", 2: "FQ_ERR_ALIGNMENT", 3: "FQ_ERR
           4: "FQ_ERR_WORKSPACE", 5: "FQ_ERR_CUDA", 6: "FQ_ERR_TIMEOUT",
           7: "FQ_ERR_DEVICE_CHECK"}
 EXPORTED = ("fq_packed_words", "fq_pack", "fq_workspace_bytes", "fq_linear_forward",
+            "fq_linear_forward_sms",
             "fq_check", "fq_status_str", "fq_frame_workspace_bytes", "fq_frame_build",
             "fq_coefficients_workspace_bytes", "fq_coefficients", "fq_quantize_rtn",
             "fq_linear_forward_static")
@@ -80,6 +82,12 @@ def lib() -> ctypes.CDLL:
             ctypes.c_void_p, ctypes.c_int, ctypes.c_int, ctypes.c_void_p,
             ctypes.POINTER(_Packed), ctypes.c_void_p, ctypes.c_int, ctypes.c_void_p,
             ctypes.c_void_p, ctypes.c_void_p, ctypes.c_size_t, ctypes.c_int, ctypes.c_void_p]
+        L.fq_linear_forward_sms.restype = ctypes.c_int
+        L.fq_linear_forward_sms.argtypes = [
+            ctypes.c_void_p, ctypes.c_int, ctypes.c_int, ctypes.c_void_p,
+            ctypes.POINTER(_Packed), ctypes.c_void_p, ctypes.c_int, ctypes.c_void_p,
+            ctypes.c_void_p, ctypes.c_void_p, ctypes.c_size_t, ctypes.c_int, ctypes.c_int,
+            ctypes.c_void_p]
         L.fq_check.restype = ctypes.c_int
         L.fq_check.argtypes = [ctypes.c_void_p, ctypes.c_void_p]
         L.fq_status_str.restype = ctypes.c_char_p
@@ -165,6 +173,18 @@ def fq_linear_forward(x, M: int, d_in: int, T_in, C: Packed, T_out_t, d_out: int
     _ok(lib().fq_linear_forward(_ptr(x), M, d_in, _ptr(T_in), ctypes.byref(pc), _ptr(T_out_t),
                                 d_out, _ptr(gamma), _ptr(y), _ptr(ws), ws_bytes, mode,
                                 _stream(stream)), "fq_linear_forward")
+
+
+def fq_linear_forward_sms(x, M: int, d_in: int, T_in, C: Packed, T_out_t, d_out: int, gamma,
+                          y, ws, ws_bytes: int, max_sms: int, mode: int = FQ_BF16,
+                          stream=None) -> None:
+    """fq_linear_forward on at most max_sms SMs (0: all), for independent layers run side by
+    side on different streams; budgets of concurrent calls must fit the device together."""
+    pc = C._c()
+    _ok(lib().fq_linear_forward_sms(_ptr(x), M, d_in, _ptr(T_in), ctypes.byref(pc),
+                                    _ptr(T_out_t), d_out, _ptr(gamma), _ptr(y), _ptr(ws),
+                                    ws_bytes, mode, max_sms, _stream(stream)),
+        "fq_linear_forward_sms")
 
 
 def fq_linear_forward_static(x, M: int, d_in: int, T_in, C: Packed, T_out_t, d_out: int, gamma,

@@ -937,10 +937,10 @@ struct Plan {
 // K blocks over the three phases, with a fixed cost per task (pipeline fill and drain,
 // reduction) and code blocks weighted by their smaller bytes.
 template <int BN>
-const Plan* plan_for(int dev, int sms, const int* R, const int* K) {
+const Plan* plan_for(int dev, int sms, int budget, const int* R, const int* K) {
   static std::mutex mu;
-  static std::map<std::array<int, 7>, Plan> cache;
-  const std::array<int, 7> key{dev, R[0], R[1], R[2], K[0], K[1], K[2]};
+  static std::map<std::array<int, 8>, Plan> cache;
+  const std::array<int, 8> key{dev, R[0], R[1], R[2], K[0], K[1], K[2], budget};
   std::lock_guard<std::mutex> g(mu);
   const auto it = cache.find(key);
   if (it != cache.end()) return &it->second;
@@ -949,7 +949,13 @@ const Plan* plan_for(int dev, int sms, const int* R, const int* K) {
   Plan best;
   double best_cost = 1e30;
   for (int S : {1, 2, 4, 8}) {
-    int ncl = S == 1 ? sms : max_clusters<BN>(dev, S);
+    // A budget below the SM count takes its share of the device's resident clusters, so
+    // that calls whose budgets add up to at most the SM count are resident together.
+    int ncl = budget;
+    if (S > 1) {
+      const int mc = max_clusters<BN>(dev, S);
+      ncl = budget >= sms ? mc : static_cast<int>(static_cast<int64_t>(mc) * budget / sms);
+    }
     ncl = std::min({ncl, total, kMaxClusters});
     if (ncl <= 0) continue;
     double cost = 0;
@@ -972,7 +978,7 @@ const Plan* plan_for(int dev, int sms, const int* R, const int* K) {
 
 template <int BN>
 fq_status run(const CUtensorMap* m, DecArgs& a, const int* R, const int* K, int sms,
-              cudaStream_t s) {
+              int budget, cudaStream_t s) {
   int dev = 0;
   cudaGetDevice(&dev);
   if (prepare<BN>(dev) != cudaSuccess) return FQ_ERR_CUDA;
@@ -983,7 +989,7 @@ fq_status run(const CUtensorMap* m, DecArgs& a, const int* R, const int* K, int 
     total += RT;
   }
   if (total > kMaxSched) return FQ_ERR_UNSUPPORTED;
-  const Plan* plan = plan_for<BN>(dev, sms, R, K);
+  const Plan* plan = plan_for<BN>(dev, sms, budget, R, K);
   if (!plan) return FQ_ERR_CUDA;
   a.S = plan->S;
   for (int p = 0; p < 3; ++p) {
@@ -1030,7 +1036,7 @@ size_t decode_workspace_bytes(int M, int d_in, int n_in, int n_out, int d_out) {
 fq_status launch_decode_forward(const void* x, int M, int d_in, const void* T_in,
                                 const fq_packed& Cq, const void* T_out_t, int d_out,
                                 const float* gamma, void* y, char* ws, size_t ws_bytes,
-                                cudaStream_t s) {
+                                int max_sms, cudaStream_t s) {
   const int n_in = Cq.n_in, n_out = Cq.n_out;
   const DecWs L = dec_ws(M, n_in, n_out);
   if (ws_bytes < L.total) return FQ_ERR_WORKSPACE;
@@ -1039,6 +1045,7 @@ fq_status launch_decode_forward(const void* x, int M, int d_in, const void* T_in
   cudaGetDevice(&dev);
   cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
   if (sms <= 0) return FQ_ERR_CUDA;
+  const int budget = max_sms > 0 ? std::min(sms, max_sms) : sms;
 
   DecArgs a{};
   a.M = M;
@@ -1065,9 +1072,9 @@ fq_status launch_decode_forward(const void* x, int M, int d_in, const void* T_in
       !tmap_bf16(&m[3], T_out_t, d_out, n_out, kBM) || !tmap_bf16(&m[4], ws + L.u, M, n_out, BN))
     return FQ_ERR_CUDA;
   switch (BN) {
-    case 16: return run<16>(m, a, R, K, sms, s);
-    case 32: return run<32>(m, a, R, K, sms, s);
-    default: return run<64>(m, a, R, K, sms, s);
+    case 16: return run<16>(m, a, R, K, sms, budget, s);
+    case 32: return run<32>(m, a, R, K, sms, budget, s);
+    default: return run<64>(m, a, R, K, sms, budget, s);
   }
 }
 

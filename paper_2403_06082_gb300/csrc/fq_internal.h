@@ -46,16 +46,17 @@ cudaError_t launch_debug_forward(const float* x, int M, int d_in, const float* T
 
 // ---- fq_decode.cu: bf16 path for small batches (one fused persistent kernel)
 size_t decode_workspace_bytes(int M, int d_in, int n_in, int n_out, int d_out);
+// max_sms > 0 caps the SMs a call's kernels occupy (the grid and the plan)
 fq_status launch_decode_forward(const void* x, int M, int d_in, const void* T_in,
                                 const fq_packed& C, const void* T_out_t, int d_out,
                                 const float* gamma, void* y, char* ws, size_t ws_bytes,
-                                cudaStream_t s);
+                                int max_sms, cudaStream_t s);
 
 // ---- fq_tc.cu: bf16 tensor-core path
 size_t tc_workspace_bytes(int M, int d_in, int n_in, int n_out, int d_out);
 fq_status launch_tc_forward(const void* x, int M, int d_in, const void* T_in,
                             const fq_packed& C, const void* T_out_t, int d_out,
                             const float* gamma, void* y, char* ws, size_t ws_bytes,
-                            cudaStream_t s);
+                            int max_sms, cudaStream_t s);
 
 }  // namespace fq

@@ -561,8 +561,9 @@ cudaError_t launch_phase(const CUtensorMap& tmA, const CUtensorMap& tmB, const P
 // maps: {T_in, x, z, T_out^T, u}.  The core phase's A operand is the packed codes, so it gets
 // an unused map in that slot.
 template <int BN>
-fq_status run_forward(const CUtensorMap* maps, PhaseArgs* a, cudaStream_t s) {
-  const DeviceInfo d = device_info();
+fq_status run_forward(const CUtensorMap* maps, PhaseArgs* a, int max_sms, cudaStream_t s) {
+  DeviceInfo d = device_info();
+  if (max_sms > 0) d.sms = std::min(d.sms, max_sms);
   if (prepare_kernel<kAnalysis, BN>(d.dev) != cudaSuccess ||
       prepare_kernel<kCore, BN>(d.dev) != cudaSuccess ||
       prepare_kernel<kSynthesis, BN>(d.dev) != cudaSuccess)
@@ -590,7 +591,7 @@ size_t tc_workspace_bytes(int M, int d_in, int n_in, int n_out, int d_out) {
 fq_status launch_tc_forward(const void* x, int M, int d_in, const void* T_in,
                             const fq_packed& Cq, const void* T_out_t, int d_out,
                             const float* gamma, void* y, char* ws, size_t ws_bytes,
-                            cudaStream_t s) {
+                            int max_sms, cudaStream_t s) {
   const int n_in = Cq.n_in, n_out = Cq.n_out;
   const WsLayout L = ws_layout(M, n_in, n_out);
   if (ws_bytes < L.total) return FQ_ERR_WORKSPACE;
@@ -625,7 +626,7 @@ fq_status launch_tc_forward(const void* x, int M, int d_in, const void* T_in,
       !make_tmap(&maps[4], u, M, n_out, BN))
     return FQ_ERR_CUDA;
 
-  return BN == 128 ? run_forward<128>(maps, a, s) : run_forward<256>(maps, a, s);
+  return BN == 128 ? run_forward<128>(maps, a, max_sms, s) : run_forward<256>(maps, a, max_sms, s);
 }
 
 }  // namespace fq
