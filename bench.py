@@ -492,6 +492,189 @@ def prefill_only(args, fq, wl, torch, dev, rank, world, dist, stream, peaks):
         dist.destroy_process_group()
 
 
+# --------------------------------------------------------------------------- structured frames
+def measure_implicit(args, fq, wl, torch, dec, stream, peaks):
+    """The decode block with T_in and T_out in structured form: one CUDA graph of the seven
+    fq_linear_forward_implicit calls on the regime's tokens, codes and workspace."""
+    wk, dev, M = dec.wk, dec.dev, dec.M
+    frames, bytes_ = [], 0
+    for L, layer in zip(dec.layers, wk.layers):
+        def fr(side, d, k):
+            dr = wl.rotation_draws(wk.seed, wk.key, layer.name, side, d=d)
+            return fq.fq_frame_implicit(k, RHO, d, (dr.a, dr.b, dr.ga, dr.gb, dr.perm, dr.signs),
+                                        dev)
+        Fi, Fo = fr("in", L["d_in"], L["k_in"]), fr("out", L["d_out"], L["k_out"])
+        frames.append((Fi, Fo))
+        bytes_ += (L["n_out"] * L["n_in"] // 4 + 4 * L["n_out"] + 2 * M * (L["d_in"] + L["d_out"])
+                   + Fi.buf.numel() + Fo.buf.numel())
+    nb = max(fq.fq_implicit_workspace_bytes(M, L["d_in"], L["n_in"], L["n_out"], L["d_out"])
+             for L in dec.layers)
+    ws = torch.zeros(nb, dtype=torch.uint8, device=dev)
+
+    def step(st):
+        for L, (Fi, Fo) in zip(dec.layers, frames):
+            fq.fq_linear_forward_implicit(L["x"], M, Fi, L["C"], Fo, None, L["y"], ws, nb, 0,
+                                          st.cuda_stream)
+
+    step(stream)
+    torch.cuda.synchronize()
+    if fq.fq_check(ws) != 0:
+        raise RuntimeError("implicit block: device status")
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g, stream=stream):
+        step(stream)
+    steps = max(50, args.steps // 4)
+    ms, _ = timed_replays(torch, [g], stream, steps, args.warmup)
+    if fq.fq_check(ws) != 0:
+        raise RuntimeError("implicit block: device status after timing")
+    us = ms * 1e3 / (steps * len(dec.layers))
+    roof_us = bytes_ / (peaks["hbm_gbs"] * 1e9) * 1e6 / len(dec.layers)
+    del g
+    return {
+        "value": round(us, 3), "unit": UNIT, "steps": steps,
+        "bytes_per_layer": round(bytes_ / len(dec.layers)),
+        "hbm_frac": round(roof_us / us, 3),
+        "kernels_per_layer": 5,
+        "how": ("fq_linear_forward_implicit: rotation, run transforms (fp32, CUDA cores) and the "
+                "fused kernel's code product; frames as rotation factors and roots of unity"),
+    }
+
+
+# --------------------------------------------------------------------------- sweep
+def prepare_layer_random_codes(fq, wl, torch, wk, layer, r, dev):
+    """Like prepare_layer, with seeded uniform codes and scale/zero in place of the real frame
+    coefficients (the kernels' work does not depend on the code values; computing C for the
+    70B shapes takes seconds of fp32 GEMM per layer)."""
+    import numpy as np
+    k_in, k_out = wl.k_for(r, layer.d_in), wl.k_for(r, layer.d_out)
+    n_in, n_out = k_in * RHO, k_out * RHO
+
+    def frame(k, d, side):
+        dr = wl.rotation_draws(wk.seed, wk.key, layer.name, side, d=d)
+        nb = fq.fq_frame_workspace_bytes(k, RHO, d, dr.a, dr.b)
+        ws = torch.empty(nb, dtype=torch.uint8, device=dev)
+        T = torch.empty(k * RHO, d, dtype=torch.float32, device=dev)
+        fq.fq_frame_build(k, RHO, d, (dr.a, dr.b, dr.ga, dr.gb, dr.perm, dr.signs), T, ws, nb)
+        return T
+
+    T_in = frame(k_in, layer.d_in, "in").to(torch.bfloat16)
+    T_out_t = frame(k_out, layer.d_out, "out").t().contiguous().to(torch.bfloat16)
+    torch.cuda.empty_cache()
+    codes = torch.from_numpy(wl.random_codes(wk.seed, wk.key, layer.name, str(r), n_out=n_out,
+                                             n_in=n_in)).to(dev)
+    words = torch.empty(fq.fq_packed_words(n_out, n_in), dtype=torch.int32, device=dev)
+    fq.fq_pack(codes, n_out, n_in, words)
+    del codes
+    sc, ze = wl.random_scale_zero(wk.seed, wk.key, layer.name, n_out=n_out, mag=0.01)
+    scale = torch.from_numpy(sc.view(np.int16)).to(dev)
+    zero = torch.from_numpy(ze.view(np.int16)).to(dev)
+    gamma = torch.ones(n_out, dtype=torch.float32, device=dev)
+    return {
+        "name": layer.name, "d_in": layer.d_in, "d_out": layer.d_out, "n_in": n_in,
+        "n_out": n_out, "k_in": k_in, "k_out": k_out, "T_in": T_in, "T_out_t": T_out_t,
+        "C": fq.Packed(words, scale, zero, n_out, n_in), "gamma": gamma,
+    }
+
+
+def time_layer(fq, torch, L, X, use_gamma, dev, stream, flush, reps=30, warm_calls=20):
+    """Cold time (median over `reps` calls, each after writing a buffer twice the size of L2,
+    CUDA events around the call alone) and warm time (`warm_calls` calls back to back in one
+    CUDA graph, total / calls) of one layer forward, in microseconds."""
+    M = X.shape[0]
+    x = X if X.is_cuda else X.to(dev)
+    y = torch.empty(M, L["d_out"], dtype=torch.bfloat16, device=dev)
+    nb = fq.fq_workspace_bytes(M, L["d_in"], L["n_in"], L["n_out"], L["d_out"], 0)
+    ws = torch.zeros(nb, dtype=torch.uint8, device=dev)
+    g = L["gamma"] if use_gamma else None
+
+    def call():
+        fq.fq_linear_forward(x, M, L["d_in"], L["T_in"], L["C"], L["T_out_t"], L["d_out"], g,
+                             y, ws, nb, fq.FQ_BF16, stream.cuda_stream)
+
+    with torch.cuda.stream(stream):
+        for _ in range(3):
+            call()
+    torch.cuda.synchronize()
+    st = fq.fq_check(ws)
+    if st != 0:
+        raise RuntimeError(f"{L['name']} M={M}: {fq.fq_status_str(st)}")
+    cold = []
+    with torch.cuda.stream(stream):
+        for _ in range(reps):
+            flush.add_(1)
+            e0 = torch.cuda.Event(enable_timing=True)
+            e1 = torch.cuda.Event(enable_timing=True)
+            e0.record(stream)
+            call()
+            e1.record(stream)
+            cold.append((e0, e1))
+    torch.cuda.synchronize()
+    cold_us = statistics.median(a.elapsed_time(b) for a, b in cold) * 1e3
+    gr = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(gr, stream=stream):
+        for _ in range(warm_calls):
+            call()
+    warm_ms, _ = timed_replays(torch, [gr], stream, 3, 3)
+    warm_us = warm_ms * 1e3 / (3 * warm_calls)
+    if fq.fq_check(ws) != 0:
+        raise RuntimeError(f"{L['name']} M={M}: device status after timing")
+    del gr
+    return cold_us, warm_us
+
+
+def sweep(args, fq, wl, torch, dev, stream, peaks):
+    """--sweep: every configuration of the workload set, one layer shape at a time: cold and
+    warm microseconds per layer, tokens/s and the fraction of the roofline
+    max(bytes / HBM peak, FLOPs / bf16 peak)."""
+    flush = torch.zeros(2 * 129 * 2**20 // 4, dtype=torch.float32, device=dev)
+    rows = []
+    plan = [("single256", None, False), ("vit_b16_mlp", None, False),
+            ("llama2_7b_decode", ("q", "gate", "down"), False),
+            ("llama2_7b_prefill", ("q", "gate", "down"), False),
+            ("llama2_70b", ("q", "gate", "down"), True)]
+    for key, names, random_codes in plan:
+        wk = wl.WORKLOADS[key]
+        layers = [l for l in wk.layers if names is None or l.name in names]
+        for layer in layers:
+            acts = {}
+            for r in wk.redundancy:
+                prep = prepare_layer_random_codes if random_codes else prepare_layer
+                L = prep(fq, wl, torch, wk, layer, r, dev)
+                for M in wk.tokens:
+                    if M not in acts:
+                        acts[M] = torch.from_numpy(wl.activations(wk, layer, M)).to(
+                            dev, torch.bfloat16)
+                    for use_gamma in wk.gamma:
+                        cold, warm = time_layer(fq, torch, L, acts[M], use_gamma, dev, stream,
+                                                flush)
+                        args_ = (L["d_in"], L["d_out"], L["n_in"], L["n_out"], M)
+                        by, fl = layer_bytes(*args_), layer_flops(*args_)
+                        t_hbm = by / (peaks["hbm_gbs"] * 1e9) * 1e6
+                        t_tc = fl / (peaks["bf16_tflops"] * 1e12) * 1e6
+                        bound = "hbm" if t_hbm >= t_tc else "tensor"
+                        rows.append({
+                            "workload": key, "layer": f"{layer.name} {layer.d_out}x{layer.d_in}",
+                            "r": str(r), "k_in": L["k_in"], "k_out": L["k_out"], "M": M,
+                            "gamma": use_gamma, "us_cold": round(cold, 2),
+                            "us_warm": round(warm, 2), "tokens_per_s": round(M / cold * 1e6),
+                            "bytes": by, "flops": fl, "bound": bound,
+                            "roof_us": round(max(t_hbm, t_tc), 2),
+                            "frac_cold": round(max(t_hbm, t_tc) / cold, 3),
+                            "frac_warm": round(max(t_hbm, t_tc) / warm, 3),
+                            "codes": "seeded uniform" if random_codes else "RTN of C",
+                        })
+                        print(json.dumps(rows[-1]), file=sys.stderr, flush=True)
+                del L
+                torch.cuda.empty_cache()
+            del acts
+    print(json.dumps({
+        "metric": METRIC, "unit": UNIT, "n_gpus": 1, "dtype": "bf16", "data": "synthetic",
+        "peaks": {"hbm_gbs": peaks["hbm_gbs"], "bf16_tflops": peaks["bf16_tflops"]},
+        "timing": ("cold: median of 30 calls, each after writing a 258 MB buffer (2 x L2), CUDA "
+                   "events around the call; warm: 20 calls back to back in a CUDA graph"),
+        "sweep": rows}), flush=True)
+
+
 # --------------------------------------------------------------------------- main
 def aggregate(elapsed_ms, steps, layers_per_step, world):
     """Whole-job microseconds per layer from the slowest rank's elapsed time: every rank
@@ -520,6 +703,8 @@ def main(argv=None):
     ap.add_argument("--regime", default="both", choices=["both", "decode", "prefill"],
                     help="decode (the headline), prefill, or both (default)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--sweep", action="store_true",
+                    help="time every configuration's layer shapes (one JSON line) and exit")
     args = ap.parse_args(argv)
     if args.warmup < 3:
         ap.error("--warmup must be at least 3")
@@ -554,6 +739,10 @@ def main(argv=None):
         if dist is not None:
             dist.barrier()
 
+    if args.sweep:
+        if rank == 0:
+            sweep(args, fq, wl, torch, dev, stream, peaks)
+        return
     if args.regime == "prefill":
         prefill_only(args, fq, wl, torch, dev, rank, world, dist, stream, peaks)
         return
@@ -606,6 +795,9 @@ def main(argv=None):
                 "per step"),
     }
     del grouped_graph
+
+    # the same block with the frames in structured form (fq_linear_forward_implicit)
+    implicit = measure_implicit(args, fq, wl, torch, dec, stream, peaks)
 
     # end to end through the C ABI with host buffers
     barrier()
@@ -668,6 +860,7 @@ def main(argv=None):
             "per_layer": per_layer,
         },
         "grouped": grouped,
+        "implicit": implicit,
         "e2e": {"value": round(e2e_us, 3), "unit": UNIT, "h2d_bytes_per_step": h2d,
                 "d2h_bytes_per_step": d2h,
                 "copies": ("per step: one host-to-device copy of the 7 layers' inputs from pinned "

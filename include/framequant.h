@@ -198,6 +198,72 @@ fq_status fq_quantize_rtn(const float* C, int n_out, int n_in, uint8_t* codes, u
                           uint16_t* zero, float* gamma, fq_stream_t stream);
 
 /* ------------------------------------------------------------------------------------------
+ * Frames in structured form (the paper's own deployment form: Sec. 2.2 and Appendix J build T
+ * from rho/2 disjoint runs of a spectral-tetris frame, each modulated by k roots of unity;
+ * Appendix K applies a random rotation).  With d a multiple of rho, run j of the un-rotated
+ * frame covers complex coordinates c = j w .. (j+1) w - 1, w = d / rho (real coordinates 2c and
+ * 2c + 1), and its k frame vectors are the realified rows of the k x w block
+ * exp(2 pi i k_i c / k) / sqrt(k).  So T = T_u R^T with T_u block-diagonal, and
+ *     z = T x = T_u (R^T x),        y = T^T u = R (T_u^T u),
+ * which needs the rotation factors and k roots of unity instead of the n x d operator: a few
+ * hundred KB per side instead of 2 n d bytes.
+ * ---------------------------------------------------------------------------------------- */
+
+/* A frame prepared by fq_frame_implicit: device arrays inside the caller's buffer. */
+typedef struct {
+  int32_t k, rho, d;       /* (k, rho, d): rho even, d a multiple of rho, k >= d / rho */
+  int32_t a, b;            /* rotation R = Pi (Q_a kron Q_b) D with a * b = d; 0, 0: R = I */
+  const float* Qa;         /* device a x a row-major, and its transpose QaT */
+  const float* QaT;
+  const float* Qb;         /* device b x b row-major, and its transpose QbT */
+  const float* QbT;
+  const int32_t* perm;     /* device d: (Pi v)[i] = v[perm[i]] */
+  const int32_t* iperm;    /* device d: the inverse permutation */
+  const float* signs;      /* device d, the diagonal of D */
+  const float* roots;      /* device 2 k: cos(2 pi m / k), sin(2 pi m / k), m = 0 .. k-1 */
+} fq_frame;
+
+/* Bytes of the device buffer fq_frame_implicit fills (a = b = 0 without rotation); 0 for an
+ * invalid triple. */
+size_t fq_frame_implicit_bytes(int k, int rho, int d, int a, int b);
+
+/* Prepare the structured form of the (k, rho, d) frame with rotation `rot` (NULL: none), the
+ * same frame fq_frame_build writes out densely.  Q_a and Q_b are computed on the host in double
+ * precision (Householder QR, columns signed as in fq_rotation) and stored as fp32; the roots of
+ * unity are computed on the host in double precision and stored as fp32.
+ *   buf    device buffer of fq_frame_implicit_bytes(k, rho, d, rot->a, rot->b) bytes, 256-byte
+ *          aligned; it must outlive every use of *out
+ *   out    host struct receiving the sizes and the device pointers into buf
+ * Synchronizes `stream` before returning.
+ * Errors: FQ_ERR_INVALID_ARG (rho odd, d not a multiple of rho, k < d / rho, a bad rotation),
+ *         FQ_ERR_WORKSPACE (buf NULL or too small), FQ_ERR_ALIGNMENT, FQ_ERR_CUDA. */
+fq_status fq_frame_implicit(int k, int rho, int d, const fq_rotation* rot, void* buf,
+                            size_t bytes, fq_frame* out, fq_stream_t stream);
+
+/* Bytes of workspace fq_linear_forward_implicit needs; 0 for invalid sizes. */
+size_t fq_implicit_workspace_bytes(int M, int d_in, int n_in, int n_out, int d_out);
+
+/* The layer forward of fq_linear_forward (Sec. 3.2) with T_in and T_out given in structured
+ * form: z = T_u,in (R_in^T x), the 2-bit code product of fq_linear_forward, then
+ * y = R_out (T_u,out^T u).  bf16 tokens in and out; the rotations and the run transforms are
+ * computed in fp32 on CUDA cores, z and u are rounded to bf16 as in FQ_BF16, and the code
+ * product runs on the tensor cores (the M <= 64 kernel of fq_linear_forward).
+ *   x      device bf16, M x F_in->d tokens;  y  device bf16, M x F_out->d
+ *   F_in, F_out  host pointers to prepared frames; C->n_in = F_in->k * F_in->rho and
+ *          C->n_out = F_out->k * F_out->rho
+ *   gamma  device fp32 [C->n_out] or NULL
+ *   ws     device workspace of fq_implicit_workspace_bytes(...) bytes, 256-byte aligned and
+ *          zero-filled before its first use (the header rules of fq_linear_forward)
+ *   max_sms  as in fq_linear_forward_sms (0: the whole device)
+ * Requirements: 1 <= M <= 64; the frames' d at most 40960; sizes as in fq_linear_forward.
+ * Errors: FQ_ERR_INVALID_ARG, FQ_ERR_ALIGNMENT, FQ_ERR_WORKSPACE, FQ_ERR_UNSUPPORTED (M > 64,
+ * d above the limit, device not compute capability 10.3), FQ_ERR_CUDA. */
+fq_status fq_linear_forward_implicit(const void* x, int M, const fq_frame* F_in,
+                                     const fq_packed* C, const fq_frame* F_out,
+                                     const float* gamma, void* y, void* ws, size_t ws_bytes,
+                                     int max_sms, fq_stream_t stream);
+
+/* ------------------------------------------------------------------------------------------
  * Forward pass without a caller-provided workspace.  The paper has no counterpart: this is a
  * convenience of the library for callers that cannot allocate device memory.
  * ---------------------------------------------------------------------------------------- */

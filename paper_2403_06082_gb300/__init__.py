@@ -19,7 +19,8 @@ __all__ = [
     "fq_linear_forward_sms", "fq_check",
     "fq_status_str", "EXPORTED", "fq_frame_workspace_bytes", "fq_frame_build",
     "fq_coefficients_workspace_bytes", "fq_coefficients", "fq_quantize_rtn",
-    "fq_linear_forward_static", "FQ_STATIC_SCRATCH_BYTES",
+    "fq_linear_forward_static", "FQ_STATIC_SCRATCH_BYTES", "Frame", "fq_frame_implicit_bytes",
+    "fq_frame_implicit", "fq_implicit_workspace_bytes", "fq_linear_forward_implicit",
 ]
 FQ_STATIC_SCRATCH_BYTES = 16 << 20
 
@@ -32,7 +33,8 @@ EXPORTED = ("fq_packed_words", "fq_pack", "fq_workspace_bytes", "fq_linear_forwa
             "fq_linear_forward_sms",
             "fq_check", "fq_status_str", "fq_frame_workspace_bytes", "fq_frame_build",
             "fq_coefficients_workspace_bytes", "fq_coefficients", "fq_quantize_rtn",
-            "fq_linear_forward_static")
+            "fq_linear_forward_static", "fq_frame_implicit_bytes", "fq_frame_implicit",
+            "fq_implicit_workspace_bytes", "fq_linear_forward_implicit")
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
 
@@ -56,6 +58,14 @@ class _Rotation(ctypes.Structure):
     _fields_ = [("a", ctypes.c_int32), ("b", ctypes.c_int32), ("gauss_a", ctypes.c_void_p),
                 ("gauss_b", ctypes.c_void_p), ("perm", ctypes.c_void_p),
                 ("signs", ctypes.c_void_p)]
+
+
+class _Frame(ctypes.Structure):
+    _fields_ = [("k", ctypes.c_int32), ("rho", ctypes.c_int32), ("d", ctypes.c_int32),
+                ("a", ctypes.c_int32), ("b", ctypes.c_int32), ("Qa", ctypes.c_void_p),
+                ("QaT", ctypes.c_void_p), ("Qb", ctypes.c_void_p), ("QbT", ctypes.c_void_p),
+                ("perm", ctypes.c_void_p), ("iperm", ctypes.c_void_p),
+                ("signs", ctypes.c_void_p), ("roots", ctypes.c_void_p)]
 
 
 _lib = None
@@ -110,6 +120,19 @@ def lib() -> ctypes.CDLL:
             ctypes.c_void_p, ctypes.c_int, ctypes.c_int, ctypes.c_void_p,
             ctypes.POINTER(_Packed), ctypes.c_void_p, ctypes.c_int, ctypes.c_void_p,
             ctypes.c_void_p, ctypes.c_int, ctypes.c_void_p]
+        L.fq_frame_implicit_bytes.restype = ctypes.c_size_t
+        L.fq_frame_implicit_bytes.argtypes = [ctypes.c_int] * 5
+        L.fq_frame_implicit.restype = ctypes.c_int
+        L.fq_frame_implicit.argtypes = [ctypes.c_int, ctypes.c_int, ctypes.c_int,
+                                        ctypes.POINTER(_Rotation), ctypes.c_void_p,
+                                        ctypes.c_size_t, ctypes.POINTER(_Frame), ctypes.c_void_p]
+        L.fq_implicit_workspace_bytes.restype = ctypes.c_size_t
+        L.fq_implicit_workspace_bytes.argtypes = [ctypes.c_int] * 5
+        L.fq_linear_forward_implicit.restype = ctypes.c_int
+        L.fq_linear_forward_implicit.argtypes = [
+            ctypes.c_void_p, ctypes.c_int, ctypes.POINTER(_Frame), ctypes.POINTER(_Packed),
+            ctypes.POINTER(_Frame), ctypes.c_void_p, ctypes.c_void_p, ctypes.c_void_p,
+            ctypes.c_size_t, ctypes.c_int, ctypes.c_void_p]
         L.fq_quantize_rtn.restype = ctypes.c_int
         L.fq_quantize_rtn.argtypes = [ctypes.c_void_p, ctypes.c_int, ctypes.c_int,
                                       ctypes.c_void_p, ctypes.c_void_p, ctypes.c_void_p,
@@ -227,6 +250,63 @@ def fq_frame_build(k: int, rho: int, d: int, rotation, T, ws, ws_bytes: int,
     _ok(lib().fq_frame_build(k, rho, d, ctypes.byref(rot) if rot is not None else None,
                              _ptr(T), _ptr(ws), ws_bytes, _stream(stream)), "fq_frame_build")
     del keep
+
+
+@dataclass
+class Frame:
+    """A frame in structured form: the device buffer filled by fq_frame_implicit and the C
+    descriptor pointing into it (the buffer must stay alive while the frame is used)."""
+    buf: object
+    c: _Frame
+
+    @property
+    def n(self) -> int:
+        return self.c.k * self.c.rho
+
+    @property
+    def d(self) -> int:
+        return self.c.d
+
+
+def fq_frame_implicit_bytes(k: int, rho: int, d: int, a: int = 0, b: int = 0) -> int:
+    return lib().fq_frame_implicit_bytes(k, rho, d, a, b)
+
+
+def fq_frame_implicit(k: int, rho: int, d: int, rotation, device=None, stream=None) -> Frame:
+    """Structured form of the (k, rho, d) frame; rotation as in fq_frame_build.  Allocates the
+    device buffer with torch."""
+    import numpy as np
+    import torch
+    a, b = (rotation[0], rotation[1]) if rotation is not None else (0, 0)
+    nb = fq_frame_implicit_bytes(k, rho, d, a, b)
+    if nb == 0:
+        raise FrameQuantError(1, "fq_frame_implicit_bytes")
+    buf = torch.empty(nb, dtype=torch.uint8, device=device or "cuda")
+    rot, keep = None, None
+    if rotation is not None:
+        _, _, ga, gb, perm, signs = rotation
+        keep = [np.ascontiguousarray(ga, np.float64), np.ascontiguousarray(gb, np.float64),
+                np.ascontiguousarray(perm, np.int64), np.ascontiguousarray(signs, np.float64)]
+        rot = _Rotation(a, b, *(k_.ctypes.data for k_ in keep))
+    c = _Frame()
+    _ok(lib().fq_frame_implicit(k, rho, d, ctypes.byref(rot) if rot is not None else None,
+                                _ptr(buf), nb, ctypes.byref(c), _stream(stream)),
+        "fq_frame_implicit")
+    del keep
+    return Frame(buf, c)
+
+
+def fq_implicit_workspace_bytes(M: int, d_in: int, n_in: int, n_out: int, d_out: int) -> int:
+    return lib().fq_implicit_workspace_bytes(M, d_in, n_in, n_out, d_out)
+
+
+def fq_linear_forward_implicit(x, M: int, F_in: Frame, C: Packed, F_out: Frame, gamma, y, ws,
+                               ws_bytes: int, max_sms: int = 0, stream=None) -> None:
+    pc = C._c()
+    _ok(lib().fq_linear_forward_implicit(_ptr(x), M, ctypes.byref(F_in.c), ctypes.byref(pc),
+                                         ctypes.byref(F_out.c), _ptr(gamma), _ptr(y), _ptr(ws),
+                                         ws_bytes, max_sms, _stream(stream)),
+        "fq_linear_forward_implicit")
 
 
 def fq_coefficients_workspace_bytes(d_out: int, n_in: int) -> int:

@@ -113,6 +113,7 @@ struct DecArgs {
   uint32_t* done;
   int pf_codes;           // prefetch this CTA's later code blocks into L2
   int pf_tout;            // prefetch the T_out^T tiles of its synthesis tasks into L2
+  int ext_in;             // bit p: phase p's input was written before the launch (no flags)
 };
 
 // Per-cluster task lists, a kernel parameter: cluster c runs task[off[c]] .. task[off[c+1]-1].
@@ -433,7 +434,7 @@ __global__ void __launch_bounds__(DecCfg<BN>::kThreads, 1)
       const CUtensorMap* tm = t.p == 0 ? &tmX : (t.p == 1 ? &tmZ : &tmU);
       while (kb < k1 && ok) {
         int kb_end = k1;
-        if (t.p > 0 && ready <= sl1) {
+        if (t.p > 0 && !((a.ext_in >> t.p) & 1) && ready <= sl1) {
           // first slice (from `ready`) that is not final yet, over the whole warp
           int first_missing = sl1 + 1;
           for (int gs = ready + lane; gs <= sl1; gs += 32)
@@ -624,7 +625,7 @@ __global__ void __launch_bounds__(DecCfg<BN>::kThreads, 1)
       bool fail = false;
       if (t.p == 1) {
         // sum of z over this CTA's K range: first the ready flags of the slices it reads
-        if (has_k) {
+        if (has_k && !(a.ext_in & 2)) {
           const int sl0 = (k0 * kBK) / rows_per, sl1 = (min(ph.K, k1 * kBK) - 1) / rows_per;
           for (int gs = sl0 + et; gs <= sl1 && !fail; gs += kEpi) {
             fail = !wait_flag(&a.ph[0].flags[(gs / S) * kWsSlices + gs % S], g, abort_flag);
@@ -911,7 +912,7 @@ void build_schedule(const int* R, const int* K, int S, int ncl, DecSched* out) {
   for (int p = 0; p < 3; ++p) {
     order.resize(RT[p]);
     for (int t = 0; t < RT[p]; ++t) order[t] = t;
-    if (p < 2) {
+    if (p < 2 && kbs[p + 1] > 0) {
       const int64_t split_rows = static_cast<int64_t>(kbs[p + 1]) * kBK;
       std::stable_sort(order.begin(), order.end(), [&](int x, int y) {
         return (static_cast<int64_t>(x) * kBM) % split_rows <
@@ -1033,10 +1034,13 @@ size_t decode_workspace_bytes(int M, int d_in, int n_in, int n_out, int d_out) {
   return dec_ws(M, n_in, n_out).total;
 }
 
-fq_status launch_decode_forward(const void* x, int M, int d_in, const void* T_in,
-                                const fq_packed& Cq, const void* T_out_t, int d_out,
-                                const float* gamma, void* y, char* ws, size_t ws_bytes,
-                                int max_sms, cudaStream_t s) {
+namespace {
+
+// The fused kernel over all three phases, or (core_only) over the code product alone with z
+// already in the workspace and u left there.
+fq_status launch_decode(const void* x, int M, int d_in, const void* T_in, const fq_packed& Cq,
+                        const void* T_out_t, int d_out, const float* gamma, void* y, char* ws,
+                        size_t ws_bytes, int max_sms, bool core_only, cudaStream_t s) {
   const int n_in = Cq.n_in, n_out = Cq.n_out;
   const DecWs L = dec_ws(M, n_in, n_out);
   if (ws_bytes < L.total) return FQ_ERR_WORKSPACE;
@@ -1049,9 +1053,9 @@ fq_status launch_decode_forward(const void* x, int M, int d_in, const void* T_in
 
   DecArgs a{};
   a.M = M;
-  const int R[3] = {n_in, n_out, d_out};
-  const int K[3] = {d_in, n_in, n_out};
-  void* outs[3] = {ws + L.z, ws + L.u, y};
+  const int R[3] = {core_only ? 0 : n_in, n_out, core_only ? 0 : d_out};
+  const int K[3] = {core_only ? 0 : d_in, n_in, core_only ? 0 : n_out};
+  void* outs[3] = {ws + L.z, ws + L.u, core_only ? static_cast<void*>(ws + L.u) : y};
   for (int p = 0; p < 3; ++p) {
     a.ph[p].R = R[p];
     a.ph[p].K = K[p];
@@ -1065,17 +1069,47 @@ fq_status launch_decode_forward(const void* x, int M, int d_in, const void* T_in
   a.status = reinterpret_cast<int32_t*>(ws);
   a.gen = reinterpret_cast<uint32_t*>(ws + kWsGen);
   a.done = reinterpret_cast<uint32_t*>(ws + kWsDone);
+  a.ext_in = core_only ? 2 : 0;
 
   CUtensorMap m[5];
-  if (!tmap_bf16(&m[0], T_in, n_in, d_in, kBM) || !tmap_bf16(&m[1], x, M, d_in, BN) ||
-      !tmap_bf16(&m[2], ws + L.z, M, n_in, BN) ||
-      !tmap_bf16(&m[3], T_out_t, d_out, n_out, kBM) || !tmap_bf16(&m[4], ws + L.u, M, n_out, BN))
+  if (!tmap_bf16(&m[2], ws + L.z, M, n_in, BN) || !tmap_bf16(&m[4], ws + L.u, M, n_out, BN))
     return FQ_ERR_CUDA;
+  if (core_only) {
+    // no analysis or synthesis tasks: their maps are never used for a copy
+    m[0] = m[2];
+    m[1] = m[2];
+    m[3] = m[4];
+  } else if (!tmap_bf16(&m[0], T_in, n_in, d_in, kBM) || !tmap_bf16(&m[1], x, M, d_in, BN) ||
+             !tmap_bf16(&m[3], T_out_t, d_out, n_out, kBM)) {
+    return FQ_ERR_CUDA;
+  }
   switch (BN) {
     case 16: return run<16>(m, a, R, K, sms, budget, s);
     case 32: return run<32>(m, a, R, K, sms, budget, s);
     default: return run<64>(m, a, R, K, sms, budget, s);
   }
+}
+
+}  // namespace
+
+fq_status launch_decode_forward(const void* x, int M, int d_in, const void* T_in,
+                                const fq_packed& Cq, const void* T_out_t, int d_out,
+                                const float* gamma, void* y, char* ws, size_t ws_bytes,
+                                int max_sms, cudaStream_t s) {
+  return launch_decode(x, M, d_in, T_in, Cq, T_out_t, d_out, gamma, y, ws, ws_bytes, max_sms,
+                       false, s);
+}
+
+fq_status launch_decode_core(int M, const fq_packed& Cq, const float* gamma, char* ws,
+                             size_t ws_bytes, int max_sms, cudaStream_t s) {
+  return launch_decode(nullptr, M, 0, nullptr, Cq, nullptr, 0, gamma, nullptr, ws, ws_bytes,
+                       max_sms, true, s);
+}
+
+size_t decode_core_z_offset() { return kWsHeader; }
+
+size_t decode_core_u_offset(int M, int n_in) {
+  return kWsHeader + round_up(static_cast<int64_t>(M) * n_in * 2, 256);
 }
 
 }  // namespace fq

@@ -5,6 +5,8 @@
 #include <cstdint>
 #include <cuda_runtime.h>
 
+#include <vector>
+
 #include "framequant.h"
 
 namespace fq {
@@ -51,6 +53,17 @@ fq_status launch_decode_forward(const void* x, int M, int d_in, const void* T_in
                                 const fq_packed& C, const void* T_out_t, int d_out,
                                 const float* gamma, void* y, char* ws, size_t ws_bytes,
                                 int max_sms, cudaStream_t s);
+
+// The code product alone (z already in the workspace at decode_core_z_offset(), u left at
+// decode_core_u_offset()), for the structured-frame forward.
+fq_status launch_decode_core(int M, const fq_packed& C, const float* gamma, char* ws,
+                             size_t ws_bytes, int max_sms, cudaStream_t s);
+size_t decode_core_z_offset();
+size_t decode_core_u_offset(int M, int n_in);
+
+// ---- fq_prep.cu: Q of the Householder QR of the a x a row-major G, columns signed so that R
+// has a positive diagonal (row-major output)
+void haar_q(const double* G, int a, std::vector<double>& Q);
 
 // ---- fq_tc.cu: bf16 tensor-core path
 size_t tc_workspace_bytes(int M, int d_in, int n_in, int n_out, int d_out);

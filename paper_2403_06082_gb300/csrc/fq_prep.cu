@@ -67,6 +67,8 @@ bool modulation_tight(const std::vector<double>& F, int rho_c, int d_c, int k) {
   return true;
 }
 
+}  // namespace
+
 // ------------------------------------------------------------------ host: Haar factor
 // Q of the Householder QR of a square matrix G (row-major, a x a), with the columns signed so
 // that R has a positive diagonal; Q is written row-major.
@@ -108,6 +110,8 @@ void haar_q(const double* G, int a, std::vector<double>& Q) {
     if (A[c * a + c] < 0)
       for (int i = 0; i < a; ++i) Q[i * a + c] = -Q[i * a + c];
 }
+
+namespace {
 
 // ------------------------------------------------------------------ device kernels
 // Real analysis operator of the modulated, Parseval-normalised, realified frame.  Row

@@ -94,3 +94,47 @@ def test_valid_bf16_request_needs_sm103(L):
         pass
     # no CUDA device: the bf16 path refuses instead of falling back to anything
     assert _call(L) == 3
+
+
+def _frame(k=18, rho=16, d=256, roots=0x8000):
+    return fq._Frame(k, rho, d, 0, 0, None, None, None, None, None, None, None, roots)
+
+
+def _call_implicit(L, x=0x1000, M=8, Fi=None, C=None, Fo=None, gamma=None, y=0x4000,
+                   ws=0x10000, ws_bytes=1 << 30, max_sms=0):
+    C = C or _P(0x5000, 0x6000, 0x7000, 288, 288)
+    Fi, Fo = Fi or _frame(), Fo or _frame()
+    return L.fq_linear_forward_implicit(x, M, ctypes.byref(Fi), ctypes.byref(C), ctypes.byref(Fo),
+                                        gamma, y, ws, ws_bytes, max_sms, None)
+
+
+def test_implicit_frame_sizes_and_validation(L):
+    # (k, rho, d) needs rho even, d a multiple of rho and k >= d / rho (tight modulation)
+    assert fq.fq_frame_implicit_bytes(18, 16, 256, 16, 16) > 0
+    assert fq.fq_frame_implicit_bytes(282, 16, 4096, 64, 64) > 0
+    assert fq.fq_frame_implicit_bytes(18, 16, 256, 0, 0) < fq.fq_frame_implicit_bytes(18, 16, 256, 16, 16)
+    assert fq.fq_frame_implicit_bytes(15, 16, 256, 16, 16) == 0     # k < w = 16
+    assert fq.fq_frame_implicit_bytes(18, 15, 255, 15, 17) == 0     # rho odd
+    assert fq.fq_frame_implicit_bytes(18, 16, 264, 8, 33) == 0      # d not a multiple of rho
+    assert fq.fq_frame_implicit_bytes(18, 16, 256, 16, 8) == 0      # a * b != d
+    assert fq.fq_implicit_workspace_bytes(16, 4096, 4512, 4512, 4096) > \
+        fq.fq_workspace_bytes(16, 4096, 4512, 4512, 4096, fq.FQ_BF16)
+    assert fq.fq_implicit_workspace_bytes(65, 4096, 4512, 4512, 4096) == 0
+    out = fq._Frame()
+    assert L.fq_frame_implicit(15, 16, 256, None, 0x1000, 1 << 20, ctypes.byref(out), None) == 1
+    assert L.fq_frame_implicit(18, 16, 256, None, None, 1 << 20, ctypes.byref(out), None) == 4
+    assert L.fq_frame_implicit(18, 16, 256, None, 0x1010, 1 << 20, ctypes.byref(out), None) == 2
+
+
+def test_implicit_host_validation_without_gpu(L):
+    assert _call_implicit(L, x=None) == 1
+    assert _call_implicit(L, M=0) == 1
+    assert _call_implicit(L, max_sms=-1) == 1
+    assert _call_implicit(L, Fi=_frame(k=15)) == 1                  # not a tight frame
+    assert _call_implicit(L, Fi=_frame(roots=None)) == 1
+    assert _call_implicit(L, C=_P(0x5000, 0x6000, 0x7000, 288, 304)) == 1   # n_in != k rho
+    assert _call_implicit(L, x=0x1002) == 2
+    assert _call_implicit(L, ws=None) == 4
+    assert _call_implicit(L, ws=0x10010) == 2
+    assert _call_implicit(L, M=65) == 3                             # decode batches only
+    assert _call_implicit(L, ws_bytes=1024) == 4
