@@ -56,6 +56,9 @@ constexpr int kChunk = 16;                  // accumulator columns per TMEM load
 struct PhaseArgs {
   int R, K, M;
   int RT, TT, KB, tiles;
+  int KS, kbs, units;        // K splits per tile, K blocks per split, tiles * KS work units
+  float* part;               // KS > 1: fp32 partial tiles [tile][split][BN][128]
+  uint32_t* cnt;             // KS > 1: arrivals per tile (the last resets it to 0)
   const uint32_t* words;     // core: packed codes
   __nv_bfloat16* out;        // [M][R]
   float* zsum_part;          // analysis writes [RT][M] sums of z; the core reads them
@@ -87,8 +90,8 @@ struct Layout {
   static constexpr int oBar = oCodes + kStages * kCodesStage;
   static constexpr int kNumBars = 4 * kStages + 2 + 2 + 1;
   static constexpr int oMisc = oBar + kNumBars * 8;
-  static constexpr int oRedSmall = oMisc + 16;                      // [4][kChunk] floats
-  static constexpr int oZsum = oRedSmall + 4 * kChunk * 4;          // [2][BN] floats
+  static constexpr int oRedSmall = oMisc + 16;                      // [4][kChunk] + 4 floats
+  static constexpr int oZsum = oRedSmall + (4 * kChunk + 4) * 4;    // [2][BN] floats
   static constexpr int kBytes = oZsum + 2 * BN * 4 + 1024;          // + alignment slack
   static_assert(BN == 128 || BN == 256, "prefill tile widths");
   static_assert(kBTileBytes % 1024 == 0, "B tiles must keep 1024-byte alignment");
@@ -164,12 +167,15 @@ __global__ void __launch_bounds__(threads_for<PHASE>(), 1)
   uint64_t* mma_done = tempty + 2;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + Lo::oMisc);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
-  float* red = reinterpret_cast<float*>(smem + Lo::oRedSmall);     // [4][kChunk]
+  float* red = reinterpret_cast<float*>(smem + Lo::oRedSmall);     // [4][kChunk], flag
   float* zsum_s = reinterpret_cast<float*>(smem + Lo::oZsum);      // [2][BN]
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const uint32_t cid = blockIdx.x, ncl = gridDim.x;
-  const int k0 = 0, k1 = p.KB;
+  // work unit u = split * tiles + tile: K blocks [split * kbs, min(KB, (split + 1) * kbs))
+  auto unit_tile = [&](int u) { return u % p.tiles; };
+  auto unit_k0 = [&](int u) { return (u / p.tiles) * p.kbs; };
+  auto unit_k1 = [&](int u) { return min(p.KB, (u / p.tiles + 1) * p.kbs); };
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < S_; ++s) {
@@ -206,8 +212,9 @@ __global__ void __launch_bounds__(threads_for<PHASE>(), 1)
       // Weight tiles of the first tile do not depend on the previous kernel: issue up to a
       // full ring of them before waiting for it, and warm L2 with the rest.
       int pre = 0;
-      if (static_cast<int>(cid) < p.tiles) {
-        const int rt = static_cast<int>(cid) / p.TT;
+      if (static_cast<int>(cid) < p.units) {
+        const int rt = unit_tile(static_cast<int>(cid)) / p.TT;
+        const int k0 = unit_k0(static_cast<int>(cid)), k1 = unit_k1(static_cast<int>(cid));
         pre = min(S_, k1 - k0);
         for (int i = 0; i < pre; ++i) {
           const int kb = k0 + i;
@@ -245,8 +252,9 @@ __global__ void __launch_bounds__(threads_for<PHASE>(), 1)
       bool issued[S_];
 #pragma unroll
       for (int s = 0; s < S_; ++s) issued[s] = false, issued_parity[s] = 0;
-      for (int tile = static_cast<int>(cid); tile < p.tiles && !*abort_flag;
-           tile += static_cast<int>(ncl)) {
+      for (int unit = static_cast<int>(cid); unit < p.units && !*abort_flag;
+           unit += static_cast<int>(ncl)) {
+        const int tile = unit_tile(unit), k0 = unit_k0(unit), k1 = unit_k1(unit);
         const int rt = tile / p.TT, tt = tile % p.TT;
         for (int kb = k0; kb < k1; ++kb, ++it) {
           if (it >= pre) {
@@ -290,8 +298,9 @@ __global__ void __launch_bounds__(threads_for<PHASE>(), 1)
       int buf = 0;
       uint32_t acc_phase = 0;
       bool issued_any = false;
-      for (int tile = static_cast<int>(cid); tile < p.tiles && !*abort_flag;
-           tile += static_cast<int>(ncl)) {
+      for (int unit = static_cast<int>(cid); unit < p.units && !*abort_flag;
+           unit += static_cast<int>(ncl)) {
+        const int k0 = unit_k0(unit), k1 = unit_k1(unit);
         if (!mbar_wait(&tempty[buf], acc_phase ^ 1, abort_flag)) {
           report(p.status, FQ_ERR_TIMEOUT);
           *abort_flag = 1;
@@ -337,7 +346,8 @@ __global__ void __launch_bounds__(threads_for<PHASE>(), 1)
     pdl_wait();
     int buf = 0;
     uint32_t acc_phase = 0;
-    for (int tile = static_cast<int>(cid); tile < p.tiles; tile += static_cast<int>(ncl)) {
+    for (int unit = static_cast<int>(cid); unit < p.units; unit += static_cast<int>(ncl)) {
+      const int tile = unit_tile(unit), split = unit / p.tiles;
       const int rt = tile / p.TT, tt = tile % p.TT;
       const int row = rt * kBM + r_in_tile;
       const int t0 = tt * BN;
@@ -370,47 +380,92 @@ __global__ void __launch_bounds__(threads_for<PHASE>(), 1)
       const uint32_t t_row = tmem_base + (static_cast<uint32_t>(quarter * 32) << 16) +
                              static_cast<uint32_t>(buf * BN);
       const float* zs = zsum_s + buf * BN;
-      {
-        const float g_i = (PHASE == kCore && row_ok && p.gamma) ? p.gamma[row] : 1.f;
+      const float g_i = (PHASE == kCore && row_ok && p.gamma) ? p.gamma[row] : 1.f;
+      // the finished values of columns c .. c + 15 of this thread's row
+      auto emit = [&](int c, float* v) {
+#pragma unroll
+        for (int q = 0; q < kChunk; ++q) {
+          if (PHASE == kCore) v[q] = g_i * fmaf(s_i, v[q], z_i * zs[c + q]);
+          const __nv_bfloat16 b = __float2bfloat16_rn(v[q]);
+          v[q] = __bfloat162float(b);
+          const int t = t0 + c + q;
+          if (row_ok && t < p.M) p.out[static_cast<int64_t>(t) * p.R + row] = b;
+        }
+        if (PHASE == kAnalysis) {
+          // per-token sum over the tile's 128 rows of the bf16 z actually stored
+#pragma unroll
+          for (int q = 0; q < kChunk; ++q) {
+            float s = row_ok ? v[q] : 0.f;
+#pragma unroll
+            for (int off = 16; off > 0; off >>= 1) s += __shfl_xor_sync(0xffffffffu, s, off);
+            v[q] = s;
+          }
+          if (lane == 0) {
+#pragma unroll
+            for (int q = 0; q < kChunk; ++q) red[ew * kChunk + q] = v[q];
+          }
+          named_barrier_sync(1, kEpi);
+          if (et < kChunk) {
+            const int t = t0 + c + et;
+            // fixed order over the TMEM quarters (rows 0.., 32.., 64.., 96..)
+            const float s = (red[2 * kChunk + et] + red[3 * kChunk + et]) +
+                            (red[0 * kChunk + et] + red[1 * kChunk + et]);
+            if (t < p.M) p.zsum_part[static_cast<int64_t>(rt) * p.M + t] = s;
+          }
+          named_barrier_sync(1, kEpi);
+        }
+      };
+      if (p.KS == 1) {
+#pragma unroll 1
+        for (int c = 0; c < BN; c += kChunk) {
+          float v[kChunk];
+          tmem_ld16(t_row + c, v);
+          tmem_wait_ld();
+          emit(c, v);
+        }
+        tc_fence_before_sync();
+        mbar_arrive(&tempty[buf]);
+      } else {
+        // Split K: store this split's partial tile (column-major, so a warp's 32 rows are one
+        // 128-byte line), release the accumulator, and count the split in.  The tile's last
+        // split to arrive adds the partials in split order and finishes the tile.
+        float* mine = p.part + (static_cast<int64_t>(tile) * p.KS + split) * BN * kBM;
 #pragma unroll 1
         for (int c = 0; c < BN; c += kChunk) {
           float v[kChunk];
           tmem_ld16(t_row + c, v);
           tmem_wait_ld();
 #pragma unroll
-          for (int q = 0; q < kChunk; ++q) {
-            if (PHASE == kCore) v[q] = g_i * fmaf(s_i, v[q], z_i * zs[c + q]);
-            const __nv_bfloat16 b = __float2bfloat16_rn(v[q]);
-            v[q] = __bfloat162float(b);
-            const int t = t0 + c + q;
-            if (row_ok && t < p.M) p.out[static_cast<int64_t>(t) * p.R + row] = b;
-          }
-          if (PHASE == kAnalysis) {
-            // per-token sum over the tile's 128 rows of the bf16 z actually stored
-#pragma unroll
-            for (int q = 0; q < kChunk; ++q) {
-              float s = row_ok ? v[q] : 0.f;
-#pragma unroll
-              for (int off = 16; off > 0; off >>= 1) s += __shfl_xor_sync(0xffffffffu, s, off);
-              v[q] = s;
-            }
-            if (lane == 0) {
-#pragma unroll
-              for (int q = 0; q < kChunk; ++q) red[ew * kChunk + q] = v[q];
-            }
-            named_barrier_sync(1, kEpi);
-            if (et < kChunk) {
-              const int t = t0 + c + et;
-              // fixed order over the TMEM quarters (rows 0.., 32.., 64.., 96..)
-              const float s = (red[2 * kChunk + et] + red[3 * kChunk + et]) +
-                              (red[0 * kChunk + et] + red[1 * kChunk + et]);
-              if (t < p.M) p.zsum_part[static_cast<int64_t>(rt) * p.M + t] = s;
-            }
-            named_barrier_sync(1, kEpi);
-          }
+          for (int q = 0; q < kChunk; ++q) mine[(c + q) * kBM + r_in_tile] = v[q];
         }
         tc_fence_before_sync();
         mbar_arrive(&tempty[buf]);
+        __threadfence();
+        named_barrier_sync(1, kEpi);
+        if (et == 0) {
+          const uint32_t old = atomicAdd(&p.cnt[tile], 1u);
+          const bool last = old == static_cast<uint32_t>(p.KS - 1);
+          if (last) p.cnt[tile] = 0;                 // ready for the next call
+          __threadfence();
+          red[4 * kChunk] = last ? 1.f : 0.f;
+        }
+        named_barrier_sync(1, kEpi);
+        if (red[4 * kChunk] != 0.f) {
+          const float* all = p.part + static_cast<int64_t>(tile) * p.KS * BN * kBM;
+#pragma unroll 1
+          for (int c = 0; c < BN; c += kChunk) {
+            float v[kChunk];
+#pragma unroll
+            for (int q = 0; q < kChunk; ++q) v[q] = 0.f;
+            for (int sp = 0; sp < p.KS; ++sp) {
+#pragma unroll
+              for (int q = 0; q < kChunk; ++q)
+                v[q] += ldcg_f32(all + (static_cast<int64_t>(sp) * BN + c + q) * kBM + r_in_tile);
+            }
+            emit(c, v);
+          }
+        }
+        named_barrier_sync(1, kEpi);                 // the flag is read before it is reused
       }
       if (++buf == 2) buf = 0, acc_phase ^= 1;
     }
@@ -423,9 +478,9 @@ __global__ void __launch_bounds__(threads_for<PHASE>(), 1)
       uint32_t phase = 0;
       int it = 0;
       bool ok = true;
-      for (int tile = static_cast<int>(cid); tile < p.tiles && ok && !*abort_flag;
-           tile += static_cast<int>(ncl)) {
-        for (int kb = k0; kb < k1; ++kb, ++it) {
+      for (int unit = static_cast<int>(cid); unit < p.units && ok && !*abort_flag;
+           unit += static_cast<int>(ncl)) {
+        for (int kb = unit_k0(unit); kb < unit_k1(unit); ++kb, ++it) {
           if ((it & 3) == dw) {
             if (!mbar_wait(&cfull[stage], phase, abort_flag)) {
               ok = false;
@@ -515,21 +570,40 @@ cudaError_t prepare_kernel(int dev) {
   return e;
 }
 
-// One tile per CTA and round: as many CTAs as tiles, at most one per SM.
+// One work unit per CTA and round, at most one CTA per SM.  A phase with fewer tiles than SMs
+// splits each tile's K range (up to kMaxSplits ways, at least kMinSplitBlocks K blocks each)
+// so that it fills the GPU: at 128 tokens a 8192-row phase has only 64 tiles.
+constexpr int kMaxSplits = 4;
+constexpr int kMinSplitBlocks = 4;
+constexpr int kMaxSplitSms = 256;      // bound on the SM count used for split-K planning
+
+int split_for(int tiles, int KB, int sms) {
+  sms = std::min(sms, kMaxSplitSms);
+  if (tiles >= sms) return 1;
+  int ks = std::min({kMaxSplits, sms / tiles, KB / kMinSplitBlocks});
+  return std::max(ks, 1);
+}
+
 template <int PHASE, int BN>
 void plan_phase(PhaseArgs& a, const DeviceInfo& d, int& grid) {
   a.RT = static_cast<int>(ceil_div(a.R, kBM));
   a.TT = static_cast<int>(ceil_div(a.M, BN));
   a.KB = static_cast<int>(ceil_div(a.K, kBK));
   a.tiles = a.RT * a.TT;
-  grid = std::min(a.tiles, d.sms);
+  a.KS = split_for(a.tiles, a.KB, d.sms);
+  a.kbs = static_cast<int>(ceil_div(a.KB, a.KS));
+  a.KS = static_cast<int>(ceil_div(a.KB, a.kbs));     // every split non-empty
+  a.units = a.tiles * a.KS;
+  grid = std::min(a.units, d.sms);
 }
 
 struct WsLayout {
-  size_t z, u, zsum, total;
+  size_t z, u, zsum, cnt, part, total;
 };
 
-WsLayout ws_layout(int M, int n_in, int n_out) {
+// Partial tiles for split K, sized for any device with at most kMaxSplitSms SMs: a phase with
+// t < kMaxSplitSms tiles keeps at most min(kMaxSplitSms, t * kMaxSplits) partial tiles.
+WsLayout ws_layout(int M, int d_in, int n_in, int n_out, int d_out) {
   WsLayout L{};
   size_t off = kWsHeader;
   L.z = off;
@@ -538,6 +612,22 @@ WsLayout ws_layout(int M, int n_in, int n_out) {
   off += round_up(static_cast<int64_t>(M) * n_out * 2, 256);
   L.zsum = off;
   off += round_up(ceil_div(n_in, kBM) * M * 4, 256);
+  const int BN = pick_bn(M);
+  const int64_t TT = ceil_div(M, BN);
+  const int64_t rows[3] = {n_in, n_out, d_out};
+  int64_t slots = 0, max_tiles = 0;
+  for (int64_t r : rows) {
+    const int64_t tiles = ceil_div(r, kBM) * TT;
+    if (tiles < kMaxSplitSms) {
+      slots = std::max(slots, std::min<int64_t>(kMaxSplitSms, tiles * kMaxSplits));
+      max_tiles = std::max(max_tiles, tiles);
+    }
+  }
+  (void)d_in;
+  L.cnt = off;
+  off += round_up(max_tiles * 4, 256);
+  L.part = off;
+  off += static_cast<size_t>(slots) * BN * kBM * 4;
   L.total = off;
   return L;
 }
@@ -583,9 +673,7 @@ fq_status run_forward(const CUtensorMap* maps, PhaseArgs* a, int max_sms, cudaSt
 }  // namespace
 
 size_t tc_workspace_bytes(int M, int d_in, int n_in, int n_out, int d_out) {
-  (void)d_in;
-  (void)d_out;
-  return ws_layout(M, n_in, n_out).total;
+  return ws_layout(M, d_in, n_in, n_out, d_out).total;
 }
 
 fq_status launch_tc_forward(const void* x, int M, int d_in, const void* T_in,
@@ -593,7 +681,7 @@ fq_status launch_tc_forward(const void* x, int M, int d_in, const void* T_in,
                             const float* gamma, void* y, char* ws, size_t ws_bytes,
                             int max_sms, cudaStream_t s) {
   const int n_in = Cq.n_in, n_out = Cq.n_out;
-  const WsLayout L = ws_layout(M, n_in, n_out);
+  const WsLayout L = ws_layout(M, d_in, n_in, n_out, d_out);
   if (ws_bytes < L.total) return FQ_ERR_WORKSPACE;
   const int BN = pick_bn(M);
   auto* status = reinterpret_cast<int32_t*>(ws);
@@ -613,6 +701,8 @@ fq_status launch_tc_forward(const void* x, int M, int d_in, const void* T_in,
     a[ph].out = outs[ph];
     a[ph].zsum_part = zsum;
     a[ph].status = status;
+    a[ph].cnt = reinterpret_cast<uint32_t*>(ws + L.cnt);
+    a[ph].part = reinterpret_cast<float*>(ws + L.part);
   }
   a[1].words = Cq.words;
   a[1].scale = reinterpret_cast<const __half*>(Cq.scale);

@@ -166,3 +166,36 @@ def test_stream_argument():
                              0, stream=s)
     assert fq.fq_check(ws, stream=s) == 0
     assert rel_frobenius(y.double().cpu().numpy(), reference(L, X, True)) <= 1e-2
+
+
+@pytest.mark.parametrize("name,M,use_gamma", [
+    ("q", 65, False), ("q", 128, True), ("gate", 100, False), ("down", 128, False),
+    ("q", 200, False), ("down", 256, True),
+])
+def test_split_k_tensor_core_path(name, M, use_gamma):
+    """Batches just above the decode kernel's range on the 7B shapes: phases with fewer tiles
+    than SMs split each tile's K range and the last split to arrive adds the partials in
+    split order, so the result is also bitwise repeatable and independent of arrival order."""
+    L = oracle_layer("llama2_7b_decode", name)
+    X = activations("llama2_7b_decode", name, M)
+    D = DeviceLayer(L, BF16)
+    got = D.forward(X, use_gamma)
+    assert rel_frobenius(got, reference(L, X, use_gamma)) <= TOL[BF16]
+    np.testing.assert_array_equal(got, D.forward(X, use_gamma))
+
+
+def test_split_k_under_sm_budget():
+    """A smaller SM budget changes the split count; the result stays within tolerance."""
+    L = oracle_layer("llama2_7b_decode", "gate")
+    X = activations("llama2_7b_decode", "gate", 128)
+    D = DeviceLayer(L, BF16)
+    x = torch.from_numpy(X).to(DEV, BF16)
+    ref = reference(L, X, False)
+    for budget in (40, 100, 0):
+        y = torch.full((128, L.d_out), float("nan"), dtype=BF16, device=DEV)
+        nb = fq.fq_workspace_bytes(128, L.d_in, L.n_in, L.n_out, L.d_out, 0)
+        ws = torch.zeros(nb, dtype=torch.uint8, device=DEV)
+        fq.fq_linear_forward_sms(x, 128, L.d_in, D.T_in, D.C, D.T_out_t, L.d_out, None, y, ws,
+                                 nb, budget)
+        assert fq.fq_check(ws) == 0
+        assert rel_frobenius(y.double().cpu().numpy(), ref) <= TOL[BF16]
