@@ -255,9 +255,10 @@ size_t fq_implicit_workspace_bytes(int M, int d_in, int n_in, int n_out, int d_o
  *   ws     device workspace of fq_implicit_workspace_bytes(...) bytes, 256-byte aligned and
  *          zero-filled before its first use (the header rules of fq_linear_forward)
  *   max_sms  as in fq_linear_forward_sms (0: the whole device)
- * Requirements: 1 <= M <= 64; the frames' d at most 40960; sizes as in fq_linear_forward.
- * Errors: FQ_ERR_INVALID_ARG, FQ_ERR_ALIGNMENT, FQ_ERR_WORKSPACE, FQ_ERR_UNSUPPORTED (M > 64,
- * d above the limit, device not compute capability 10.3), FQ_ERR_CUDA. */
+ * Requirements: 1 <= M <= 64; for each frame d / rho <= 2560, k <= 4096 and b <= 1024 (the
+ * shared-memory footprint of its kernels); sizes and alignment as in fq_linear_forward.
+ * Errors: FQ_ERR_INVALID_ARG, FQ_ERR_ALIGNMENT, FQ_ERR_WORKSPACE, FQ_ERR_UNSUPPORTED (M > 64, a
+ * frame above those limits, device not compute capability 10.3), FQ_ERR_CUDA. */
 fq_status fq_linear_forward_implicit(const void* x, int M, const fq_frame* F_in,
                                      const fq_packed* C, const fq_frame* F_out,
                                      const float* gamma, void* y, void* ws, size_t ws_bytes,
