@@ -231,23 +231,31 @@ class Regime:
                 raise RuntimeError(f"{L['name']}: {fq.fq_status_str(st)}")
         torch.cuda.synchronize()
 
-    def forward(self, L, stream):
+    def forward(self, L, stream, prefetch=None):
         fq = self.fq
-        fq.fq_linear_forward(L["x"], self.M, L["d_in"], L["T_in"], L["C"], L["T_out_t"],
-                             L["d_out"], L["gamma"] if self.use_gamma else None, L["y"],
-                             self.ws, self.ws_bytes, fq.FQ_BF16, stream)
+        if prefetch is None:
+            fq.fq_linear_forward(L["x"], self.M, L["d_in"], L["T_in"], L["C"], L["T_out_t"],
+                                 L["d_out"], L["gamma"] if self.use_gamma else None, L["y"],
+                                 self.ws, self.ws_bytes, fq.FQ_BF16, stream)
+        else:
+            fq.fq_linear_forward_ex(L["x"], self.M, L["d_in"], L["T_in"], L["C"], L["T_out_t"],
+                                    L["d_out"], L["gamma"] if self.use_gamma else None, L["y"],
+                                    self.ws, self.ws_bytes, fq.FQ_BF16, 0, prefetch, stream)
 
-    def capture(self, layers, stream, host=False):
+    def capture(self, layers, stream, host=False, chain=False):
         """One graph: the layers' forwards in order; with host=True (all layers) the step's
-        inputs come from pinned host memory first and its results go back at the end."""
+        inputs come from pinned host memory first and its results go back at the end.  With
+        chain=True each forward names the next layer's T_in (the first layer's after the last)
+        as its L2 prefetch hint."""
         torch = self.torch
         assert not host or layers is self.layers
         g = torch.cuda.CUDAGraph()
         with torch.cuda.graph(g, stream=stream):
             if host:
                 self.x_all.copy_(self.x_host_all, non_blocking=True)
-            for L in layers:
-                self.forward(L, stream.cuda_stream)
+            for i, L in enumerate(layers):
+                nxt = layers[(i + 1) % len(layers)]["T_in"] if chain else None
+                self.forward(L, stream.cuda_stream, nxt)
             if host:
                 self.y_host_all.copy_(self.y_all, non_blocking=True)
         return g
@@ -751,9 +759,9 @@ def main(argv=None):
 
     # ---------------- decode: Llama-2-7B block, M = 16
     dec = Regime(fq, wl, torch, "llama2_7b_decode", 16, dev, rank)
-    step_graph = dec.capture(dec.layers, stream)
+    step_graph = dec.capture(dec.layers, stream, chain=True)
     layer_graphs = [dec.capture([L], stream) for L in dec.layers]
-    e2e_graph = dec.capture(dec.layers, stream, host=True)
+    e2e_graph = dec.capture(dec.layers, stream, host=True, chain=True)
     nL = len(dec.layers)
 
     uuid = None
@@ -846,7 +854,8 @@ def main(argv=None):
             "layers": {n: f"{o}x{i} k_in={ki} k_out={ko}" for n, o, i, ki, ko in dec_layers},
             "l2": ("no flush: each step streams 1.2 GB of distinct layer operands (> 126 MB "
                    "L2), so every layer's operands were last touched one step earlier"),
-            "timing": "one CUDA graph per step (7 layer forwards), CUDA events around K replays",
+            "timing": ("one CUDA graph per step (7 layer forwards, each naming the next layer's "
+                       "T_in as its L2 prefetch hint), CUDA events around K replays"),
             "parallelism": f"replicas x{world}, no data-path collective",
         },
         "roofline": {

@@ -141,6 +141,27 @@ fq_status fq_linear_forward_sms(const void* x, int M, int d_in, const void* T_in
                                 const float* gamma, void* y, void* ws, size_t ws_bytes, int mode,
                                 int max_sms, fq_stream_t stream);
 
+/* Options of fq_linear_forward_ex. */
+typedef struct {
+  int32_t max_sms;             /* 0: the whole device; otherwise the SM budget of
+                                  fq_linear_forward_sms */
+  const void* l2_prefetch;     /* device range to bring into L2 while this call runs, or NULL */
+  size_t l2_prefetch_bytes;    /* its length; rounded down to a multiple of 16 */
+} fq_forward_opts;
+
+/* fq_linear_forward with options (opts NULL: none).  The L2 prefetch is a hint for chaining
+ * layers, typically the next layer's T_in: the M <= 64 kernel issues it when this layer's own
+ * T_out^T is small enough to be warmed in L2 during the code product, so that its synthesis
+ * leaves HBM idle; each CTA then prefetches its share of the range when it reaches its first
+ * synthesis task.  Other calls ignore it.  Results never depend on it.  This entry point has
+ * no counterpart in the paper.
+ * Errors: those of fq_linear_forward; FQ_ERR_INVALID_ARG for max_sms < 0 or a NULL range of
+ * nonzero length; FQ_ERR_ALIGNMENT for a range start that is not 16-byte aligned. */
+fq_status fq_linear_forward_ex(const void* x, int M, int d_in, const void* T_in,
+                               const fq_packed* C, const void* T_out_t, int d_out,
+                               const float* gamma, void* y, void* ws, size_t ws_bytes, int mode,
+                               const fq_forward_opts* opts, fq_stream_t stream);
+
 /* ------------------------------------------------------------------------------------------
  * Offline preparation of a layer (not on the inference path).  These produce the inputs of
  * fq_linear_forward on the device from a weight matrix W and the frame parameters.

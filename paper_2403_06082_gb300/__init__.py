@@ -16,7 +16,7 @@ from dataclasses import dataclass
 __all__ = [
     "FQ_BF16", "FQ_FP32_DEBUG", "FrameQuantError", "Packed", "lib", "lib_path",
     "fq_packed_words", "fq_pack", "fq_workspace_bytes", "fq_linear_forward",
-    "fq_linear_forward_sms", "fq_check",
+    "fq_linear_forward_sms", "fq_linear_forward_ex", "fq_check",
     "fq_status_str", "EXPORTED", "fq_frame_workspace_bytes", "fq_frame_build",
     "fq_coefficients_workspace_bytes", "fq_coefficients", "fq_quantize_rtn",
     "fq_linear_forward_static", "FQ_STATIC_SCRATCH_BYTES", "Frame", "fq_frame_implicit_bytes",
@@ -30,7 +30,7 @@ STATUS = {0: "FQ_OK", 1: "FQ_ERR_INVALID_ARG", 2: "FQ_ERR_ALIGNMENT", 3: "FQ_ERR
           4: "FQ_ERR_WORKSPACE", 5: "FQ_ERR_CUDA", 6: "FQ_ERR_TIMEOUT",
           7: "FQ_ERR_DEVICE_CHECK"}
 EXPORTED = ("fq_packed_words", "fq_pack", "fq_workspace_bytes", "fq_linear_forward",
-            "fq_linear_forward_sms",
+            "fq_linear_forward_sms", "fq_linear_forward_ex",
             "fq_check", "fq_status_str", "fq_frame_workspace_bytes", "fq_frame_build",
             "fq_coefficients_workspace_bytes", "fq_coefficients", "fq_quantize_rtn",
             "fq_linear_forward_static", "fq_frame_implicit_bytes", "fq_frame_implicit",
@@ -58,6 +58,11 @@ class _Rotation(ctypes.Structure):
     _fields_ = [("a", ctypes.c_int32), ("b", ctypes.c_int32), ("gauss_a", ctypes.c_void_p),
                 ("gauss_b", ctypes.c_void_p), ("perm", ctypes.c_void_p),
                 ("signs", ctypes.c_void_p)]
+
+
+class _Opts(ctypes.Structure):
+    _fields_ = [("max_sms", ctypes.c_int32), ("l2_prefetch", ctypes.c_void_p),
+                ("l2_prefetch_bytes", ctypes.c_size_t)]
 
 
 class _Frame(ctypes.Structure):
@@ -98,6 +103,12 @@ def lib() -> ctypes.CDLL:
             ctypes.POINTER(_Packed), ctypes.c_void_p, ctypes.c_int, ctypes.c_void_p,
             ctypes.c_void_p, ctypes.c_void_p, ctypes.c_size_t, ctypes.c_int, ctypes.c_int,
             ctypes.c_void_p]
+        L.fq_linear_forward_ex.restype = ctypes.c_int
+        L.fq_linear_forward_ex.argtypes = [
+            ctypes.c_void_p, ctypes.c_int, ctypes.c_int, ctypes.c_void_p,
+            ctypes.POINTER(_Packed), ctypes.c_void_p, ctypes.c_int, ctypes.c_void_p,
+            ctypes.c_void_p, ctypes.c_void_p, ctypes.c_size_t, ctypes.c_int,
+            ctypes.POINTER(_Opts), ctypes.c_void_p]
         L.fq_check.restype = ctypes.c_int
         L.fq_check.argtypes = [ctypes.c_void_p, ctypes.c_void_p]
         L.fq_status_str.restype = ctypes.c_char_p
@@ -208,6 +219,19 @@ def fq_linear_forward_sms(x, M: int, d_in: int, T_in, C: Packed, T_out_t, d_out:
                                     _ptr(T_out_t), d_out, _ptr(gamma), _ptr(y), _ptr(ws),
                                     ws_bytes, mode, max_sms, _stream(stream)),
         "fq_linear_forward_sms")
+
+
+def fq_linear_forward_ex(x, M: int, d_in: int, T_in, C: Packed, T_out_t, d_out: int, gamma, y,
+                         ws, ws_bytes: int, mode: int = FQ_BF16, max_sms: int = 0,
+                         prefetch=None, stream=None) -> None:
+    """fq_linear_forward with options: an SM budget and a device tensor to warm in L2 while
+    the call runs (typically the next layer's T_in; a hint, results do not depend on it)."""
+    pc = C._c()
+    nb = 0 if prefetch is None else prefetch.numel() * prefetch.element_size()
+    opts = _Opts(max_sms, _ptr(prefetch), nb)
+    _ok(lib().fq_linear_forward_ex(_ptr(x), M, d_in, _ptr(T_in), ctypes.byref(pc), _ptr(T_out_t),
+                                   d_out, _ptr(gamma), _ptr(y), _ptr(ws), ws_bytes, mode,
+                                   ctypes.byref(opts), _stream(stream)), "fq_linear_forward_ex")
 
 
 def fq_linear_forward_static(x, M: int, d_in: int, T_in, C: Packed, T_out_t, d_out: int, gamma,

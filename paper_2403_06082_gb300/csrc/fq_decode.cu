@@ -114,6 +114,8 @@ struct DecArgs {
   int pf_codes;           // prefetch this CTA's later code blocks into L2
   int pf_tout;            // prefetch the T_out^T tiles of its synthesis tasks into L2
   int ext_in;             // bit p: phase p's input was written before the launch (no flags)
+  const char* pf_next;    // a range to warm in L2 from the first synthesis task (next layer)
+  int64_t pf_next_bytes;  // its length, a multiple of 16 (0: none)
 };
 
 // Per-cluster task lists, a kernel parameter: cluster c runs task[off[c]] .. task[off[c+1]-1].
@@ -319,7 +321,19 @@ __global__ void __launch_bounds__(DecCfg<BN>::kThreads, 1)
       const uint64_t pol_w = policy_evict_first();
       int stage = 0;
       uint32_t phase = 0;
-      bool first = true, tout_pf = a.pf_tout > 0;
+      bool first = true, tout_pf = a.pf_tout > 0, next_pf = a.pf_next_bytes > 0;
+      // this CTA's share of the next layer's range, into L2 (64 KiB per prefetch)
+      auto prefetch_next = [&]() {
+        next_pf = false;
+        if (lane != 0) return;
+        const int64_t per = ((a.pf_next_bytes + gridDim.x - 1) / gridDim.x + 15) & ~15ll;
+        const int64_t b0 = static_cast<int64_t>(blockIdx.x) * per;
+        const int64_t b1 = min(a.pf_next_bytes, b0 + per);
+        for (int64_t o = b0; o < b1; o += 65536)
+          asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(a.pf_next + o),
+                       "r"(static_cast<uint32_t>(b1 - o < 65536 ? b1 - o : 65536))
+                       : "memory");
+      };
       // bit s: stage s filled / its last fill a code block / parity of that fill's phase of
       // fullA (weight tile) or cfull (code block)
       uint32_t used = 0, last_code = 0, last_par = 0, cpar = 0;
@@ -330,6 +344,7 @@ __global__ void __launch_bounds__(DecCfg<BN>::kThreads, 1)
         const DecPhase ph = phase_of(a, t.p);
         int k0, k1;
         krange(ph, k0, k1);
+        if (next_pf && t.p == 2) prefetch_next();
         if (tout_pf && t.p >= 1) {
           tout_pf = false;
           // this CTA's synthesis tiles, in the order they will be read, into L2
@@ -397,6 +412,7 @@ __global__ void __launch_bounds__(DecCfg<BN>::kThreads, 1)
           }
         }
       }
+      if (next_pf) prefetch_next();      // a CTA without synthesis tasks still takes its share
       // no copy may still be landing when the CTA leaves: the last fill of every stage (no
       // later phase of its barrier exists, so the parity wait is exact)
       for (int s = 0; s < S_ && lane == 0; ++s)
@@ -1005,6 +1021,9 @@ fq_status run(const CUtensorMap* m, DecArgs& a, const int* R, const int* K, int 
     const int64_t tout_bytes = static_cast<int64_t>(R[2]) * K[2] * 2;
     a.pf_codes = code_bytes <= kL2PrefetchBudget;
     a.pf_tout = code_bytes + tout_bytes <= kL2PrefetchBudget;
+    // the next layer's range only when this synthesis reads from L2 (HBM idle), and at most
+    // the warming budget
+    a.pf_next_bytes = a.pf_tout ? std::min<int64_t>(a.pf_next_bytes, kL2PrefetchBudget) : 0;
   }
   cudaLaunchConfig_t cfg{};
   cfg.gridDim = dim3(static_cast<unsigned>(plan->ncl * plan->S));
@@ -1040,7 +1059,8 @@ namespace {
 // already in the workspace and u left there.
 fq_status launch_decode(const void* x, int M, int d_in, const void* T_in, const fq_packed& Cq,
                         const void* T_out_t, int d_out, const float* gamma, void* y, char* ws,
-                        size_t ws_bytes, int max_sms, bool core_only, cudaStream_t s) {
+                        size_t ws_bytes, int max_sms, bool core_only, const void* pf,
+                        size_t pf_bytes, cudaStream_t s) {
   const int n_in = Cq.n_in, n_out = Cq.n_out;
   const DecWs L = dec_ws(M, n_in, n_out);
   if (ws_bytes < L.total) return FQ_ERR_WORKSPACE;
@@ -1070,6 +1090,8 @@ fq_status launch_decode(const void* x, int M, int d_in, const void* T_in, const 
   a.gen = reinterpret_cast<uint32_t*>(ws + kWsGen);
   a.done = reinterpret_cast<uint32_t*>(ws + kWsDone);
   a.ext_in = core_only ? 2 : 0;
+  a.pf_next = static_cast<const char*>(pf);
+  a.pf_next_bytes = pf ? static_cast<int64_t>(pf_bytes) : 0;
 
   CUtensorMap m[5];
   if (!tmap_bf16(&m[2], ws + L.z, M, n_in, BN) || !tmap_bf16(&m[4], ws + L.u, M, n_out, BN))
@@ -1095,15 +1117,15 @@ fq_status launch_decode(const void* x, int M, int d_in, const void* T_in, const 
 fq_status launch_decode_forward(const void* x, int M, int d_in, const void* T_in,
                                 const fq_packed& Cq, const void* T_out_t, int d_out,
                                 const float* gamma, void* y, char* ws, size_t ws_bytes,
-                                int max_sms, cudaStream_t s) {
+                                int max_sms, const void* pf, size_t pf_bytes, cudaStream_t s) {
   return launch_decode(x, M, d_in, T_in, Cq, T_out_t, d_out, gamma, y, ws, ws_bytes, max_sms,
-                       false, s);
+                       false, pf, pf_bytes, s);
 }
 
 fq_status launch_decode_core(int M, const fq_packed& Cq, const float* gamma, char* ws,
                              size_t ws_bytes, int max_sms, cudaStream_t s) {
   return launch_decode(nullptr, M, 0, nullptr, Cq, nullptr, 0, gamma, nullptr, ws, ws_bytes,
-                       max_sms, true, s);
+                       max_sms, true, nullptr, 0, s);
 }
 
 size_t decode_core_z_offset() { return kWsHeader; }

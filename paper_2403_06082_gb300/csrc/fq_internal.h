@@ -48,11 +48,13 @@ cudaError_t launch_debug_forward(const float* x, int M, int d_in, const float* T
 
 // ---- fq_decode.cu: bf16 path for small batches (one fused persistent kernel)
 size_t decode_workspace_bytes(int M, int d_in, int n_in, int n_out, int d_out);
-// max_sms > 0 caps the SMs a call's kernels occupy (the grid and the plan)
+// max_sms > 0 caps the SMs a call's kernels occupy (the grid and the plan); pf/pf_bytes is an
+// optional device range (16-byte aligned, multiple of 16 bytes) to warm in L2 during the
+// synthesis when this layer's T_out^T is itself warmed during the code product
 fq_status launch_decode_forward(const void* x, int M, int d_in, const void* T_in,
                                 const fq_packed& C, const void* T_out_t, int d_out,
                                 const float* gamma, void* y, char* ws, size_t ws_bytes,
-                                int max_sms, cudaStream_t s);
+                                int max_sms, const void* pf, size_t pf_bytes, cudaStream_t s);
 
 // The code product alone (z already in the workspace at decode_core_z_offset(), u left at
 // decode_core_u_offset()), for the structured-frame forward.

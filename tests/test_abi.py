@@ -138,3 +138,17 @@ def test_implicit_host_validation_without_gpu(L):
     assert _call_implicit(L, ws=0x10010) == 2
     assert _call_implicit(L, M=65) == 3                             # decode batches only
     assert _call_implicit(L, ws_bytes=1024) == 4
+
+
+def test_forward_ex_host_validation_without_gpu(L):
+    def ex(opts, **kw):
+        C = _P(0x5000, 0x6000, 0x7000, 288, 288)
+        a = dict(x=0x1000, M=8, d_in=256, T_in=0x2000, T_out=0x3000, d_out=256, y=0x4000)
+        a.update(kw)
+        return L.fq_linear_forward_ex(a["x"], a["M"], a["d_in"], a["T_in"], ctypes.byref(C),
+                                      a["T_out"], a["d_out"], None, a["y"], 0x10000, 1 << 30, 0,
+                                      ctypes.byref(opts) if opts is not None else None, None)
+    assert ex(fq._Opts(-1, None, 0)) == 1                  # negative SM budget
+    assert ex(fq._Opts(0, None, 4096)) == 1                # range without a pointer
+    assert ex(fq._Opts(0, 0x9008, 4096)) == 2              # range start not 16-byte aligned
+    assert ex(fq._Opts(0, 0x9000, 4096), x=None) == 1

@@ -94,3 +94,22 @@ def test_budget_fp32_debug_and_negative():
     assert fq.fq_check(ws) == 0
     assert rel_frobenius(y.double().cpu().numpy(), reference(L, X, False)) <= 1e-5
     assert np.isfinite(y.cpu().numpy()).all()
+
+
+def test_l2_prefetch_hint_changes_nothing():
+    """The chaining hint (the next layer's T_in) only warms L2: outputs are bitwise equal."""
+    Lq, Lk = oracle_layer("llama2_7b_decode", "q"), oracle_layer("llama2_7b_decode", "k")
+    Dq, Dk = DeviceLayer(Lq, BF16), DeviceLayer(Lk, BF16)
+    X = activations("llama2_7b_decode", "q", 16)
+    x = torch.from_numpy(X).to(DEV, BF16)
+    nb = fq.fq_workspace_bytes(16, Lq.d_in, Lq.n_in, Lq.n_out, Lq.d_out, 0)
+    ws = torch.zeros(nb, dtype=torch.uint8, device=DEV)
+    outs = []
+    for hint in (None, Dk.T_in, Dk.T_in[:1000]):
+        y = torch.full((16, Lq.d_out), float("nan"), dtype=BF16, device=DEV)
+        fq.fq_linear_forward_ex(x, 16, Lq.d_in, Dq.T_in, Dq.C, Dq.T_out_t, Lq.d_out, None, y, ws,
+                                nb, prefetch=hint)
+        assert fq.fq_check(ws) == 0
+        outs.append(y.cpu())
+    assert torch.equal(outs[0], outs[1]) and torch.equal(outs[0], outs[2])
+    assert rel_frobenius(outs[0].double().numpy(), reference(Lq, X, False)) <= 1e-2
