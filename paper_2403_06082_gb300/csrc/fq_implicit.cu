@@ -433,7 +433,8 @@ fq_status fq_frame_implicit(int k, int rho, int d, const fq_rotation* rot, void*
     std::vector<char> seen(d, 0);
     for (int i = 0; i < d; ++i) {
       const int64_t p = rot->perm[i];
-      if (p < 0 || p >= d || seen[p]) return FQ_ERR_INVALID_ARG;
+      if (p < 0 || p >= d || seen[p] || (rot->signs[i] != 1.0 && rot->signs[i] != -1.0))
+        return FQ_ERR_INVALID_ARG;
       seen[p] = 1;
     }
   }
@@ -474,7 +475,7 @@ fq_status fq_frame_implicit(int k, int rho, int d, const fq_rotation* rot, void*
     pm.resize(d);
     ipm.resize(d);
     for (int i = 0; i < d; ++i) {
-      sg[i] = rot->signs[i] < 0 ? -1.f : 1.f;
+      sg[i] = static_cast<float>(rot->signs[i]);
       pm[i] = static_cast<int32_t>(rot->perm[i]);
       ipm[pm[i]] = i;
     }

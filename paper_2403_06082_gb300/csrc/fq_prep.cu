@@ -350,8 +350,13 @@ fq_status fq_frame_build(int k, int rho, int d, const fq_rotation* rot, float* T
     if (!rot->gauss_a || !rot->gauss_b || !rot->perm || !rot->signs || rot->a <= 0 ||
         rot->b <= 0 || static_cast<int64_t>(rot->a) * rot->b != d)
       return FQ_ERR_INVALID_ARG;
-    for (int i = 0; i < d; ++i)
-      if (rot->perm[i] < 0 || rot->perm[i] >= d) return FQ_ERR_INVALID_ARG;
+    std::vector<char> seen(d, 0);
+    for (int i = 0; i < d; ++i) {
+      const int64_t p = rot->perm[i];
+      if (p < 0 || p >= d || seen[p] || (rot->signs[i] != 1.0 && rot->signs[i] != -1.0))
+        return FQ_ERR_INVALID_ARG;
+      seen[p] = 1;
+    }
   }
   const FrameWs L = frame_ws(k, rho, d, rot ? rot->a : 0, rot ? rot->b : 0);
   if (!ws || ws_bytes < L.total) return FQ_ERR_WORKSPACE;

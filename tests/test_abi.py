@@ -152,3 +152,30 @@ def test_forward_ex_host_validation_without_gpu(L):
     assert ex(fq._Opts(0, None, 4096)) == 1                # range without a pointer
     assert ex(fq._Opts(0, 0x9008, 4096)) == 2              # range start not 16-byte aligned
     assert ex(fq._Opts(0, 0x9000, 4096), x=None) == 1
+
+
+def test_rotation_validation_without_gpu(L):
+    """A rotation whose perm is not a permutation, or whose signs are not +-1, is refused on
+    the host by both frame builders."""
+    import numpy as np
+    a = b = 16
+    ga = np.eye(a)
+    gb = np.eye(b)
+
+    def rot(perm, signs):
+        keep = [np.ascontiguousarray(ga), np.ascontiguousarray(gb),
+                np.ascontiguousarray(perm, np.int64), np.ascontiguousarray(signs, np.float64)]
+        return fq._Rotation(a, b, *(k.ctypes.data for k in keep)), keep
+
+    good_perm, good_signs = np.arange(256), np.ones(256)
+    dup = good_perm.copy()
+    dup[3] = 4
+    half = good_signs.copy()
+    half[7] = 0.5
+    out = fq._Frame()
+    for perm, signs in ((dup, good_signs), (good_perm, half)):
+        r, keep = rot(perm, signs)
+        assert L.fq_frame_build(18, 16, 256, ctypes.byref(r), 0x1000, 0x2000, 1 << 30, None) == 1
+        assert L.fq_frame_implicit(18, 16, 256, ctypes.byref(r), 0x1000, 1 << 30,
+                                   ctypes.byref(out), None) == 1
+        del keep
