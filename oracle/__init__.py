@@ -9,6 +9,7 @@ it and shares no code with it; the two meet only in the seeded input generators 
   pack     the packed 2-bit code layout declared by the library header
   forward  analysis -> dequantized product -> synthesis (Sec. 3.2)
   layer    one call that builds a whole quantized layer from a workload
+  gptq     the frame-domain GPTQ quantizer of Algorithm 1, step 4 (calibration Hessian)
 
 Parity status: every function is pinned by tests/test_oracle_*.py except wiener_gain's formula,
 which the paper does not print ("parity unpinned" for the formula itself; its gamma == 1

@@ -16,7 +16,7 @@ import numpy as np
 
 import workloads as wlmod
 
-from . import frames, pack, quant
+from . import frames, gptq, pack, quant
 
 
 @dataclass
@@ -49,21 +49,27 @@ class QuantLayer:
 
 
 def build(W: np.ndarray, k_in: int, k_out: int, rho: int = wlmod.RHO, *, rot_in=None,
-          rot_out=None, clip: bool = False, name: str = "layer") -> QuantLayer:
+          rot_out=None, clip: bool = False, name: str = "layer", A_calib=None) -> QuantLayer:
+    """With A_calib (calibration tokens, one per row) the codes come from the frame-domain GPTQ
+    of Algorithm 1, step 4, against H = (T_in A^T)(T_in A^T)^T; otherwise from per-row RTN."""
     d_out, d_in = W.shape
     T_in = frames.frame(k_in, rho if k_in > 1 else d_in, d_in, rot_in)
     T_out = frames.frame(k_out, rho if k_out > 1 else d_out, d_out, rot_out)
     C = quant.coefficients(W, T_in, T_out)
     if clip:
         C = quant.clip_2sigma(C)
-    codes, scale, zero = quant.rtn(C)
+    if A_calib is None:
+        codes, scale, zero = quant.rtn(C)
+    else:
+        C_prev = T_in @ np.asarray(A_calib, dtype=np.float64).T
+        codes, scale, zero = gptq.gptq(C, gptq.hessian(C_prev))
     gamma = quant.wiener_gain(C, scale)
     return QuantLayer(name, d_in, d_out, k_in, k_out, rho, T_in, T_out, W, C, codes, scale,
                       zero, gamma)
 
 
 def from_workload(wl_key: str, layer_name: str, r: Fraction | None = None, *,
-                  rotate: bool = True, clip: bool = False) -> QuantLayer:
+                  rotate: bool = True, clip: bool = False, calib_tokens: int = 0) -> QuantLayer:
     """Quantized layer for one layer of a workload, with the workload's seed and draws."""
     wl = wlmod.WORKLOADS[wl_key]
     layer = next(l for l in wl.layers if l.name == layer_name)
@@ -78,5 +84,6 @@ def from_workload(wl_key: str, layer_name: str, r: Fraction | None = None, *,
     if rotate:
         rot_in = wlmod.rotation_draws(wl.seed, wl.key, layer.name, "in", d=layer.d_in)
         rot_out = wlmod.rotation_draws(wl.seed, wl.key, layer.name, "out", d=layer.d_out)
+    A = wlmod.calibration(wl, layer, calib_tokens) if calib_tokens else None
     return build(W, k_in, k_out, rot_in=rot_in, rot_out=rot_out, clip=clip,
-                 name=f"{wl_key}/{layer_name}")
+                 name=f"{wl_key}/{layer_name}", A_calib=A)

@@ -159,6 +159,20 @@ def activations(wl: Workload, layer: Layer, M: int) -> np.ndarray:
     return round_bf16(X)
 
 
+def calibration(wl: Workload, layer: Layer, N: int) -> np.ndarray:
+    """N calibration tokens (N x d_in) with the distribution of `activations`, drawn from their
+    own stream (the quantizer's A_prev of Algorithm 1)."""
+    g = rng(wl.seed, wl.key, layer.name, "calibration", str(N))
+    X = g.standard_normal((N, layer.d_in))
+    if wl.act == "normal_bf16_outlier30":
+        go = rng(wl.seed, wl.key, layer.name, "X-outlier-channels")
+        ch = go.choice(layer.d_in, max(1, layer.d_in // 100), replace=False)
+        X[:, ch] *= 30.0
+    elif wl.act != "normal_bf16":
+        raise ValueError(wl.act)
+    return round_bf16(X)
+
+
 @dataclass
 class RotationDraws:
     """Raw random numbers for one d x d random rotation: two Gaussian matrices (a x a, b x b,
