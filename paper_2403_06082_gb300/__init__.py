@@ -21,6 +21,8 @@ __all__ = [
     "fq_coefficients_workspace_bytes", "fq_coefficients", "fq_quantize_rtn",
     "fq_linear_forward_static", "FQ_STATIC_SCRATCH_BYTES", "Frame", "fq_frame_implicit_bytes",
     "fq_frame_implicit", "fq_implicit_workspace_bytes", "fq_linear_forward_implicit",
+    "fq_reconstruct_workspace_bytes", "fq_reconstruct_weight", "fq_dense_workspace_bytes",
+    "fq_dense_forward",
 ]
 FQ_STATIC_SCRATCH_BYTES = 16 << 20
 
@@ -34,7 +36,9 @@ EXPORTED = ("fq_packed_words", "fq_pack", "fq_workspace_bytes", "fq_linear_forwa
             "fq_check", "fq_status_str", "fq_frame_workspace_bytes", "fq_frame_build",
             "fq_coefficients_workspace_bytes", "fq_coefficients", "fq_quantize_rtn",
             "fq_linear_forward_static", "fq_frame_implicit_bytes", "fq_frame_implicit",
-            "fq_implicit_workspace_bytes", "fq_linear_forward_implicit")
+            "fq_implicit_workspace_bytes", "fq_linear_forward_implicit",
+            "fq_reconstruct_workspace_bytes", "fq_reconstruct_weight", "fq_dense_workspace_bytes",
+            "fq_dense_forward")
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
 
@@ -144,6 +148,18 @@ def lib() -> ctypes.CDLL:
             ctypes.c_void_p, ctypes.c_int, ctypes.POINTER(_Frame), ctypes.POINTER(_Packed),
             ctypes.POINTER(_Frame), ctypes.c_void_p, ctypes.c_void_p, ctypes.c_void_p,
             ctypes.c_size_t, ctypes.c_int, ctypes.c_void_p]
+        L.fq_reconstruct_workspace_bytes.restype = ctypes.c_size_t
+        L.fq_reconstruct_workspace_bytes.argtypes = [ctypes.c_int] * 4
+        L.fq_reconstruct_weight.restype = ctypes.c_int
+        L.fq_reconstruct_weight.argtypes = [
+            ctypes.c_void_p, ctypes.POINTER(_Packed), ctypes.c_void_p, ctypes.c_int, ctypes.c_int,
+            ctypes.c_void_p, ctypes.c_void_p, ctypes.c_void_p, ctypes.c_size_t, ctypes.c_void_p]
+        L.fq_dense_workspace_bytes.restype = ctypes.c_size_t
+        L.fq_dense_workspace_bytes.argtypes = [ctypes.c_int] * 3
+        L.fq_dense_forward.restype = ctypes.c_int
+        L.fq_dense_forward.argtypes = [
+            ctypes.c_void_p, ctypes.c_int, ctypes.c_int, ctypes.c_void_p, ctypes.c_int,
+            ctypes.c_void_p, ctypes.c_void_p, ctypes.c_size_t, ctypes.c_void_p]
         L.fq_quantize_rtn.restype = ctypes.c_int
         L.fq_quantize_rtn.argtypes = [ctypes.c_void_p, ctypes.c_int, ctypes.c_int,
                                       ctypes.c_void_p, ctypes.c_void_p, ctypes.c_void_p,
@@ -331,6 +347,30 @@ def fq_linear_forward_implicit(x, M: int, F_in: Frame, C: Packed, F_out: Frame, 
                                          ctypes.byref(F_out.c), _ptr(gamma), _ptr(y), _ptr(ws),
                                          ws_bytes, max_sms, _stream(stream)),
         "fq_linear_forward_implicit")
+
+
+def fq_reconstruct_workspace_bytes(d_in: int, n_in: int, n_out: int, d_out: int) -> int:
+    return lib().fq_reconstruct_workspace_bytes(d_in, n_in, n_out, d_out)
+
+
+def fq_reconstruct_weight(T_in, C: Packed, T_out_t, d_in: int, d_out: int, gamma, W_hat, ws,
+                          ws_bytes: int, stream=None) -> None:
+    """W_hat = T_out^T diag(gamma) C_hat T_in (bf16 d_out x d_in), include/framequant_dense.h."""
+    pc = C._c()
+    _ok(lib().fq_reconstruct_weight(_ptr(T_in), ctypes.byref(pc), _ptr(T_out_t), d_in, d_out,
+                                    _ptr(gamma), _ptr(W_hat), _ptr(ws), ws_bytes,
+                                    _stream(stream)), "fq_reconstruct_weight")
+
+
+def fq_dense_workspace_bytes(M: int, d_in: int, d_out: int) -> int:
+    return lib().fq_dense_workspace_bytes(M, d_in, d_out)
+
+
+def fq_dense_forward(x, M: int, d_in: int, W_hat, d_out: int, y, ws, ws_bytes: int,
+                     stream=None) -> None:
+    """y = x W_hat^T on the tensor cores (include/framequant_dense.h)."""
+    _ok(lib().fq_dense_forward(_ptr(x), M, d_in, _ptr(W_hat), d_out, _ptr(y), _ptr(ws), ws_bytes,
+                               _stream(stream)), "fq_dense_forward")
 
 
 def fq_coefficients_workspace_bytes(d_out: int, n_in: int) -> int:

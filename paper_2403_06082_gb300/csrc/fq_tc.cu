@@ -39,6 +39,7 @@
 
 #include "fq_device.cuh"
 #include "fq_internal.h"
+#include "framequant_dense.h"
 
 namespace fq {
 namespace {
@@ -670,6 +671,60 @@ fq_status run_forward(const CUtensorMap* maps, PhaseArgs* a, int max_sms, cudaSt
   return FQ_OK;
 }
 
+// The dense product of the weight-reconstruction path: one analysis-phase kernel with the
+// reconstructed weight as its A operand (the per-tile sums of the output it also writes go to
+// the workspace and are not used).
+WsLayout dense_ws_layout(int M, int d_out) {
+  WsLayout L{};
+  size_t off = kWsHeader;
+  L.zsum = off;
+  off += round_up(ceil_div(d_out, kBM) * M * 4, 256);
+  const int BN = pick_bn(M);
+  const int64_t tiles = ceil_div(d_out, kBM) * ceil_div(M, BN);
+  int64_t slots = 0, max_tiles = 0;
+  if (tiles < kMaxSplitSms) {
+    slots = std::min<int64_t>(kMaxSplitSms, tiles * kMaxSplits);
+    max_tiles = tiles;
+  }
+  L.cnt = off;
+  off += round_up(max_tiles * 4, 256);
+  L.part = off;
+  off += static_cast<size_t>(slots) * BN * kBM * 4;
+  L.total = off;
+  return L;
+}
+
+template <int BN>
+fq_status run_dense(const CUtensorMap& tmW, const CUtensorMap& tmX, PhaseArgs& a,
+                    cudaStream_t s) {
+  const DeviceInfo d = device_info();
+  if (prepare_kernel<kAnalysis, BN>(d.dev) != cudaSuccess) return FQ_ERR_CUDA;
+  int grid = 0;
+  plan_phase<kAnalysis, BN>(a, d, grid);
+  return launch_phase<kAnalysis, BN>(tmW, tmX, a, grid, s) == cudaSuccess ? FQ_OK : FQ_ERR_CUDA;
+}
+
+fq_status launch_tc_dense(const void* x, int M, int d_in, const void* W, int d_out, void* y,
+                          char* ws, size_t ws_bytes, cudaStream_t s) {
+  const WsLayout L = dense_ws_layout(M, d_out);
+  if (ws_bytes < L.total) return FQ_ERR_WORKSPACE;
+  const int BN = pick_bn(M);
+  PhaseArgs a{};
+  a.R = d_out;
+  a.K = d_in;
+  a.M = M;
+  a.out = reinterpret_cast<__nv_bfloat16*>(y);
+  a.zsum_part = reinterpret_cast<float*>(ws + L.zsum);
+  a.status = reinterpret_cast<int32_t*>(ws);
+  a.cnt = reinterpret_cast<uint32_t*>(ws + L.cnt);
+  a.part = reinterpret_cast<float*>(ws + L.part);
+  CUtensorMap mW, mX;
+  if (!make_tmap(&mW, W, d_out, d_in, kBM) || !make_tmap(&mX, x, M, d_in, BN)) return FQ_ERR_CUDA;
+  return BN == 128 ? run_dense<128>(mW, mX, a, s) : run_dense<256>(mW, mX, a, s);
+}
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
 }  // namespace
 
 size_t tc_workspace_bytes(int M, int d_in, int n_in, int n_out, int d_out) {
@@ -720,3 +775,30 @@ fq_status launch_tc_forward(const void* x, int M, int d_in, const void* T_in,
 }
 
 }  // namespace fq
+
+extern "C" {
+
+size_t fq_dense_workspace_bytes(int M, int d_in, int d_out) {
+  if (M <= 0 || d_in <= 0 || d_out <= 0) return 0;
+  return fq::dense_ws_layout(M, d_out).total;
+}
+
+fq_status fq_dense_forward(const void* x, int M, int d_in, const void* W_hat, int d_out, void* y,
+                           void* ws, size_t ws_bytes, fq_stream_t stream) {
+  if (!x || !W_hat || !y || M <= 0 || d_in <= 0 || d_out <= 0) return FQ_ERR_INVALID_ARG;
+  if (d_in % 8 || d_out % 8 || !fq::aligned16(x) || !fq::aligned16(W_hat) || !fq::aligned16(y))
+    return FQ_ERR_ALIGNMENT;
+  if (!ws) return FQ_ERR_WORKSPACE;
+  if ((reinterpret_cast<uintptr_t>(ws) & 255u) != 0) return FQ_ERR_ALIGNMENT;
+  if (ws_bytes < fq_dense_workspace_bytes(M, d_in, d_out)) return FQ_ERR_WORKSPACE;
+  int dev = 0, major = 0, minor = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess ||
+      cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, dev) != cudaSuccess ||
+      cudaDeviceGetAttribute(&minor, cudaDevAttrComputeCapabilityMinor, dev) != cudaSuccess)
+    return FQ_ERR_CUDA;
+  if (major * 10 + minor != 103) return FQ_ERR_UNSUPPORTED;
+  return fq::launch_tc_dense(x, M, d_in, W_hat, d_out, y, static_cast<char*>(ws), ws_bytes,
+                             reinterpret_cast<cudaStream_t>(stream));
+}
+
+}  // extern "C"

@@ -8,14 +8,16 @@ import pytest
 
 import paper_2403_06082_gb300 as fq
 
-HEADER = os.path.join(os.path.dirname(os.path.dirname(os.path.abspath(__file__))), "include",
-                      "framequant.h")
+INCLUDE = os.path.join(os.path.dirname(os.path.dirname(os.path.abspath(__file__))), "include")
 
 
 def _declared():
-    text = open(HEADER).read()
-    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
-    return sorted(set(re.findall(r"\b(fq_[a-z_]+)\s*\(", text)))
+    names = set()
+    for f in sorted(os.listdir(INCLUDE)):
+        if f.endswith(".h"):
+            text = re.sub(r"/\*.*?\*/", "", open(os.path.join(INCLUDE, f)).read(), flags=re.S)
+            names |= set(re.findall(r"\b(fq_[a-z_]+)\s*\(", text))
+    return sorted(names)
 
 
 @pytest.fixture(scope="module")
@@ -179,3 +181,20 @@ def test_rotation_validation_without_gpu(L):
         assert L.fq_frame_implicit(18, 16, 256, ctypes.byref(r), 0x1000, 1 << 30,
                                    ctypes.byref(out), None) == 1
         del keep
+
+
+def test_dense_path_sizes_and_validation_without_gpu(L):
+    assert fq.fq_dense_workspace_bytes(0, 256, 256) == 0
+    assert fq.fq_dense_workspace_bytes(2048, 4096, 4096) > 0
+    assert fq.fq_reconstruct_workspace_bytes(4096, 4512, 4512, 4096) >= 4096 * 4096 * 2 * 2
+    assert fq.fq_reconstruct_workspace_bytes(0, 4512, 4512, 4096) == 0
+    C = _P(0x5000, 0x6000, 0x7000, 288, 288)
+    assert L.fq_reconstruct_weight(None, ctypes.byref(C), 0x3000, 256, 256, None, 0x4000,
+                                   0x10000, 1 << 30, None) == 1
+    assert L.fq_reconstruct_weight(0x2000, ctypes.byref(C), 0x3000, 256, 256, None, 0x4002,
+                                   0x10000, 1 << 30, None) == 2
+    assert L.fq_reconstruct_weight(0x2000, ctypes.byref(C), 0x3000, 256, 256, None, 0x4000,
+                                   0x10000, 1024, None) == 4
+    assert L.fq_dense_forward(None, 8, 256, 0x2000, 256, 0x4000, 0x10000, 1 << 30, None) == 1
+    assert L.fq_dense_forward(0x1000, 8, 260, 0x2000, 256, 0x4000, 0x10000, 1 << 30, None) == 2
+    assert L.fq_dense_forward(0x1000, 8, 256, 0x2000, 256, 0x4000, 0x10000, 64, None) == 4
