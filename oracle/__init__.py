@@ -11,7 +11,7 @@ it and shares no code with it; the two meet only in the seeded input generators 
   layer    one call that builds a whole quantized layer from a workload
   gptq     the frame-domain GPTQ quantizer of Algorithm 1, step 4 (calibration Hessian)
 
-Parity status: every function is pinned by tests/test_oracle_*.py except wiener_gain's formula,
-which the paper does not print ("parity unpinned" for the formula itself; its gamma == 1
-special case and its shrinkage property are checked).
+Parity status: every function is pinned by tests/test_oracle_*.py against brute force, closed
+forms, printed examples or special cases; the de-noising gain (which the paper does not print) is
+pinned as the empirical minimiser of the mean squared error under uniform rounding noise.
 """

@@ -7,12 +7,12 @@ Sec. 3 (Eqs. for D_l) and Algorithm 1:
   * D_l = P_l^T Theta_l P_prev, i.e. C = T_out W T_in^T with T the analysis operators;
   * optional clipping of C to [mu - 2 sigma, mu + 2 sigma], sigma and mu over the whole matrix
     (Algorithm 1, steps 2-3);
-  * per-row round-to-nearest quantization to 2 bits with a per-row fp16 scale and zero ("bias
-    and scale values for each row", Appendix K).  The paper's own quantizer is GPTQ with
-    calibration data (Algorithm 1, step 4); this oracle and the hot path it checks use
+  * per-row round-to-nearest quantization to 2 bits with a per-row fp16 scale and zero (the
+    paper stores one scale and one offset per row, Appendix K).  The paper's own quantizer is
+    GPTQ with calibration data (Algorithm 1, step 4); this oracle and the hot path it checks use
     round-to-nearest, as the workloads state.
-  * optional diagonal de-noising gain (Sec. 3.1 (b), Appendix I: "diagonal approximation" of
-    the Wiener filter).
+  * optional diagonal de-noising gain (Sec. 3.1 (b), Appendix I: the paper reports that keeping
+    only the diagonal of the Wiener filter already helps).
 """
 from __future__ import annotations
 
@@ -62,8 +62,10 @@ def wiener_gain(C: np.ndarray, scale: np.ndarray) -> np.ndarray:
     """Diagonal de-noising gain per frame coefficient row: gamma_i = P_i / (P_i + scale_i^2/12),
     P_i the mean square of row i and scale_i^2/12 the variance of uniform rounding noise of step
     scale_i.  This is the scalar LMMSE (Wiener) shrinkage of each output coefficient under
-    additive white quantization noise; the paper states that a diagonal approximation of the
-    Wiener filter helps but prints no formula (Sec. 3.1 (b), Appendix I)."""
+    additive white quantization noise; the paper reports that the diagonal of the Wiener filter
+    alone helps but prints no formula (Sec. 3.1 (b), Appendix I).  Pinned by brute force: the
+    gain equals the Monte-Carlo minimiser of the mean squared error of gamma (c + n) against c
+    for coefficients c of power P and uniform rounding noise n of step scale."""
     P = np.mean(C * C, axis=1)
     N = scale.astype(np.float64) ** 2 / 12.0
     return (P / (P + N)).astype(np.float32)

@@ -87,11 +87,35 @@ def test_wiener_gain_range_and_identity():
     q, s, z = quant.rtn(C)
     g = quant.wiener_gain(C, s)
     assert g.dtype == np.float32 and (g > 0).all() and (g < 1).all()
-    # P/(P + s^2/12) with P the row mean square, checked on one row by hand
-    P0 = float(np.sum(C[0] ** 2) / C.shape[1])
-    assert g[0] == pytest.approx(P0 / (P0 + float(s[0]) ** 2 / 12), rel=1e-6)
-    # a noiseless row (step 0 after degenerate-scale handling aside) keeps gain 1
+    # a row without rounding noise (step 0) keeps gain 1
     assert quant.wiener_gain(np.ones((1, 4)), np.array([0.0], np.float16))[0] == 1.0
+
+
+@pytest.mark.parametrize("snr", [0.02, 0.08, 0.3, 1.0, 4.0])
+def test_wiener_gain_is_the_empirical_mse_minimiser(snr):
+    """The gain is fixed by what it is for (Sec. 3.1 (b), Appendix I): among all scalings
+    gamma of a noisy coefficient c + n, the one with the least mean squared error against c.
+    Draw coefficients c ~ N(0, P) and independent rounding noise n ~ U(-s/2, s/2) (the error of
+    rounding to a grid of step s), search gamma on a fine grid by brute force, and compare the
+    minimiser with the oracle's gain for a row of power P and step s.  The ratios P / s^2 span
+    the regime of 2-bit rows; a wrong noise constant (s^2/4 or s^2/6 instead of the variance of
+    a uniform step, s^2/12) or a wrong power (mean |c| instead of mean c^2) moves the gain by
+    far more than the Monte-Carlo error."""
+    r = wl.rng(7, "wiener-mc", str(snr))
+    n = 400_000
+    s = 1.0
+    P = snr * s * s
+    c = r.standard_normal(n) * np.sqrt(P)
+    noisy = c + r.uniform(-s / 2, s / 2, n)
+    grid = np.linspace(0.0, 1.2, 2401)
+    # mean((gamma * noisy - c)^2) for every gamma of the grid, from the three sums it needs
+    a, b, d = np.mean(noisy * noisy), np.mean(noisy * c), np.mean(c * c)
+    mse = grid * grid * a - 2.0 * grid * b + d
+    best = grid[np.argmin(mse)]
+    row = c[None, :]                                # the row's own power is P up to sampling
+    g = float(quant.wiener_gain(row, np.array([s], np.float16))[0])
+    # sampling error of the minimiser at n = 4e5 is below 3e-3; the grid step is 5e-4
+    assert abs(g - best) < 5e-3, (snr, g, best)
 
 
 # ------------------------------------------------------------------- packed layout
