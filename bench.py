@@ -172,15 +172,15 @@ def prepare_layer(fq, wl, torch, wk, layer, r, dev):
     del C
     words = torch.empty(fq.fq_packed_words(n_out, n_in), dtype=torch.int32, device=dev)
     status = torch.zeros(1, dtype=torch.int32, device=dev)
-    fq.fq_pack(codes, n_out, n_in, words, status)
+    C_packed = fq.fq_pack(codes, scale, zero, n_out, n_in, words, status)
     if fq.fq_check(status) != 0:
-        raise RuntimeError("fq_pack reported out-of-range codes")
+        raise RuntimeError("fq_pack reported out-of-range codes or a non-finite scale or zero")
     del codes
     return {
         "name": layer.name, "d_in": layer.d_in, "d_out": layer.d_out, "n_in": n_in,
         "n_out": n_out, "k_in": k_in, "k_out": k_out,
         "T_in": T_in.to(torch.bfloat16), "T_out_t": T_out.t().contiguous().to(torch.bfloat16),
-        "C": fq.Packed(words, scale, zero, n_out, n_in), "gamma": gamma,
+        "C": C_packed, "gamma": gamma,
     }
 
 
@@ -571,16 +571,16 @@ def prepare_layer_random_codes(fq, wl, torch, wk, layer, r, dev):
     codes = torch.from_numpy(wl.random_codes(wk.seed, wk.key, layer.name, str(r), n_out=n_out,
                                              n_in=n_in)).to(dev)
     words = torch.empty(fq.fq_packed_words(n_out, n_in), dtype=torch.int32, device=dev)
-    fq.fq_pack(codes, n_out, n_in, words)
-    del codes
     sc, ze = wl.random_scale_zero(wk.seed, wk.key, layer.name, n_out=n_out, mag=0.01)
     scale = torch.from_numpy(sc.view(np.int16)).to(dev)
     zero = torch.from_numpy(ze.view(np.int16)).to(dev)
+    C_packed = fq.fq_pack(codes, scale, zero, n_out, n_in, words)
+    del codes
     gamma = torch.ones(n_out, dtype=torch.float32, device=dev)
     return {
         "name": layer.name, "d_in": layer.d_in, "d_out": layer.d_out, "n_in": n_in,
         "n_out": n_out, "k_in": k_in, "k_out": k_out, "T_in": T_in, "T_out_t": T_out_t,
-        "C": fq.Packed(words, scale, zero, n_out, n_in), "gamma": gamma,
+        "C": C_packed, "gamma": gamma,
     }
 
 

@@ -2,7 +2,7 @@
  * libframequant: forward pass of a frame-quantized linear layer (FrameQuant, Adepu et al.,
  * ICML 2024, arXiv 2403.06082) on one NVIDIA GB300 GPU (sm_103a).
  *
- * The layer (Sec. 3.2 "Inference Procedure"; Sec. 3, D_l = P_l^T Theta_l P_prev):
+ * The layer (Sec. 3.2, the inference procedure; Sec. 3, D_l = P_l^T Theta_l P_prev):
  *
  *     z = T_in x                          analysis onto the input tight fusion frame
  *     u_i = gamma_i (s_i sum_j q_ij z_j + zero_i sum_j z_j)
@@ -47,7 +47,8 @@ typedef enum {
   FQ_ERR_WORKSPACE = 4,     /* ws is NULL or smaller than fq_workspace_bytes() */
   FQ_ERR_CUDA = 5,          /* a CUDA runtime or launch error */
   FQ_ERR_TIMEOUT = 6,       /* device: a bounded wait inside a kernel ran out (fq_check) */
-  FQ_ERR_DEVICE_CHECK = 7   /* device: a code value above 3 was seen by fq_pack (fq_check) */
+  FQ_ERR_DEVICE_CHECK = 7   /* device: fq_pack met a code above 3 or a non-finite scale or
+                               zero (fq_check) */
 } fq_status;
 
 /* Arithmetic modes of fq_linear_forward. */
@@ -57,8 +58,10 @@ enum {
   FQ_FP32_DEBUG = 1   /* x, T_in, T_out^T, y, z, u are fp32 throughout (CUDA cores) */
 };
 
-/* Packed 2-bit frame coefficients with their per-row scale and zero ("bias and scale values
- * for each row", Appendix K).  Code q_ij in {0,1,2,3} dequantizes to s_i q_ij + zero_i.
+/* Packed 2-bit frame coefficients with their per-row scale and zero (the paper keeps one scale
+ * and one offset per row next to the 2-bit codes, Appendix K).  Code q_ij in {0,1,2,3}
+ * dequantizes to s_i q_ij + zero_i.  fq_pack fills this descriptor; it is the one unit every
+ * forward entry point takes.
  *
  * Layout of `words` (uint32; written by fq_pack): rows are grouped in tiles of 128 and
  * columns in blocks of 64; n_out and n_in are padded up to those multiples with code 0.  The
@@ -68,30 +71,42 @@ enum {
  *     KB = ceil(n_in/64);
  * inside a word, column c = col%16 occupies bits [2*(c/2) + 16*(c%2), +2): even columns in the
  * low half-word, odd columns in the high half-word, so that one mask of 0x00030003 shifted by
- * 2*(c/2) isolates the adjacent pair (c, c+1).
+ * 2*(c/2) isolates the adjacent pair (c, c+1).  ld_words = 4 * KB is the number of words that
+ * hold one row (spread over its KB column blocks); a row tile spans 128 * ld_words contiguous
+ * words, and the whole buffer ceil(n_out/128) * 128 * ld_words = fq_packed_words(n_out, n_in).
  */
 typedef struct {
-  const uint32_t* words;   /* device, fq_packed_words(n_out, n_in) words */
-  const uint16_t* scale;   /* device, IEEE fp16 bit patterns, n_out entries */
-  const uint16_t* zero;    /* device, IEEE fp16 bit patterns, n_out entries */
-  int32_t n_out;           /* rows of C_hat, = k_out * rho, a multiple of 16 */
-  int32_t n_in;            /* columns of C_hat, = k_in * rho, a multiple of 16 */
+  const uint32_t* words;      /* device, fq_packed_words(n_out, n_in) words, 16-byte aligned */
+  const uint16_t* scale_f16;  /* device, IEEE fp16 bit patterns, n_out entries, 16-byte aligned */
+  const uint16_t* zero_f16;   /* device, IEEE fp16 bit patterns, n_out entries, 16-byte aligned */
+  int32_t n_out;              /* rows of C_hat, = k_out * rho, a multiple of 16 */
+  int32_t n_in;               /* columns of C_hat, = k_in * rho, a multiple of 16 */
+  int32_t ld_words;           /* words per row of codes, 4 * ceil(n_in / 64) */
+  int32_t bits;               /* bits per code; 2 is the only width this library runs */
 } fq_packed;
 
 /* Number of uint32 words of the packed layout above: ceil(n_out/128)*128 * ceil(n_in/64)*64 / 16.
  * Returns 0 when n_out or n_in is not positive. */
 size_t fq_packed_words(int n_out, int n_in);
 
-/* Pack 2-bit codes (Algorithm 1, step 5 "store D_hat"; layout above).
- *   codes   device uint8, n_out x n_in row-major, values 0..3 (any alignment)
- *   words   device uint32 output, fq_packed_words(n_out, n_in) words, 16-byte aligned;
- *           padding positions are written with code 0
- *   status  device int32 or NULL: when a code above 3 is met, bit (1 << FQ_ERR_DEVICE_CHECK)
- *           is set there (the code's low 2 bits are packed); fq_pack never clears it
- * Errors: FQ_ERR_INVALID_ARG (null codes/words, n_out or n_in <= 0), FQ_ERR_ALIGNMENT,
- *         FQ_ERR_CUDA. */
-fq_status fq_pack(const uint8_t* codes, int n_out, int n_in, uint32_t* words, int32_t* status,
-                  fq_stream_t stream);
+/* Pack 2-bit codes with their per-row scale and zero into one descriptor (Algorithm 1, step 5,
+ * which stores the quantized D_hat; layout above).
+ *   codes      device uint8, n_out x n_in row-major, values 0..3 (any alignment)
+ *   scale_f16  device fp16 bit patterns [n_out], 16-byte aligned: the step s_i of row i
+ *   zero_f16   device fp16 bit patterns [n_out], 16-byte aligned: the offset zero_i of row i
+ *   out        host descriptor.  On input out->words must point to a writable device buffer of
+ *              fq_packed_words(n_out, n_in) uint32 words, 16-byte aligned (caller-owned); fq_pack
+ *              writes the packed codes there (padding positions with code 0) and sets every
+ *              other field: scale_f16 and zero_f16 point at the caller's arrays (not copied, so
+ *              they must outlive the descriptor's use), n_out, n_in, ld_words and bits = 2.
+ *   status     device int32 or NULL: bit (1 << FQ_ERR_DEVICE_CHECK) is set there when a code
+ *              above 3 is met (its low 2 bits are packed) or a scale or zero is not finite;
+ *              fq_pack never clears it.  Read it with fq_check.
+ * Any positive n_out and n_in can be packed; the forward entry points take multiples of 16.
+ * Errors (nothing is launched and *out is left unchanged): FQ_ERR_INVALID_ARG (null codes,
+ * scale, zero, out or out->words; n_out or n_in <= 0), FQ_ERR_ALIGNMENT, FQ_ERR_CUDA. */
+fq_status fq_pack(const uint8_t* codes, const uint16_t* scale_f16, const uint16_t* zero_f16,
+                  int n_out, int n_in, fq_packed* out, int32_t* status, fq_stream_t stream);
 
 /* Bytes of workspace fq_linear_forward needs for these sizes and mode (independent of the
  * device).  Returns 0 for invalid sizes. */
@@ -102,7 +117,10 @@ size_t fq_workspace_bytes(int M, int d_in, int n_in, int n_out, int d_out, int m
  *   T_in     device, n_in x d_in analysis operator of the input frame (P_prev^T)
  *   C        host pointer to a descriptor of device data (codes, scale, zero); C->n_in and
  *            C->n_out give the frame sizes
- *   T_out_t  device, d_out x n_out synthesis operator of the output frame (T_out^T = P_l)
+ *   T_out_t  device, d_out x n_out synthesis operator of the output frame (T_out^T = P_l),
+ *            i.e. the output frame's analysis operator T_out (n_out x d_out) transposed, so that
+ *            the synthesis contracts over the contiguous dimension of both of its operands, as
+ *            the analysis and the code product do
  *   gamma    device fp32 [n_out] de-noising gain, or NULL for none
  *   y        device, M x d_out output (bf16 or fp32 by mode)
  *   ws       device workspace of at least fq_workspace_bytes(M, d_in, n_in, n_out, d_out,
@@ -115,10 +133,12 @@ size_t fq_workspace_bytes(int M, int d_in, int n_in, int n_out, int d_out, int m
  *            bytes are the device status word, which each call clears before reporting.
  *   mode     FQ_BF16 or FQ_FP32_DEBUG
  * Requirements: M, d_in, d_out >= 1; d_in and d_out multiples of 8; C->n_in and C->n_out
- * positive multiples of 16; all device pointers 16-byte aligned.
- * Errors: FQ_ERR_INVALID_ARG, FQ_ERR_ALIGNMENT, FQ_ERR_WORKSPACE, FQ_ERR_UNSUPPORTED (the
- * current device is not compute capability 10.3 in FQ_BF16 mode, or M <= 64 in FQ_BF16 mode
- * with n_in, n_out or d_out above 81920 = 640 tiles of 128 rows), FQ_ERR_CUDA. */
+ * positive multiples of 16, C->ld_words = 4 * ceil(C->n_in / 64) and C->bits = 2 (as fq_pack
+ * sets them); all device pointers 16-byte aligned.
+ * Errors: FQ_ERR_INVALID_ARG (also an ld_words that does not match n_in), FQ_ERR_ALIGNMENT,
+ * FQ_ERR_WORKSPACE, FQ_ERR_UNSUPPORTED (C->bits other than 2; the current device is not
+ * compute capability 10.3 in FQ_BF16 mode; M <= 64 in FQ_BF16 mode with n_in, n_out or d_out
+ * above 81920 = 640 tiles of 128 rows), FQ_ERR_CUDA. */
 fq_status fq_linear_forward(const void* x, int M, int d_in, const void* T_in,
                             const fq_packed* C, const void* T_out_t, int d_out,
                             const float* gamma, void* y, void* ws, size_t ws_bytes, int mode,

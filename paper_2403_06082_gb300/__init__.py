@@ -14,7 +14,7 @@ import os
 from dataclasses import dataclass
 
 __all__ = [
-    "FQ_BF16", "FQ_FP32_DEBUG", "FrameQuantError", "Packed", "lib", "lib_path",
+    "FQ_BF16", "FQ_FP32_DEBUG", "FrameQuantError", "Packed", "ld_words", "lib", "lib_path",
     "fq_packed_words", "fq_pack", "fq_workspace_bytes", "fq_linear_forward",
     "fq_linear_forward_sms", "fq_linear_forward_ex", "fq_check",
     "fq_status_str", "EXPORTED", "fq_frame_workspace_bytes", "fq_frame_build",
@@ -54,8 +54,9 @@ class FrameQuantError(RuntimeError):
 
 
 class _Packed(ctypes.Structure):
-    _fields_ = [("words", ctypes.c_void_p), ("scale", ctypes.c_void_p),
-                ("zero", ctypes.c_void_p), ("n_out", ctypes.c_int32), ("n_in", ctypes.c_int32)]
+    _fields_ = [("words", ctypes.c_void_p), ("scale_f16", ctypes.c_void_p),
+                ("zero_f16", ctypes.c_void_p), ("n_out", ctypes.c_int32), ("n_in", ctypes.c_int32),
+                ("ld_words", ctypes.c_int32), ("bits", ctypes.c_int32)]
 
 
 class _Rotation(ctypes.Structure):
@@ -92,8 +93,9 @@ def lib() -> ctypes.CDLL:
         L.fq_packed_words.restype = ctypes.c_size_t
         L.fq_packed_words.argtypes = [ctypes.c_int, ctypes.c_int]
         L.fq_pack.restype = ctypes.c_int
-        L.fq_pack.argtypes = [ctypes.c_void_p, ctypes.c_int, ctypes.c_int, ctypes.c_void_p,
-                              ctypes.c_void_p, ctypes.c_void_p]
+        L.fq_pack.argtypes = [ctypes.c_void_p, ctypes.c_void_p, ctypes.c_void_p, ctypes.c_int,
+                              ctypes.c_int, ctypes.POINTER(_Packed), ctypes.c_void_p,
+                              ctypes.c_void_p]
         L.fq_workspace_bytes.restype = ctypes.c_size_t
         L.fq_workspace_bytes.argtypes = [ctypes.c_int] * 6
         L.fq_linear_forward.restype = ctypes.c_int
@@ -189,27 +191,46 @@ def _ok(st: int, where: str) -> None:
         raise FrameQuantError(st, where)
 
 
+def ld_words(n_in: int) -> int:
+    """Words per row of the packed layout, 4 * ceil(n_in / 64) (include/framequant.h)."""
+    return 4 * (-(-n_in // 64))
+
+
 @dataclass
 class Packed:
-    """Device tensors of packed codes (int32 view of the uint32 words), fp16 scale and zero."""
+    """The packed descriptor of include/framequant.h: device tensors of packed codes (int32 view
+    of the uint32 words), fp16 scale and zero (int16 views of the bit patterns), the sizes, the
+    row pitch in words and the code width.  fq_pack returns one."""
     words: object
     scale: object
     zero: object
     n_out: int
     n_in: int
+    ld_words: int | None = None
+    bits: int = 2
+
+    def __post_init__(self):
+        if self.ld_words is None:
+            self.ld_words = ld_words(self.n_in)
 
     def _c(self) -> _Packed:
         return _Packed(_ptr(self.words), _ptr(self.scale), _ptr(self.zero), self.n_out,
-                       self.n_in)
+                       self.n_in, self.ld_words, self.bits)
 
 
 def fq_packed_words(n_out: int, n_in: int) -> int:
     return lib().fq_packed_words(n_out, n_in)
 
 
-def fq_pack(codes, n_out: int, n_in: int, words, status=None, stream=None) -> None:
-    _ok(lib().fq_pack(_ptr(codes), n_out, n_in, _ptr(words), _ptr(status), _stream(stream)),
-        "fq_pack")
+def fq_pack(codes, scale, zero, n_out: int, n_in: int, words, status=None,
+            stream=None) -> Packed:
+    """Pack uint8 codes (n_out x n_in) into `words` and return the descriptor, which refers to
+    `words`, `scale` and `zero` (fp16 bit patterns, any 16-bit dtype)."""
+    pc = _Packed()
+    pc.words = _ptr(words)
+    _ok(lib().fq_pack(_ptr(codes), _ptr(scale), _ptr(zero), n_out, n_in, ctypes.byref(pc),
+                      _ptr(status), _stream(stream)), "fq_pack")
+    return Packed(words, scale, zero, pc.n_out, pc.n_in, pc.ld_words, pc.bits)
 
 
 def fq_workspace_bytes(M: int, d_in: int, n_in: int, n_out: int, d_out: int,

@@ -24,6 +24,21 @@ int current_cc() {
 
 }  // namespace
 
+namespace fq {
+
+fq_status check_packed(const fq_packed* C) {
+  if (!C || !C->words || !C->scale_f16 || !C->zero_f16) return FQ_ERR_INVALID_ARG;
+  if (C->n_in <= 0 || C->n_out <= 0) return FQ_ERR_INVALID_ARG;
+  if (C->n_in % 16 || C->n_out % 16) return FQ_ERR_ALIGNMENT;
+  if (C->ld_words != 4 * ceil_div(C->n_in, kColBlock)) return FQ_ERR_INVALID_ARG;
+  if (C->bits != 2) return FQ_ERR_UNSUPPORTED;
+  if (!aligned16(C->words) || !aligned16(C->scale_f16) || !aligned16(C->zero_f16))
+    return FQ_ERR_ALIGNMENT;
+  return FQ_OK;
+}
+
+}  // namespace fq
+
 extern "C" {
 
 size_t fq_packed_words(int n_out, int n_in) {
@@ -31,12 +46,24 @@ size_t fq_packed_words(int n_out, int n_in) {
   return static_cast<size_t>(round_up(n_out, kRowTile)) * round_up(n_in, kColBlock) / 16;
 }
 
-fq_status fq_pack(const uint8_t* codes, int n_out, int n_in, uint32_t* words, int32_t* status,
-                  fq_stream_t stream) {
-  if (!codes || !words || n_out <= 0 || n_in <= 0) return FQ_ERR_INVALID_ARG;
-  if (!aligned16(words)) return FQ_ERR_ALIGNMENT;
-  return cuda_status(launch_pack(codes, n_out, n_in, words, status,
-                                 reinterpret_cast<cudaStream_t>(stream)));
+fq_status fq_pack(const uint8_t* codes, const uint16_t* scale_f16, const uint16_t* zero_f16,
+                  int n_out, int n_in, fq_packed* out, int32_t* status, fq_stream_t stream) {
+  if (!codes || !scale_f16 || !zero_f16 || !out || !out->words || n_out <= 0 || n_in <= 0)
+    return FQ_ERR_INVALID_ARG;
+  if (!aligned16(out->words) || !aligned16(scale_f16) || !aligned16(zero_f16))
+    return FQ_ERR_ALIGNMENT;
+  // the caller's buffer, writable by contract (the descriptor's view of it is const)
+  uint32_t* words = const_cast<uint32_t*>(out->words);
+  const cudaError_t e = launch_pack(codes, scale_f16, zero_f16, n_out, n_in, words, status,
+                                    reinterpret_cast<cudaStream_t>(stream));
+  if (e != cudaSuccess) return FQ_ERR_CUDA;
+  out->scale_f16 = scale_f16;
+  out->zero_f16 = zero_f16;
+  out->n_out = n_out;
+  out->n_in = n_in;
+  out->ld_words = static_cast<int32_t>(4 * ceil_div(n_in, kColBlock));
+  out->bits = 2;
+  return FQ_OK;
 }
 
 size_t fq_workspace_bytes(int M, int d_in, int n_in, int n_out, int d_out, int mode) {
@@ -58,13 +85,11 @@ fq_status fq_linear_forward_ex(const void* x, int M, int d_in, const void* T_in,
   if (max_sms < 0 || (pf_bytes > 0 && !pf)) return FQ_ERR_INVALID_ARG;
   if (pf_bytes > 0 && !aligned16(pf)) return FQ_ERR_ALIGNMENT;
   if (!x || !T_in || !C || !T_out_t || !y) return FQ_ERR_INVALID_ARG;
-  if (!C->words || !C->scale || !C->zero) return FQ_ERR_INVALID_ARG;
   if (mode != FQ_BF16 && mode != FQ_FP32_DEBUG) return FQ_ERR_INVALID_ARG;
-  if (M <= 0 || d_in <= 0 || d_out <= 0 || C->n_in <= 0 || C->n_out <= 0)
-    return FQ_ERR_INVALID_ARG;
-  if (C->n_in % 16 || C->n_out % 16 || d_in % 8 || d_out % 8) return FQ_ERR_ALIGNMENT;
+  if (M <= 0 || d_in <= 0 || d_out <= 0) return FQ_ERR_INVALID_ARG;
+  if (const fq_status cs = check_packed(C)) return cs;
+  if (d_in % 8 || d_out % 8) return FQ_ERR_ALIGNMENT;
   if (!aligned16(x) || !aligned16(T_in) || !aligned16(T_out_t) || !aligned16(y) ||
-      !aligned16(C->words) || !aligned16(C->scale) || !aligned16(C->zero) ||
       (gamma && !aligned16(gamma)))
     return FQ_ERR_ALIGNMENT;
   if (!ws) return FQ_ERR_WORKSPACE;

@@ -93,8 +93,8 @@ cudaError_t launch_debug_forward(const float* x, int M, int d_in, const float* T
       T_in, nullptr, 0, n_in, d_in, x, M, z, nullptr, nullptr, nullptr);
   // frame-coefficient product with dequantization and optional gain
   rowdot_kernel<true><<<dim3(static_cast<unsigned>(ceil_div(n_out, kWarps)), gy), block, 0, s>>>(
-      nullptr, C.words, KB, n_out, n_in, z, M, u, reinterpret_cast<const __half*>(C.scale),
-      reinterpret_cast<const __half*>(C.zero), gamma);
+      nullptr, C.words, KB, n_out, n_in, z, M, u, reinterpret_cast<const __half*>(C.scale_f16),
+      reinterpret_cast<const __half*>(C.zero_f16), gamma);
   // synthesis: y = T_out^T u
   rowdot_kernel<false><<<dim3(static_cast<unsigned>(ceil_div(d_out, kWarps)), gy), block, 0, s>>>(
       T_out_t, nullptr, 0, d_out, n_out, u, M, y, nullptr, nullptr, nullptr);

@@ -1083,8 +1083,8 @@ fq_status launch_decode(const void* x, int M, int d_in, const void* T_in, const 
     a.ph[p].flags = reinterpret_cast<uint32_t*>(ws + kWsFlags) + p * kWsMaxTiles * kWsSlices;
   }
   a.words = Cq.words;
-  a.scale = reinterpret_cast<const __half*>(Cq.scale);
-  a.zero = reinterpret_cast<const __half*>(Cq.zero);
+  a.scale = reinterpret_cast<const __half*>(Cq.scale_f16);
+  a.zero = reinterpret_cast<const __half*>(Cq.zero_f16);
   a.gamma = gamma;
   a.status = reinterpret_cast<int32_t*>(ws);
   a.gen = reinterpret_cast<uint32_t*>(ws + kWsGen);

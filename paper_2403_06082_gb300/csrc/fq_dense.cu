@@ -71,14 +71,11 @@ size_t fq_reconstruct_workspace_bytes(int d_in, int n_in, int n_out, int d_out) 
 fq_status fq_reconstruct_weight(const void* T_in, const fq_packed* C, const void* T_out_t,
                                 int d_in, int d_out, const float* gamma, void* W_hat, void* ws,
                                 size_t ws_bytes, fq_stream_t stream) {
-  if (!T_in || !C || !T_out_t || !W_hat || d_in <= 0 || d_out <= 0 || C->n_in <= 0 ||
-      C->n_out <= 0)
-    return FQ_ERR_INVALID_ARG;
-  if (!C->words || !C->scale || !C->zero) return FQ_ERR_INVALID_ARG;
+  if (!T_in || !C || !T_out_t || !W_hat || d_in <= 0 || d_out <= 0) return FQ_ERR_INVALID_ARG;
   // the checks of the forward this call makes, before anything is launched
-  if (d_in % 8 || d_out % 8 || C->n_in % 16 || C->n_out % 16 || !aligned16(W_hat) ||
-      !aligned16(T_in) || !aligned16(T_out_t) || !aligned16(C->words) || !aligned16(C->scale) ||
-      !aligned16(C->zero) || (gamma && !aligned16(gamma)))
+  if (const fq_status cs = check_packed(C)) return cs;
+  if (d_in % 8 || d_out % 8 || !aligned16(W_hat) || !aligned16(T_in) || !aligned16(T_out_t) ||
+      (gamma && !aligned16(gamma)))
     return FQ_ERR_ALIGNMENT;
   if (!ws) return FQ_ERR_WORKSPACE;
   if ((reinterpret_cast<uintptr_t>(ws) & 255u) != 0) return FQ_ERR_ALIGNMENT;

@@ -519,15 +519,14 @@ fq_status fq_linear_forward_implicit(const void* x, int M, const fq_frame* F_in,
                                      const fq_packed* C, const fq_frame* F_out,
                                      const float* gamma, void* y, void* ws, size_t ws_bytes,
                                      int max_sms, fq_stream_t stream) {
-  if (!x || !y || !C || !C->words || !C->scale || !C->zero || max_sms < 0 || M <= 0)
-    return FQ_ERR_INVALID_ARG;
+  if (!x || !y || !C || max_sms < 0 || M <= 0) return FQ_ERR_INVALID_ARG;
+  if (const fq_status cs = check_packed(C)) return cs;
   if (!valid_frame(F_in) || !valid_frame(F_out)) return FQ_ERR_INVALID_ARG;
   const fq_frame fi = *F_in, fo = *F_out;
   const int n_in = fi.k * fi.rho, n_out = fo.k * fo.rho;
   if (C->n_in != n_in || C->n_out != n_out) return FQ_ERR_INVALID_ARG;
   if (n_in % 16 || n_out % 16 || fi.d % 8 || fo.d % 8) return FQ_ERR_ALIGNMENT;
-  if (!aligned16(x) || !aligned16(y) || !aligned16(C->words) || !aligned16(C->scale) ||
-      !aligned16(C->zero) || (gamma && !aligned16(gamma)) || !aligned16(fi.roots) ||
+  if (!aligned16(x) || !aligned16(y) || (gamma && !aligned16(gamma)) || !aligned16(fi.roots) ||
       !aligned16(fo.roots))
     return FQ_ERR_ALIGNMENT;
   if (!ws) return FQ_ERR_WORKSPACE;

@@ -35,10 +35,14 @@ constexpr int kDecodeMaxM = 64;   // batches up to this size take the fused deco
 }  // namespace fq
 extern "C" size_t fq_packed_words(int n_out, int n_in);
 namespace fq {
+// The checks every entry point makes on a packed descriptor: pointers set and 16-byte aligned,
+// n_in and n_out positive multiples of 16, ld_words = 4 ceil(n_in / 64) (FQ_ERR_INVALID_ARG /
+// FQ_ERR_ALIGNMENT), bits = 2 (FQ_ERR_UNSUPPORTED).
+fq_status check_packed(const fq_packed* C);
 
 // ---- fq_pack.cu
-cudaError_t launch_pack(const uint8_t* codes, int n_out, int n_in, uint32_t* words,
-                        int32_t* status, cudaStream_t s);
+cudaError_t launch_pack(const uint8_t* codes, const uint16_t* scale, const uint16_t* zero,
+                        int n_out, int n_in, uint32_t* words, int32_t* status, cudaStream_t s);
 
 // ---- fq_debug.cu: fp32 path
 size_t debug_workspace_bytes(int M, int n_in, int n_out);

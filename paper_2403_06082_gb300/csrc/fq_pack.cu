@@ -1,4 +1,5 @@
-// fq_pack: 2-bit codes (uint8, row-major) -> the tiled packed layout of framequant.h.
+// fq_pack: 2-bit codes (uint8, row-major) -> the tiled packed layout of framequant.h, with a
+// check of the per-row scale and zero the descriptor will carry.
 // Memory-bound: one thread writes one 16-byte group of 4 words (64 codes of one row).
 #include "fq_device.cuh"
 #include "fq_internal.h"
@@ -6,7 +7,12 @@
 namespace fq {
 namespace {
 
-__global__ void __launch_bounds__(256) pack_kernel(const uint8_t* __restrict__ codes, int n_out,
+// an fp16 bit pattern with the exponent field all ones is an infinity or a NaN
+__device__ __forceinline__ bool f16_nonfinite(uint16_t h) { return (h & 0x7C00u) == 0x7C00u; }
+
+__global__ void __launch_bounds__(256) pack_kernel(const uint8_t* __restrict__ codes,
+                                                   const uint16_t* __restrict__ scale,
+                                                   const uint16_t* __restrict__ zero, int n_out,
                                                    int n_in, int KB, int64_t groups,
                                                    uint4* __restrict__ out,
                                                    int32_t* __restrict__ status) {
@@ -21,6 +27,8 @@ __global__ void __launch_bounds__(256) pack_kernel(const uint8_t* __restrict__ c
   uint32_t w[4] = {0u, 0u, 0u, 0u};
   bool bad = false;
   if (row < n_out) {
+    // the row's scale and zero, once per row (by its first column block)
+    if (kb == 0) bad |= f16_nonfinite(scale[row]) || f16_nonfinite(zero[row]);
     const uint8_t* src = codes + static_cast<int64_t>(row) * n_in;
     const int c0 = kb * kColBlock;
 #pragma unroll
@@ -41,14 +49,14 @@ __global__ void __launch_bounds__(256) pack_kernel(const uint8_t* __restrict__ c
 
 }  // namespace
 
-cudaError_t launch_pack(const uint8_t* codes, int n_out, int n_in, uint32_t* words,
-                        int32_t* status, cudaStream_t s) {
+cudaError_t launch_pack(const uint8_t* codes, const uint16_t* scale, const uint16_t* zero,
+                        int n_out, int n_in, uint32_t* words, int32_t* status, cudaStream_t s) {
   const int KB = static_cast<int>(ceil_div(n_in, kColBlock));
   const int64_t groups = ceil_div(n_out, kRowTile) * kRowTile * KB;
   const int threads = 256;
   const int64_t blocks = ceil_div(groups, threads);
   pack_kernel<<<static_cast<unsigned>(blocks), threads, 0, s>>>(
-      codes, n_out, n_in, KB, groups, reinterpret_cast<uint4*>(words), status);
+      codes, scale, zero, n_out, n_in, KB, groups, reinterpret_cast<uint4*>(words), status);
   return cudaGetLastError();
 }
 

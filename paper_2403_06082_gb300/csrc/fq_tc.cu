@@ -760,8 +760,8 @@ fq_status launch_tc_forward(const void* x, int M, int d_in, const void* T_in,
     a[ph].part = reinterpret_cast<float*>(ws + L.part);
   }
   a[1].words = Cq.words;
-  a[1].scale = reinterpret_cast<const __half*>(Cq.scale);
-  a[1].zero = reinterpret_cast<const __half*>(Cq.zero);
+  a[1].scale = reinterpret_cast<const __half*>(Cq.scale_f16);
+  a[1].zero = reinterpret_cast<const __half*>(Cq.zero_f16);
   a[1].gamma = gamma;
 
   // maps: T_in, x, z, T_out^T, u  (A maps use 128-row boxes, B maps BN-row boxes)

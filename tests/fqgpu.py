@@ -34,9 +34,9 @@ class DeviceLayer:
         self.T_out_t = torch.from_numpy(np.ascontiguousarray(L.T_out.T)).to(DEV, dtype)
         codes = torch.from_numpy(L.codes).to(DEV)
         words = torch.zeros(fq.fq_packed_words(L.n_out, L.n_in), dtype=torch.int32, device=DEV)
-        fq.fq_pack(codes, L.n_out, L.n_in, words)
-        self.C = fq.Packed(words, torch.from_numpy(L.scale.view(np.int16)).to(DEV),
-                           torch.from_numpy(L.zero.view(np.int16)).to(DEV), L.n_out, L.n_in)
+        self.C = fq.fq_pack(codes, torch.from_numpy(L.scale.view(np.int16)).to(DEV),
+                            torch.from_numpy(L.zero.view(np.int16)).to(DEV), L.n_out, L.n_in,
+                            words)
         self.gamma = torch.from_numpy(L.gamma).to(DEV)
 
     def forward(self, X: np.ndarray, use_gamma: bool = False, ws=None):

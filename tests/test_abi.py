@@ -58,7 +58,10 @@ def test_workspace_bytes(L):
     assert b >= 2048 * (4512 + 4512) * 2
 
 
-_P = fq._Packed
+def _P(words, scale, zero, n_out, n_in, ld=None, bits=2):
+    """A packed descriptor as fq_pack fills it (ld_words = 4 ceil(n_in / 64), bits = 2)."""
+    return fq._Packed(words, scale, zero, n_out, n_in, fq.ld_words(n_in) if ld is None else ld,
+                      bits)
 
 
 def _call(L, x=0x1000, M=8, d_in=256, T_in=0x2000, C=None, T_out=0x3000, d_out=256, gamma=None,
@@ -83,8 +86,29 @@ def test_host_validation_without_gpu(L):
     assert _call(L, ws=None) == 4
     assert _call(L, ws_bytes=1024) == 4
     assert _call(L, ws=0x10010) == 2                    # workspace not 256-byte aligned
-    assert L.fq_pack(None, 4, 4, 0x1000, None, None) == 1
-    assert L.fq_pack(0x1000, 4, 4, 0x1004, None, None) == 2
+    assert _call(L, C=_P(0x5000, 0x6000, 0x7000, 288, 288, ld=16)) == 1   # wrong row pitch
+    assert _call(L, C=_P(0x5000, 0x6000, 0x7000, 288, 288, bits=3)) == 3  # only 2-bit codes
+    assert _call(L, C=_P(0x5000, 0x6008, 0x7000, 288, 288)) == 2          # scale misaligned
+
+
+def test_pack_host_validation_without_gpu(L):
+    def pack(codes=0x1000, scale=0x2000, zero=0x3000, n_out=128, n_in=64, words=0x4000,
+             out=True):
+        o = fq._Packed()
+        o.words = words
+        st = L.fq_pack(codes, scale, zero, n_out, n_in, ctypes.byref(o) if out else None, None,
+                       None)
+        return st, o
+    assert pack(codes=None)[0] == 1
+    assert pack(scale=None)[0] == 1
+    assert pack(zero=None)[0] == 1
+    assert pack(words=None)[0] == 1
+    assert pack(out=False)[0] == 1
+    assert pack(n_in=0)[0] == 1
+    assert pack(words=0x4004)[0] == 2
+    assert pack(scale=0x2002)[0] == 2
+    st, o = pack(zero=0x3008)
+    assert st == 2 and o.n_out == 0 and o.bits == 0          # a refused call leaves *out alone
 
 
 def test_valid_bf16_request_needs_sm103(L):

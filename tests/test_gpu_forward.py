@@ -141,7 +141,7 @@ def test_argument_errors_launch_nothing():
     assert call(M=0) == 1
     assert call(mode=3) == 1
     assert call(d_in=L.d_in + 4) == 2
-    bad = fq.Packed(D.C.words, D.C.scale, D.C.zero, L.n_out, L.n_in + 8)
+    bad = fq.Packed(D.C.words, D.C.scale, D.C.zero, L.n_out, L.n_in + 8, D.C.ld_words)
     assert call(C=bad) == 2
     torch.cuda.synchronize()
     assert (y == 7.0).all()                                 # nothing was written

@@ -132,9 +132,8 @@ def test_llama70b_shapes(name, M):
                               (dr_out.a, dr_out.b, dr_out.ga, dr_out.gb, dr_out.perm,
                                dr_out.signs), DEV)
     words = torch.zeros(fq.fq_packed_words(n_out, n_in), dtype=torch.int32, device=DEV)
-    fq.fq_pack(torch.from_numpy(codes).to(DEV), n_out, n_in, words)
-    C = fq.Packed(words, torch.from_numpy(scale.view(np.int16)).to(DEV),
-                  torch.from_numpy(zero.view(np.int16)).to(DEV), n_out, n_in)
+    C = fq.fq_pack(torch.from_numpy(codes).to(DEV), torch.from_numpy(scale.view(np.int16)).to(DEV),
+                   torch.from_numpy(zero.view(np.int16)).to(DEV), n_out, n_in, words)
     got = _run(X, Fi, C, Fo, None, layer.d_out)
     Z = frames.analysis_apply(k_in, RHO, layer.d_in, dr_in, X)
     U = forward.core(Z, codes, scale, zero)

@@ -53,9 +53,8 @@ def run_layer(name, r, M):
     T_out_t = gpu_frame(k_out, layer.d_out, draws_out).t().contiguous()
     torch.cuda.empty_cache()
     words = torch.zeros(fq.fq_packed_words(n_out, n_in), dtype=torch.int32, device=DEV)
-    fq.fq_pack(torch.from_numpy(codes).to(DEV), n_out, n_in, words)
-    C = fq.Packed(words, torch.from_numpy(scale.view(np.int16)).to(DEV),
-                  torch.from_numpy(zero.view(np.int16)).to(DEV), n_out, n_in)
+    C = fq.fq_pack(torch.from_numpy(codes).to(DEV), torch.from_numpy(scale.view(np.int16)).to(DEV),
+                   torch.from_numpy(zero.view(np.int16)).to(DEV), n_out, n_in, words)
     x = torch.from_numpy(X).to(DEV, torch.bfloat16)
     y = torch.empty(M, layer.d_out, dtype=torch.bfloat16, device=DEV)
     nb = fq.fq_workspace_bytes(M, layer.d_in, n_in, n_out, layer.d_out)
