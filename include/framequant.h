@@ -167,6 +167,15 @@ typedef struct {
                                   fq_linear_forward_sms */
   const void* l2_prefetch;     /* device range to bring into L2 while this call runs, or NULL */
   size_t l2_prefetch_bytes;    /* its length; rounded down to a multiple of 16 */
+  int64_t inject_timeout_cycles; /* 0 in normal use.  A test hook for the device-error path:
+                                  when > 0 (FQ_BF16, M <= 64 and max_sms = 1 only, i.e. one
+                                  CTA with no cluster peers) the kernel's first wait for
+                                  another phase's output expects a stamp that no call writes
+                                  and gives up after this many SM clock cycles, so the call
+                                  ends with FQ_ERR_TIMEOUT in the workspace status word (and
+                                  the waiting role, task, stage and detail in the next four
+                                  words) instead of a result, without a fault.  Zero the
+                                  workspace again before its next use. */
 } fq_forward_opts;
 
 /* fq_linear_forward with options (opts NULL: none).  The L2 prefetch is a hint for chaining
@@ -175,8 +184,9 @@ typedef struct {
  * leaves HBM idle; each CTA then prefetches its share of the range when it reaches its first
  * synthesis task.  Other calls ignore it.  Results never depend on it.  This entry point has
  * no counterpart in the paper.
- * Errors: those of fq_linear_forward; FQ_ERR_INVALID_ARG for max_sms < 0 or a NULL range of
- * nonzero length; FQ_ERR_ALIGNMENT for a range start that is not 16-byte aligned. */
+ * Errors: those of fq_linear_forward; FQ_ERR_INVALID_ARG for max_sms < 0, a NULL range of
+ * nonzero length, or inject_timeout_cycles < 0 or set outside its one-CTA decode case;
+ * FQ_ERR_ALIGNMENT for a range start that is not 16-byte aligned. */
 fq_status fq_linear_forward_ex(const void* x, int M, int d_in, const void* T_in,
                                const fq_packed* C, const void* T_out_t, int d_out,
                                const float* gamma, void* y, void* ws, size_t ws_bytes, int mode,
@@ -320,15 +330,23 @@ fq_status fq_linear_forward_implicit(const void* x, int M, const fq_frame* F_in,
  * process exits; this call allocates nothing.
  *   - Requests whose fq_workspace_bytes(M, d_in, C->n_in, C->n_out, d_out, mode) exceeds
  *     FQ_STATIC_SCRATCH_BYTES return FQ_ERR_UNSUPPORTED and launch nothing.
- *   - The first call on a device looks up the array's device address for that device (with
- *     that device current); make that first call before any stream capture.
+ *   - Every call looks up the array's device address for the current device.  The first call
+ *     on a device, and the first after a device reset, loads the library's device code there:
+ *     make it before any stream capture.
  *   - All calls share the array and it keeps the last call's contents: calls whose work may
  *     overlap on the GPU (other streams, other host threads) race on it.
- *   - The device status word is inside the array, so device-side findings are not reported.
+ *   - The device status word is the head of the array: read it with fq_static_check.
  * Other arguments, requirements and errors are those of fq_linear_forward. */
 fq_status fq_linear_forward_static(const void* x, int M, int d_in, const void* T_in,
                                    const fq_packed* C, const void* T_out_t, int d_out,
                                    const float* gamma, void* y, int mode, fq_stream_t stream);
+
+/* Synchronize `stream` and return the device status of the last fq_linear_forward_static call
+ * on the current device (as fq_check does for a workspace).  When it is FQ_ERR_TIMEOUT, the
+ * header of the library's scratch array is also cleared (on `stream`, synchronized before
+ * returning), which a workspace's owner would do by zeroing it, so that later static calls run
+ * again.  Allocates nothing.  Returns FQ_OK, FQ_ERR_TIMEOUT or FQ_ERR_CUDA. */
+fq_status fq_static_check(fq_stream_t stream);
 
 /* Synchronize `stream` and read the device status word at `status_word` (the head of a
  * forward workspace, or the `status` given to fq_pack).  Returns FQ_OK, FQ_ERR_TIMEOUT,

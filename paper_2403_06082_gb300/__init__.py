@@ -22,7 +22,7 @@ __all__ = [
     "fq_linear_forward_static", "FQ_STATIC_SCRATCH_BYTES", "Frame", "fq_frame_implicit_bytes",
     "fq_frame_implicit", "fq_implicit_workspace_bytes", "fq_linear_forward_implicit",
     "fq_reconstruct_workspace_bytes", "fq_reconstruct_weight", "fq_dense_workspace_bytes",
-    "fq_dense_forward",
+    "fq_dense_forward", "fq_static_check",
 ]
 FQ_STATIC_SCRATCH_BYTES = 16 << 20
 
@@ -38,7 +38,7 @@ EXPORTED = ("fq_packed_words", "fq_pack", "fq_workspace_bytes", "fq_linear_forwa
             "fq_linear_forward_static", "fq_frame_implicit_bytes", "fq_frame_implicit",
             "fq_implicit_workspace_bytes", "fq_linear_forward_implicit",
             "fq_reconstruct_workspace_bytes", "fq_reconstruct_weight", "fq_dense_workspace_bytes",
-            "fq_dense_forward")
+            "fq_dense_forward", "fq_static_check")
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
 
@@ -67,7 +67,7 @@ class _Rotation(ctypes.Structure):
 
 class _Opts(ctypes.Structure):
     _fields_ = [("max_sms", ctypes.c_int32), ("l2_prefetch", ctypes.c_void_p),
-                ("l2_prefetch_bytes", ctypes.c_size_t)]
+                ("l2_prefetch_bytes", ctypes.c_size_t), ("inject_timeout_cycles", ctypes.c_int64)]
 
 
 class _Frame(ctypes.Structure):
@@ -137,6 +137,8 @@ def lib() -> ctypes.CDLL:
             ctypes.c_void_p, ctypes.c_int, ctypes.c_int, ctypes.c_void_p,
             ctypes.POINTER(_Packed), ctypes.c_void_p, ctypes.c_int, ctypes.c_void_p,
             ctypes.c_void_p, ctypes.c_int, ctypes.c_void_p]
+        L.fq_static_check.restype = ctypes.c_int
+        L.fq_static_check.argtypes = [ctypes.c_void_p]
         L.fq_frame_implicit_bytes.restype = ctypes.c_size_t
         L.fq_frame_implicit_bytes.argtypes = [ctypes.c_int] * 5
         L.fq_frame_implicit.restype = ctypes.c_int
@@ -260,12 +262,13 @@ def fq_linear_forward_sms(x, M: int, d_in: int, T_in, C: Packed, T_out_t, d_out:
 
 def fq_linear_forward_ex(x, M: int, d_in: int, T_in, C: Packed, T_out_t, d_out: int, gamma, y,
                          ws, ws_bytes: int, mode: int = FQ_BF16, max_sms: int = 0,
-                         prefetch=None, stream=None) -> None:
-    """fq_linear_forward with options: an SM budget and a device tensor to warm in L2 while
-    the call runs (typically the next layer's T_in; a hint, results do not depend on it)."""
+                         prefetch=None, stream=None, inject_timeout_cycles: int = 0) -> None:
+    """fq_linear_forward with options: an SM budget, a device tensor to warm in L2 while the
+    call runs (typically the next layer's T_in; a hint, results do not depend on it), and the
+    timeout test hook of include/framequant.h (0 in normal use)."""
     pc = C._c()
     nb = 0 if prefetch is None else prefetch.numel() * prefetch.element_size()
-    opts = _Opts(max_sms, _ptr(prefetch), nb)
+    opts = _Opts(max_sms, _ptr(prefetch), nb, inject_timeout_cycles)
     _ok(lib().fq_linear_forward_ex(_ptr(x), M, d_in, _ptr(T_in), ctypes.byref(pc), _ptr(T_out_t),
                                    d_out, _ptr(gamma), _ptr(y), _ptr(ws), ws_bytes, mode,
                                    ctypes.byref(opts), _stream(stream)), "fq_linear_forward_ex")
@@ -279,6 +282,12 @@ def fq_linear_forward_static(x, M: int, d_in: int, T_in, C: Packed, T_out_t, d_o
     _ok(lib().fq_linear_forward_static(_ptr(x), M, d_in, _ptr(T_in), ctypes.byref(pc),
                                        _ptr(T_out_t), d_out, _ptr(gamma), _ptr(y), mode,
                                        _stream(stream)), "fq_linear_forward_static")
+
+
+def fq_static_check(stream=None) -> int:
+    """Synchronize and return the device status of the last fq_linear_forward_static call on
+    the current device; after a timeout it also clears the library scratch array's header."""
+    return lib().fq_static_check(_stream(stream))
 
 
 def fq_check(status_word, stream=None) -> int:

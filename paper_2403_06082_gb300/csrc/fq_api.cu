@@ -82,7 +82,10 @@ fq_status fq_linear_forward_ex(const void* x, int M, int d_in, const void* T_in,
   const int max_sms = opts ? opts->max_sms : 0;
   const void* pf = opts ? opts->l2_prefetch : nullptr;
   const size_t pf_bytes = opts ? (opts->l2_prefetch_bytes & ~static_cast<size_t>(15)) : 0;
-  if (max_sms < 0 || (pf_bytes > 0 && !pf)) return FQ_ERR_INVALID_ARG;
+  const int64_t inject = opts ? opts->inject_timeout_cycles : 0;
+  if (max_sms < 0 || (pf_bytes > 0 && !pf) || inject < 0) return FQ_ERR_INVALID_ARG;
+  if (inject > 0 && (mode != FQ_BF16 || M <= 0 || M > kDecodeMaxM || max_sms != 1))
+    return FQ_ERR_INVALID_ARG;
   if (pf_bytes > 0 && !aligned16(pf)) return FQ_ERR_ALIGNMENT;
   if (!x || !T_in || !C || !T_out_t || !y) return FQ_ERR_INVALID_ARG;
   if (mode != FQ_BF16 && mode != FQ_FP32_DEBUG) return FQ_ERR_INVALID_ARG;
@@ -108,7 +111,8 @@ fq_status fq_linear_forward_ex(const void* x, int M, int d_in, const void* T_in,
   // the status word is cleared by the forward's first kernel, in stream order
   if (M <= kDecodeMaxM)
     return launch_decode_forward(x, M, d_in, T_in, *C, T_out_t, d_out, gamma, y,
-                                 static_cast<char*>(ws), ws_bytes, max_sms, pf, pf_bytes, s);
+                                 static_cast<char*>(ws), ws_bytes, max_sms, pf, pf_bytes, inject,
+                                 s);
   return launch_tc_forward(x, M, d_in, T_in, *C, T_out_t, d_out, gamma, y,
                            static_cast<char*>(ws), ws_bytes, max_sms, s);
 }
@@ -117,7 +121,7 @@ fq_status fq_linear_forward_sms(const void* x, int M, int d_in, const void* T_in
                                 const fq_packed* C, const void* T_out_t, int d_out,
                                 const float* gamma, void* y, void* ws, size_t ws_bytes, int mode,
                                 int max_sms, fq_stream_t stream) {
-  const fq_forward_opts o{max_sms, nullptr, 0};
+  const fq_forward_opts o{max_sms, nullptr, 0, 0};
   return fq_linear_forward_ex(x, M, d_in, T_in, C, T_out_t, d_out, gamma, y, ws, ws_bytes, mode,
                               &o, stream);
 }

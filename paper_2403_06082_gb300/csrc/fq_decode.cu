@@ -116,6 +116,10 @@ struct DecArgs {
   int ext_in;             // bit p: phase p's input was written before the launch (no flags)
   const char* pf_next;    // a range to warm in L2 from the first synthesis task (next layer)
   int64_t pf_next_bytes;  // its length, a multiple of 16 (0: none)
+  // Test hook (0 in normal use): > 0 makes the activation producer's waits for another
+  // phase's slices expect a stamp no call ever writes and give up after this many cycles, so
+  // that the timeout path can be exercised without a fault (one-CTA launches only).
+  int64_t inject_wait;
 };
 
 // Per-cluster task lists, a kernel parameter: cluster c runs task[off[c]] .. task[off[c+1]-1].
@@ -426,8 +430,14 @@ __global__ void __launch_bounds__(DecCfg<BN>::kThreads, 1)
     // the whole warp polls ready flags (one lane per slice); lane 0 issues the loads
     const uint64_t pol_x = policy_evict_last();
     pdl_wait();
-    if (blockIdx.x == 0 && lane == 0) *a.status = 0;      // a new call
+    if (blockIdx.x == 0 && lane == 0) {
+      // a new call: clear the status word and the previous call's timeout details
+      *a.status = 0;
+      for (int w = 4; w < 8; ++w) a.status[w] = 0;
+    }
     const uint32_t g = ld_acquire_gpu(a.gen) + 1;
+    const uint32_t g_want = a.inject_wait > 0 ? g + 0x40000000u : g;
+    const long long wait_limit = a.inject_wait > 0 ? a.inject_wait : kWaitLimitCycles;
     const int rows_per = kBM / S;
     int stage = 0;
     uint32_t phase = 0;
@@ -454,7 +464,7 @@ __global__ void __launch_bounds__(DecCfg<BN>::kThreads, 1)
           // first slice (from `ready`) that is not final yet, over the whole warp
           int first_missing = sl1 + 1;
           for (int gs = ready + lane; gs <= sl1; gs += 32)
-            if (ld_acquire_gpu(&src.flags[(gs / S) * kWsSlices + gs % S]) != g) {
+            if (ld_acquire_gpu(&src.flags[(gs / S) * kWsSlices + gs % S]) != g_want) {
               first_missing = gs;
               break;
             }
@@ -465,7 +475,8 @@ __global__ void __launch_bounds__(DecCfg<BN>::kThreads, 1)
           // K blocks whose rows all lie below the first missing slice
           kb_end = ready > sl1 ? k1 : min(k1, (ready * rows_per) / kBK);
           if (kb_end <= kb) {
-            if (clock64() - t_start > kWaitLimitCycles || *abort_flag) {
+            // lane 0 decides for the warp, so that every lane leaves the loop together
+            if (__shfl_sync(0xffffffffu, clock64() - t_start > wait_limit || *abort_flag, 0)) {
               if (lane == 0 && !*abort_flag) {
                 const uint32_t* f = &src.flags[(ready / S) * kWsSlices + ready % S];
                 note_timeout(a.status, 2, i, ready, static_cast<int>(ld_acquire_gpu(f) - g) * 1000 + t.p);
@@ -1060,7 +1071,7 @@ namespace {
 fq_status launch_decode(const void* x, int M, int d_in, const void* T_in, const fq_packed& Cq,
                         const void* T_out_t, int d_out, const float* gamma, void* y, char* ws,
                         size_t ws_bytes, int max_sms, bool core_only, const void* pf,
-                        size_t pf_bytes, cudaStream_t s) {
+                        size_t pf_bytes, int64_t inject_wait, cudaStream_t s) {
   const int n_in = Cq.n_in, n_out = Cq.n_out;
   const DecWs L = dec_ws(M, n_in, n_out);
   if (ws_bytes < L.total) return FQ_ERR_WORKSPACE;
@@ -1092,6 +1103,7 @@ fq_status launch_decode(const void* x, int M, int d_in, const void* T_in, const 
   a.ext_in = core_only ? 2 : 0;
   a.pf_next = static_cast<const char*>(pf);
   a.pf_next_bytes = pf ? static_cast<int64_t>(pf_bytes) : 0;
+  a.inject_wait = inject_wait;
 
   CUtensorMap m[5];
   if (!tmap_bf16(&m[2], ws + L.z, M, n_in, BN) || !tmap_bf16(&m[4], ws + L.u, M, n_out, BN))
@@ -1105,6 +1117,7 @@ fq_status launch_decode(const void* x, int M, int d_in, const void* T_in, const 
              !tmap_bf16(&m[3], T_out_t, d_out, n_out, kBM)) {
     return FQ_ERR_CUDA;
   }
+  if (inject_wait > 0 && budget != 1) return FQ_ERR_INVALID_ARG;   // one CTA, no cluster peers
   switch (BN) {
     case 16: return run<16>(m, a, R, K, sms, budget, s);
     case 32: return run<32>(m, a, R, K, sms, budget, s);
@@ -1117,15 +1130,16 @@ fq_status launch_decode(const void* x, int M, int d_in, const void* T_in, const 
 fq_status launch_decode_forward(const void* x, int M, int d_in, const void* T_in,
                                 const fq_packed& Cq, const void* T_out_t, int d_out,
                                 const float* gamma, void* y, char* ws, size_t ws_bytes,
-                                int max_sms, const void* pf, size_t pf_bytes, cudaStream_t s) {
+                                int max_sms, const void* pf, size_t pf_bytes,
+                                int64_t inject_wait, cudaStream_t s) {
   return launch_decode(x, M, d_in, T_in, Cq, T_out_t, d_out, gamma, y, ws, ws_bytes, max_sms,
-                       false, pf, pf_bytes, s);
+                       false, pf, pf_bytes, inject_wait, s);
 }
 
 fq_status launch_decode_core(int M, const fq_packed& Cq, const float* gamma, char* ws,
                              size_t ws_bytes, int max_sms, cudaStream_t s) {
   return launch_decode(nullptr, M, 0, nullptr, Cq, nullptr, 0, gamma, nullptr, ws, ws_bytes,
-                       max_sms, true, nullptr, 0, s);
+                       max_sms, true, nullptr, 0, 0, s);
 }
 
 size_t decode_core_z_offset() { return kWsHeader; }

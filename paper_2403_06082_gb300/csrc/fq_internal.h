@@ -19,7 +19,8 @@ inline int64_t round_up(int64_t a, int64_t b) { return ceil_div(a, b) * b; }
 
 // Workspace header (64 KiB, at fixed offsets whatever the layer's sizes, so that one workspace
 // can serve layers of different shapes): [0] device status word, [4] generation counter,
-// [8] end-of-call ticket, [kWsFlags] ready flags, kWsSlices per row tile of up to kWsMaxTiles
+// [8] end-of-call ticket, [16..31] the first timeout's role, task, stage and detail words
+// (cleared by each call), [kWsFlags] ready flags, kWsSlices per row tile of up to kWsMaxTiles
 // row tiles per phase.  A zero-filled header is a valid initial state and every completed call
 // leaves it valid for the next one.
 constexpr size_t kWsHeader = 64 * 1024;
@@ -54,11 +55,13 @@ cudaError_t launch_debug_forward(const float* x, int M, int d_in, const float* T
 size_t decode_workspace_bytes(int M, int d_in, int n_in, int n_out, int d_out);
 // max_sms > 0 caps the SMs a call's kernels occupy (the grid and the plan); pf/pf_bytes is an
 // optional device range (16-byte aligned, multiple of 16 bytes) to warm in L2 during the
-// synthesis when this layer's T_out^T is itself warmed during the code product
+// synthesis when this layer's T_out^T is itself warmed during the code product; inject_wait > 0
+// is the timeout test hook of fq_forward_opts (requires max_sms == 1)
 fq_status launch_decode_forward(const void* x, int M, int d_in, const void* T_in,
                                 const fq_packed& C, const void* T_out_t, int d_out,
                                 const float* gamma, void* y, char* ws, size_t ws_bytes,
-                                int max_sms, const void* pf, size_t pf_bytes, cudaStream_t s);
+                                int max_sms, const void* pf, size_t pf_bytes,
+                                int64_t inject_wait, cudaStream_t s);
 
 // The code product alone (z already in the workspace at decode_core_z_offset(), u left at
 // decode_core_u_offset()), for the structured-frame forward.

@@ -13,11 +13,15 @@
 // entry point accepts; larger requests are refused with FQ_ERR_UNSUPPORTED.  Every call uses
 // the same array and leaves its contents behind for the next call, so calls whose kernels may
 // run at the same time on the GPU (different streams, or different host threads) race on it.
-// The device status word lives in that array too, out of the caller's reach: device-side
-// findings (a bounded wait that ran out) are not reported by this entry point.
+// The device status word lives at the head of that array; fq_static_check reads it and, after
+// a timeout, clears the array's header so that later calls start from a valid state.
+//
+// The array's device address is looked up on every call (cudaGetSymbolAddress, with the
+// caller's device current), never cached: a cached address would outlive a device reset
+// (cudaDeviceReset, or anything else that destroys and re-creates the primary context), after
+// which the module is loaded again and the array may sit elsewhere.  The first call on a device
+// (and the first after a reset) loads the library's device code there.
 #include <cuda_runtime.h>
-
-#include <mutex>
 
 #include "fq_internal.h"
 
@@ -28,25 +32,13 @@ constexpr size_t kStaticScratchBytes = FQ_STATIC_SCRATCH_BYTES;
 
 static __device__ __align__(256) unsigned char g_static_scratch[kStaticScratchBytes];
 
-constexpr int kMaxDevices = 64;
-
-// Device address of g_static_scratch on the current device, looked up once per device (the
-// symbol's host-side name is not a device address and must never be passed to a kernel).
+// Device address of g_static_scratch on the current device.  The symbol's host-side name is a
+// stand-in, not a device address, and must never be passed to a kernel.
 cudaError_t scratch_for_current_device(void** out) {
-  static std::mutex mu;
-  static void* addr[kMaxDevices] = {};
-  int dev = 0;
-  cudaError_t e = cudaGetDevice(&dev);
+  void* p = nullptr;
+  const cudaError_t e = cudaGetSymbolAddress(&p, g_static_scratch);
   if (e != cudaSuccess) return e;
-  if (dev < 0 || dev >= kMaxDevices) return cudaErrorInvalidDevice;
-  std::lock_guard<std::mutex> g(mu);
-  if (!addr[dev]) {
-    void* p = nullptr;
-    e = cudaGetSymbolAddress(&p, g_static_scratch);
-    if (e != cudaSuccess) return e;
-    addr[dev] = p;
-  }
-  *out = addr[dev];
+  *out = p;
   return cudaSuccess;
 }
 
@@ -68,4 +60,18 @@ extern "C" fq_status fq_linear_forward_static(const void* x, int M, int d_in, co
   // and the sums of z are written before they are read within one call.
   return fq_linear_forward(x, M, d_in, T_in, C, T_out_t, d_out, gamma, y, scratch,
                            fq::kStaticScratchBytes, mode, stream);
+}
+
+extern "C" fq_status fq_static_check(fq_stream_t stream) {
+  void* scratch = nullptr;
+  if (fq::scratch_for_current_device(&scratch) != cudaSuccess) return FQ_ERR_CUDA;
+  const fq_status st = fq_check(scratch, stream);
+  if (st == FQ_ERR_TIMEOUT) {
+    // the header's flags and counters may be mid-call: a zero-filled header is a valid start
+    auto s = reinterpret_cast<cudaStream_t>(stream);
+    if (cudaMemsetAsync(scratch, 0, fq::kWsHeader, s) != cudaSuccess ||
+        cudaStreamSynchronize(s) != cudaSuccess)
+      return FQ_ERR_CUDA;
+  }
+  return st;
 }

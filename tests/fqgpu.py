@@ -62,3 +62,33 @@ def reference(L, X: np.ndarray, use_gamma: bool = False) -> np.ndarray:
 
 def rel_frobenius(got: np.ndarray, ref: np.ndarray) -> float:
     return float(np.linalg.norm(got - ref) / np.linalg.norm(ref))
+
+
+# Elementwise companions of the whole-output bound, per tolerance: |got - ref| <= a * rms(ref)
+# + r * |ref| for every element.  The whole-output relative Frobenius error is the stated
+# tolerance; on its own it lets one wrong output column through on the widest layers (a zero
+# column of an 11008-wide output adds only sqrt(1/11008) ~ 0.0095).  bf16: rounding z, u and y
+# to bf16 gives an error of ~3e-3 of the rms per element, ~1.5e-2 at the tail of 1e5-1e6
+# elements; a = 0.05 and r = 0.02 leave margin above that and fail any element that is off by
+# more than ~5% of the output's rms (a dropped or misplaced column or row fails at almost every
+# element).  fp32 (debug mode): a = r = 1e-4.
+ELEMENTWISE = {1e-2: (0.05, 0.02), 1e-5: (1e-4, 1e-4)}
+
+
+def assert_parity(got: np.ndarray, ref: np.ndarray, tol: float) -> float:
+    """Relative Frobenius error <= tol, and every element within the companion bound above.
+    Returns the relative Frobenius error."""
+    got = np.asarray(got, dtype=np.float64)
+    ref = np.asarray(ref, dtype=np.float64)
+    assert got.shape == ref.shape, (got.shape, ref.shape)
+    assert np.isfinite(got).all(), "non-finite output"
+    err = rel_frobenius(got, ref)
+    assert err <= tol, f"relative Frobenius error {err:.3e} > {tol:g}"
+    a, r = ELEMENTWISE[tol]
+    bound = a * np.sqrt(np.mean(ref * ref)) + r * np.abs(ref)
+    ratio = np.abs(got - ref) / bound
+    worst = np.unravel_index(int(np.argmax(ratio)), ratio.shape)
+    assert ratio[worst] <= 1.0, (
+        f"element {worst}: got {got[worst]:.6g}, oracle {ref[worst]:.6g}, "
+        f"{ratio[worst]:.2f} x the elementwise bound (Frobenius {err:.3e})")
+    return err

@@ -178,6 +178,10 @@ def test_forward_ex_host_validation_without_gpu(L):
     assert ex(fq._Opts(0, None, 4096)) == 1                # range without a pointer
     assert ex(fq._Opts(0, 0x9008, 4096)) == 2              # range start not 16-byte aligned
     assert ex(fq._Opts(0, 0x9000, 4096), x=None) == 1
+    # the timeout test hook: one-CTA decode launches only, never negative
+    assert ex(fq._Opts(0, None, 0, 100000)) == 1           # needs max_sms = 1
+    assert ex(fq._Opts(1, None, 0, -5)) == 1
+    assert ex(fq._Opts(1, None, 0, 100000), M=100) == 1    # not the M <= 64 kernel
 
 
 def test_rotation_validation_without_gpu(L):

@@ -10,7 +10,7 @@ import pytest
 torch = pytest.importorskip("torch")
 
 import paper_2403_06082_gb300 as fq  # noqa: E402
-from fqgpu import DEV, DeviceLayer, activations, oracle_layer, reference, rel_frobenius  # noqa: E402
+from fqgpu import DEV, DeviceLayer, activations, oracle_layer, reference, assert_parity, rel_frobenius  # noqa: E402
 
 pytestmark = pytest.mark.gpu
 BF16 = torch.bfloat16
@@ -41,8 +41,7 @@ def _group(wl_key, names, M, budget, use_gamma=False, sample=None):
         Xs = X
         if sample is not None:
             got, Xs = got[sample], X[sample]
-        err = rel_frobenius(got, reference(L, Xs, use_gamma))
-        assert err <= 1e-2, (L.name, err)
+        err = assert_parity(got, reference(L, Xs, use_gamma), 1e-2)
 
 
 def test_qkv_decode_side_by_side():
@@ -71,7 +70,7 @@ def test_budget_edges(M, budget):
     fq.fq_linear_forward_sms(x, M, L.d_in, D.T_in, D.C, D.T_out_t, L.d_out, D.gamma, y, ws, nb,
                              budget)
     assert fq.fq_check(ws) == 0
-    assert rel_frobenius(y.double().cpu().numpy(), reference(L, X, True)) <= 1e-2
+    assert_parity(y.double().cpu().numpy(), reference(L, X, True), 1e-2)
 
 
 def test_budget_fp32_debug_and_negative():
@@ -92,7 +91,7 @@ def test_budget_fp32_debug_and_negative():
     fq.fq_linear_forward_sms(x, M, L.d_in, D.T_in, D.C, D.T_out_t, L.d_out, None, y, ws, nb, 2,
                              mode=fq.FQ_FP32_DEBUG)
     assert fq.fq_check(ws) == 0
-    assert rel_frobenius(y.double().cpu().numpy(), reference(L, X, False)) <= 1e-5
+    assert_parity(y.double().cpu().numpy(), reference(L, X, False), 1e-5)
     assert np.isfinite(y.cpu().numpy()).all()
 
 
@@ -112,4 +111,4 @@ def test_l2_prefetch_hint_changes_nothing():
         assert fq.fq_check(ws) == 0
         outs.append(y.cpu())
     assert torch.equal(outs[0], outs[1]) and torch.equal(outs[0], outs[2])
-    assert rel_frobenius(outs[0].double().numpy(), reference(Lq, X, False)) <= 1e-2
+    assert_parity(outs[0].double().numpy(), reference(Lq, X, False), 1e-2)

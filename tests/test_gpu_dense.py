@@ -7,7 +7,7 @@ import pytest
 torch = pytest.importorskip("torch")
 
 import paper_2403_06082_gb300 as fq  # noqa: E402
-from fqgpu import DEV, DeviceLayer, activations, oracle_layer, reference, rel_frobenius  # noqa: E402
+from fqgpu import DEV, DeviceLayer, activations, oracle_layer, reference, assert_parity, rel_frobenius  # noqa: E402
 from oracle import quant  # noqa: E402
 
 pytestmark = pytest.mark.gpu
@@ -38,8 +38,7 @@ def _oracle_w_hat(L, use_gamma):
 def test_reconstructed_weight(wl_key, name, use_gamma):
     L = oracle_layer(wl_key, name)
     W = _w_hat(L, DeviceLayer(L, BF16), use_gamma)
-    err = rel_frobenius(W.double().cpu().numpy(), _oracle_w_hat(L, use_gamma))
-    assert err <= 1e-2, err
+    err = assert_parity(W.double().cpu().numpy(), _oracle_w_hat(L, use_gamma), 1e-2)
 
 
 @pytest.mark.parametrize("M", [1, 8, 100, 300])
@@ -54,8 +53,7 @@ def test_dense_forward_matches_the_layer(M):
     ws = torch.zeros(nb, dtype=torch.uint8, device=DEV)
     fq.fq_dense_forward(x, M, L.d_in, W, L.d_out, y, ws, nb)
     assert fq.fq_check(ws) == 0
-    err = rel_frobenius(y.double().cpu().numpy(), reference(L, X, True))
-    assert err <= 1e-2, err
+    err = assert_parity(y.double().cpu().numpy(), reference(L, X, True), 1e-2)
 
 
 def test_dense_forward_vit_batch():
@@ -71,8 +69,7 @@ def test_dense_forward_vit_batch():
     fq.fq_dense_forward(x, M, L.d_in, W, L.d_out, y, ws, nb)
     assert fq.fq_check(ws) == 0
     rows = [0, 1, 127, 128, 499, 998, 999]
-    err = rel_frobenius(y.double().cpu().numpy()[rows], reference(L, X[rows], False))
-    assert err <= 1e-2, err
+    err = assert_parity(y.double().cpu().numpy()[rows], reference(L, X[rows], False), 1e-2)
 
 
 def test_errors_launch_nothing():

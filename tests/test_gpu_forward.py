@@ -10,7 +10,7 @@ torch = pytest.importorskip("torch")
 import paper_2403_06082_gb300 as fq  # noqa: E402
 import workloads as wl  # noqa: E402
 from fqgpu import (DEV, DeviceLayer, activations, oracle_layer, reference,  # noqa: E402
-                   rel_frobenius)
+                   rel_frobenius, assert_parity)
 
 pytestmark = pytest.mark.gpu
 BF16, FP32 = torch.bfloat16, torch.float32
@@ -22,8 +22,7 @@ def _check(L, X, dtype, use_gamma, sample=None):
     got = DeviceLayer(L, dtype).forward(X, use_gamma)
     if sample is not None:
         got, X = got[sample], X[sample]
-    err = rel_frobenius(got, reference(L, X, use_gamma))
-    assert err <= TOL[dtype], err
+    err = assert_parity(got, reference(L, X, use_gamma), TOL[dtype])
     return err
 
 
@@ -48,10 +47,30 @@ def test_llama7b_decode_full(name, M):
     _check(L, activations("llama2_7b_decode", name, M), BF16, False)
 
 
-@pytest.mark.parametrize("name", ["q", "down"])
-def test_llama7b_decode_fp32_debug(name):
+@pytest.mark.parametrize("name", ["q", "gate", "down"])
+@pytest.mark.parametrize("M", [1, 16])
+def test_llama7b_decode_fp32_debug(name, M):
     L = oracle_layer("llama2_7b_decode", name)
-    _check(L, activations("llama2_7b_decode", name, 16), FP32, False)
+    _check(L, activations("llama2_7b_decode", name, M), FP32, name == "gate")
+
+
+@pytest.mark.parametrize("name,use_gamma", [("q", True), ("gate", False), ("down", True)])
+def test_llama7b_prefill_fp32_debug_sampled(name, use_gamma):
+    """The prefill configuration (2048 tokens, filter on and off) in FQ_FP32_DEBUG: the whole
+    batch runs on the GPU, the oracle checks a seeded sample of tokens."""
+    L = oracle_layer("llama2_7b_prefill", name)
+    X = activations("llama2_7b_prefill", name, 2048)
+    sample = np.sort(wl.rng(3, "sample-fp32", name).choice(2048, 32, replace=False))
+    _check(L, X, FP32, use_gamma, sample)
+
+
+@pytest.mark.parametrize("name", ["fc1", "fc2"])
+def test_vit_mlp_fp32_debug_sampled(name):
+    """The ViT-B/16 MLP pair at its full 12608-token batch in FQ_FP32_DEBUG, sampled tokens."""
+    L = oracle_layer("vit_b16_mlp", name)
+    X = activations("vit_b16_mlp", name, 12608)
+    sample = np.sort(wl.rng(1, "sample-fp32", name).choice(12608, 48, replace=False))
+    _check(L, X, FP32, name == "fc2", sample)
 
 
 @pytest.mark.parametrize("name,use_gamma", [("q", False), ("q", True), ("up", True)])
@@ -114,8 +133,8 @@ def test_workspace_reuse_across_shapes_and_determinism():
     yb2 = Db.forward(Xb, False, ws=ws)
     np.testing.assert_array_equal(ya1, ya2)       # fixed-order reductions: bitwise repeatable
     np.testing.assert_array_equal(yb1, yb2)
-    assert rel_frobenius(ya1, reference(La, Xa, True)) <= 1e-2
-    assert rel_frobenius(yb1, reference(Lb, Xb, False)) <= 1e-2
+    assert_parity(ya1, reference(La, Xa, True), 1e-2)
+    assert_parity(yb1, reference(Lb, Xb, False), 1e-2)
 
 
 def test_argument_errors_launch_nothing():
@@ -165,7 +184,7 @@ def test_stream_argument():
         fq.fq_linear_forward(x, 16, L.d_in, D.T_in, D.C, D.T_out_t, L.d_out, D.gamma, y, ws, nb,
                              0, stream=s)
     assert fq.fq_check(ws, stream=s) == 0
-    assert rel_frobenius(y.double().cpu().numpy(), reference(L, X, True)) <= 1e-2
+    assert_parity(y.double().cpu().numpy(), reference(L, X, True), 1e-2)
 
 
 @pytest.mark.parametrize("name,M,use_gamma", [
@@ -180,7 +199,7 @@ def test_split_k_tensor_core_path(name, M, use_gamma):
     X = activations("llama2_7b_decode", name, M)
     D = DeviceLayer(L, BF16)
     got = D.forward(X, use_gamma)
-    assert rel_frobenius(got, reference(L, X, use_gamma)) <= TOL[BF16]
+    assert_parity(got, reference(L, X, use_gamma), TOL[BF16])
     np.testing.assert_array_equal(got, D.forward(X, use_gamma))
 
 
@@ -198,4 +217,4 @@ def test_split_k_under_sm_budget():
         fq.fq_linear_forward_sms(x, 128, L.d_in, D.T_in, D.C, D.T_out_t, L.d_out, None, y, ws,
                                  nb, budget)
         assert fq.fq_check(ws) == 0
-        assert rel_frobenius(y.double().cpu().numpy(), ref) <= TOL[BF16]
+        assert_parity(y.double().cpu().numpy(), ref, TOL[BF16])

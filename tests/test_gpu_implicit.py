@@ -14,7 +14,7 @@ torch = pytest.importorskip("torch")
 
 import paper_2403_06082_gb300 as fq  # noqa: E402
 import workloads as wl  # noqa: E402
-from fqgpu import DEV, DeviceLayer, activations, oracle_layer, reference, rel_frobenius  # noqa: E402
+from fqgpu import DEV, DeviceLayer, activations, oracle_layer, reference, assert_parity, rel_frobenius  # noqa: E402
 from oracle import forward, frames  # noqa: E402
 
 pytestmark = pytest.mark.gpu
@@ -56,8 +56,7 @@ def _check(wl_key, name, M, use_gamma, rotate=True, tol=1e-2):
     Fi, Fo = _frames(wl_key, name, L, rotate)
     X = activations(wl_key, name, M)
     got = _run(X, Fi, D.C, Fo, D.gamma if use_gamma else None, L.d_out)
-    err = rel_frobenius(got, reference(L, X, use_gamma))
-    assert err <= tol, err
+    err = assert_parity(got, reference(L, X, use_gamma), tol)
     return got
 
 
@@ -90,7 +89,7 @@ def test_matches_dense_path():
     X = activations("llama2_7b_decode", "q", 16)
     dense = D.forward(X)
     got = _run(X, Fi, D.C, Fo, None, L.d_out)
-    assert rel_frobenius(got, dense) <= 1e-2
+    assert_parity(got, dense, 1e-2)
 
 
 def test_workspace_reuse_and_budget():
@@ -109,8 +108,8 @@ def test_workspace_reuse_and_budget():
     Db.forward(Xb, ws=ws)
     ya2 = _run(Xa, Fa[0], Da.C, Fa[1], Da.gamma, La.d_out, ws)
     np.testing.assert_array_equal(ya1, ya2)
-    assert rel_frobenius(ya1, reference(La, Xa, True)) <= 1e-2
-    assert rel_frobenius(yb1, reference(Lb, Xb, False)) <= 1e-2
+    assert_parity(ya1, reference(La, Xa, True), 1e-2)
+    assert_parity(yb1, reference(Lb, Xb, False), 1e-2)
 
 
 @pytest.mark.parametrize("name,M", [("q", 16), ("gate", 1), ("down", 16)])
@@ -138,8 +137,7 @@ def test_llama70b_shapes(name, M):
     Z = frames.analysis_apply(k_in, RHO, layer.d_in, dr_in, X)
     U = forward.core(Z, codes, scale, zero)
     ref = frames.synthesis_apply(k_out, RHO, layer.d_out, dr_out, U)
-    err = rel_frobenius(got, ref)
-    assert err <= 1e-2, err
+    err = assert_parity(got, ref, 1e-2)
 
 
 def test_errors_launch_nothing():

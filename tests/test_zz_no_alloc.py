@@ -9,15 +9,20 @@ import pytest
 torch = pytest.importorskip("torch")
 
 import paper_2403_06082_gb300 as fq  # noqa: E402
-from fqgpu import DEV, DeviceLayer, activations, oracle_layer, rel_frobenius  # noqa: E402
+from fqgpu import DEV, DeviceLayer, activations, oracle_layer, assert_parity, rel_frobenius  # noqa: E402
 
 pytestmark = pytest.mark.gpu
 TOL = {torch.bfloat16: 1e-2, torch.float32: 1e-5}
 
 
-@pytest.mark.parametrize("dtype", [torch.bfloat16, torch.float32], ids=["bf16", "fp32"])
-@pytest.mark.parametrize("M", [16, 40])
+@pytest.mark.parametrize("dtype,M", [(torch.bfloat16, 16), (torch.bfloat16, 40),
+                                     (torch.float32, 16), (torch.float32, 40),
+                                     (torch.bfloat16, 128), (torch.bfloat16, 300)],
+                         ids=["bf16-16", "bf16-40", "fp32-16", "fp32-40", "bf16-128",
+                              "bf16-300"])
 def test_static_matches_workspace_forward_twice(dtype, M):
+    """M <= 64 runs the fused decode kernel through the array, M = 128 and 300 the tensor-core
+    kernels (whose split-K counters must be left zeroed for the next call)."""
     L = oracle_layer("single256", "single")
     D = DeviceLayer(L, dtype)
     mode = fq.FQ_BF16 if dtype == torch.bfloat16 else fq.FQ_FP32_DEBUG
@@ -29,9 +34,10 @@ def test_static_matches_workspace_forward_twice(dtype, M):
         fq.fq_linear_forward_static(x, M, L.d_in, D.T_in, D.C, D.T_out_t, L.d_out, D.gamma, y,
                                     mode)
         torch.cuda.synchronize()
+        assert fq.fq_static_check() == 0
         got = y.double().cpu().numpy()
         assert np.isfinite(got).all()
-        assert rel_frobenius(got, ref) <= TOL[dtype]
+        assert_parity(got, ref, TOL[dtype])
 
 
 def test_static_refuses_sizes_beyond_the_array():
