@@ -35,6 +35,8 @@ METRIC = ("frame-quant linear µs/layer; HBM GB/s (M≤16) & TFLOP/s (M=2048) vs
           "GB300 peak")
 UNIT = "us/layer"
 RHO = 16
+# the launches of one decoder block: independent layers share a launch
+GROUPS = (("q", "k", "v"), ("o",), ("gate", "up"), ("down",))
 FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
 SMI_FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
               "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
@@ -194,8 +196,14 @@ class Regime:
         self.layers = [prepare_layer(fq, wl, torch, self.wk, l, self.r, dev)
                        for l in self.wk.layers]
         self.use_gamma = use_gamma
+        # independent layers of the block, one fq_linear_forward_group launch each (a
+        # transformer's q, k and v read the same input, and so do gate and up)
+        by = {L["name"]: L for L in self.layers}
+        self.groups = [[by[n] for n in names] for names in GROUPS if all(n in by for n in names)]
         ws_bytes = max(fq.fq_workspace_bytes(M, L["d_in"], L["n_in"], L["n_out"], L["d_out"], 0)
                        for L in self.layers)
+        for grp in self.groups:
+            ws_bytes = max(ws_bytes, fq.fq_group_workspace_bytes(M, self.group_layers(grp)))
         self.ws_bytes = ws_bytes
         self.ws = torch.zeros(ws_bytes, dtype=torch.uint8, device=dev)
         # The step's activations and outputs live in one device buffer each (every layer a
@@ -231,6 +239,41 @@ class Regime:
                 raise RuntimeError(f"{L['name']}: {fq.fq_status_str(st)}")
         torch.cuda.synchronize()
 
+    def group_layers(self, grp):
+        fq = self.fq
+        return [fq.Layer(L["x"], L["d_in"], L["T_in"], L["C"], L["T_out_t"], L["d_out"],
+                         L["gamma"] if self.use_gamma else None, L["y"]) for L in grp]
+
+    def forward_group(self, grp, stream, prefetch=None):
+        """One launch for the group's layers (fq_linear_forward_group; a single layer through
+        fq_linear_forward_ex), naming `prefetch` as the L2 hint."""
+        if len(grp) == 1:
+            self.forward(grp[0], stream, prefetch)
+            return
+        self.fq.fq_linear_forward_group(self.M, self.group_layers(grp), self.ws, self.ws_bytes,
+                                        0, prefetch, stream)
+
+    def capture_groups(self, stream, host=False):
+        """One graph: the block as its launches (groups in order), each naming the next
+        launch's first T_in as its L2 prefetch hint; with host=True the step's inputs come
+        from pinned host memory first and its results go back at the end."""
+        torch = self.torch
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, stream=stream):
+            if host:
+                self.x_all.copy_(self.x_host_all, non_blocking=True)
+            self.launch_groups(stream)
+            if host:
+                self.y_host_all.copy_(self.y_all, non_blocking=True)
+        return g
+
+    def launch_groups(self, stream, only=None):
+        n = len(self.groups)
+        for i, grp in enumerate(self.groups):
+            if only is not None and i != only:
+                continue
+            self.forward_group(grp, stream.cuda_stream, self.groups[(i + 1) % n][0]["T_in"])
+
     def forward(self, L, stream, prefetch=None):
         fq = self.fq
         if prefetch is None:
@@ -260,47 +303,6 @@ class Regime:
                 self.y_host_all.copy_(self.y_all, non_blocking=True)
         return g
 
-    def capture_grouped(self, groups, stream):
-        """One graph of all layers with the independent layers of a group side by side: group
-        members run on their own streams and workspaces, each on `budget` SMs
-        (fq_linear_forward_sms); the groups run in order."""
-        torch, fq = self.torch, self.fq
-        by_name = {L["name"]: L for L in self.layers}
-        width = max(len(names) for names, _ in groups)
-        if not hasattr(self, "group_ws"):
-            self.group_ws = [self.ws] + [torch.zeros(self.ws_bytes, dtype=torch.uint8,
-                                                     device=self.dev) for _ in range(width - 1)]
-        side = [torch.cuda.Stream(device=self.dev) for _ in range(width - 1)]
-
-        def launch(names, budget, streams):
-            for name, st, ws in zip(names, streams, self.group_ws):
-                L = by_name[name]
-                fq.fq_linear_forward_sms(L["x"], self.M, L["d_in"], L["T_in"], L["C"],
-                                         L["T_out_t"], L["d_out"],
-                                         L["gamma"] if self.use_gamma else None, L["y"], ws,
-                                         self.ws_bytes, budget, fq.FQ_BF16, st.cuda_stream)
-
-        for names, budget in groups:             # eager calls: plans for each budget, status
-            launch(names, budget, [stream] + side)
-            torch.cuda.synchronize()
-            for ws in self.group_ws[:len(names)]:
-                st = fq.fq_check(ws)
-                if st != 0:
-                    raise RuntimeError(f"group {names}: {fq.fq_status_str(st)}")
-        g = torch.cuda.CUDAGraph()
-        with torch.cuda.graph(g, stream=stream):
-            for names, budget in groups:
-                fork = torch.cuda.Event()
-                fork.record(stream)
-                for st in side[:len(names) - 1]:
-                    st.wait_event(fork)
-                launch(names, budget, [stream] + side)
-                for st in side[:len(names) - 1]:
-                    join = torch.cuda.Event()
-                    join.record(st)
-                    stream.wait_event(join)
-        return g
-
     def host_bytes(self):
         """Bytes one host-backed step copies in and out."""
         return self.x_all.numel() * 2, self.y_all.numel() * 2
@@ -308,6 +310,33 @@ class Regime:
     def bytes_flops(self, L):
         args = (L["d_in"], L["d_out"], L["n_in"], L["n_out"], self.M)
         return layer_bytes(*args), layer_flops(*args)
+
+
+def eager_e2e(torch, dec, stream, steps, warmup):
+    """Total ms of `steps` end-to-end steps issued as plain API calls on `stream`: the H2D
+    copy of the step's inputs from pinned memory, the block's 4 launches (q|k|v and gate|up
+    through fq_linear_forward_group, o and down through fq_linear_forward_ex, each naming the
+    next launch's T_in as its L2 prefetch hint), the D2H copy of the outputs."""
+    def step():
+        dec.x_all.copy_(dec.x_host_all, non_blocking=True)
+        dec.launch_groups(stream)
+        dec.y_host_all.copy_(dec.y_all, non_blocking=True)
+
+    with torch.cuda.stream(stream):
+        for _ in range(warmup):
+            step()
+    torch.cuda.synchronize()
+    start = torch.cuda.Event(enable_timing=True)
+    end = torch.cuda.Event(enable_timing=True)
+    with torch.cuda.stream(stream):
+        start.record(stream)
+        for _ in range(steps):
+            step()
+        end.record(stream)
+    torch.cuda.synchronize()
+    if dec.fq.fq_check(dec.ws) != 0:
+        raise RuntimeError("eager end-to-end step: device status")
+    return start.elapsed_time(end)
 
 
 def timed_replays(torch, graphs, stream, steps, warmup, events_between=False):
@@ -350,6 +379,27 @@ def timed_replays(torch, graphs, stream, steps, warmup, events_between=False):
 
 
 # --------------------------------------------------------------------------- CPU oracle
+def cpu_model():
+    """The host CPU's model name (lscpu, else /proc/cpuinfo), or the machine type."""
+    import platform
+    try:
+        out = subprocess.run(["lscpu"], capture_output=True, text=True, timeout=10).stdout
+        fields = dict(l.split(":", 1) for l in out.splitlines() if ":" in l)
+        name = " ".join(fields.get(k, "").strip() for k in ("Vendor ID", "Model name")).strip()
+        if name:
+            return f"{name} ({platform.machine()})"
+    except (OSError, subprocess.SubprocessError, ValueError):
+        pass
+    try:
+        with open("/proc/cpuinfo") as f:
+            for line in f:
+                if line.lower().startswith(("model name", "cpu part")):
+                    return f"{line.split(':', 1)[1].strip()} ({platform.machine()})"
+    except OSError:
+        pass
+    return platform.machine()
+
+
 def cpu_baseline(seconds=12.0):
     """The fp64 oracle's layer forward on this host's cores, on a bounded sample of the
     decode workload: the q (4096x4096) and down (4096x11008) layer shapes at M = 16, repeated
@@ -387,7 +437,7 @@ def cpu_baseline(seconds=12.0):
     per_layer_us = (4 * tq + 3 * tl) / 7 * 1e6
     n = sum(len(v) for v in times.values())
     return {"value": round(per_layer_us, 1), "unit": UNIT, "cores": os.cpu_count(),
-            "kind": "oracle",
+            "cpu": cpu_model(), "kind": "oracle",
             "sample": (f"fp64 numpy oracle forward, M=16, {n} layer calls over "
                        f"{seconds:.0f}+ s: q-shape median {tq * 1e3:.1f} ms, "
                        f"down-shape median {tl * 1e3:.1f} ms, weighted 4:3 as in the block; "
@@ -448,7 +498,7 @@ def reference_arm(args, rank):
         "vs_baseline": None, "dtype": "f64", "data": "synthetic",
         "config": {"workload": "llama2_7b_block_decode", "M": 16, "r": "1.1", "rho": RHO},
         "cpu_baseline": {"value": round(us, 1), "unit": UNIT, "cores": os.cpu_count(),
-                         "kind": "oracle", "sample": sample},
+                         "cpu": cpu_model(), "kind": "oracle", "sample": sample},
         "e2e": {"value": round(us, 1), "unit": UNIT, "h2d_bytes_per_step": 0,
                 "d2h_bytes_per_step": 0},
     }), flush=True)
@@ -474,13 +524,16 @@ def measure_prefill(args, fq, wl, torch, dev, rank, world, dist, stream, peaks):
         "M": 2048, "gamma": True, "steps": args.prefill_steps,
         "us_per_layer": round(aggregate(p_ms, args.prefill_steps, len(fl), world), 2),
         "tflops": round(tflops * world, 1),
-        "tensor_frac": round(tflops / peaks["bf16_tflops_sustained"], 3),
-        "peak_tflops": peaks["bf16_tflops_sustained"],
+        # each layer is a graph of 0.2-0.7 ms and the step a few ms: the burst peak applies
+        "tensor_frac": round(tflops / peaks["bf16_tflops"], 3),
+        "peak_tflops": peaks["bf16_tflops"],
+        "peak_kind": "burst (cuBLAS bf16, timed alone)",
+        "tensor_frac_of_sustained": round(tflops / peaks["bf16_tflops_sustained"], 3),
         "per_layer_us": {L["name"]: round(p_per[i] * 1e3, 1) for i, L in enumerate(pre.layers)},
         "dominant": {"kernel": f"fq_linear_forward[{pre.layers[pdom]['name']}]",
                      "achieved_tflops": round(fl[pdom] / (p_per[pdom] * 1e-3) / 1e12, 1),
                      "frac": round(fl[pdom] / (p_per[pdom] * 1e-3) / 1e12
-                                   / peaks["bf16_tflops_sustained"], 3)},
+                                   / peaks["bf16_tflops"], 3)},
     }
     del pg, lgs, pre
     torch.cuda.empty_cache()
@@ -683,6 +736,122 @@ def sweep(args, fq, wl, torch, dev, stream, peaks):
         "sweep": rows}), flush=True)
 
 
+# --------------------------------------------------------------------------- summaries
+SUMMARY_PLAN = (
+    # (configuration, workload, layer, r, M, gamma, seeded codes)
+    ("cfg1 single 256x256", "single256", "single", None, 8, False, False),
+    ("cfg2 ViT-B/16 fc1 3072x768", "vit_b16_mlp", "fc1", None, 12608, False, False),
+    ("cfg2 ViT-B/16 fc2 768x3072", "vit_b16_mlp", "fc2", None, 12608, False, False),
+    ("cfg4 7B gate 11008x4096", "llama2_7b_prefill", "gate", None, 4096, True, False),
+    ("cfg5 70B q 8192x8192", "llama2_70b", "q", "11/10", 16, False, True),
+    ("cfg5 70B gate 28672x8192", "llama2_70b", "gate", "11/10", 16, False, True),
+    ("cfg5 70B down 8192x28672", "llama2_70b", "down", "11/10", 128, False, True),
+    ("cfg5 70B q 8192x8192 M=4096", "llama2_70b", "q", "11/10", 4096, False, True),
+)
+
+
+def config_summary(fq, wl, torch, dev, stream, peaks):
+    """One representative layer of the configurations the headline block does not cover,
+    timed cold (a 258 MB L2 flush before each call, CUDA events around the call): us/layer,
+    tokens/s and the fraction of max(bytes / HBM peak, FLOPs / burst bf16 peak)."""
+    from fractions import Fraction
+    flush = torch.zeros(2 * 129 * 2**20 // 4, dtype=torch.float32, device=dev)
+    out = {}
+    for label, key, name, r, M, use_gamma, seeded in SUMMARY_PLAN:
+        wk = wl.WORKLOADS[key]
+        layer = next(l for l in wk.layers if l.name == name)
+        rr = wk.redundancy[0] if r is None else Fraction(r)
+        prep = prepare_layer_random_codes if seeded else prepare_layer
+        L = prep(fq, wl, torch, wk, layer, rr, dev)
+        X = torch.from_numpy(wl.activations(wk, layer, M)).to(dev, torch.bfloat16)
+        cold, warm = time_layer(fq, torch, L, X, use_gamma, dev, stream, flush, reps=20,
+                                warm_calls=10)
+        args_ = (L["d_in"], L["d_out"], L["n_in"], L["n_out"], M)
+        by, fl = layer_bytes(*args_), layer_flops(*args_)
+        t_hbm = by / (peaks["hbm_gbs"] * 1e9) * 1e6
+        t_tc = fl / (peaks["bf16_tflops"] * 1e12) * 1e6
+        out[label] = {"M": M, "r": str(rr), "gamma": use_gamma, "us_cold": round(cold, 2),
+                      "us_warm": round(warm, 2), "tokens_per_s": round(M / cold * 1e6),
+                      "bound": "hbm" if t_hbm >= t_tc else "tensor",
+                      "roof_us": round(max(t_hbm, t_tc), 2),
+                      "frac_cold": round(max(t_hbm, t_tc) / cold, 3),
+                      "codes": "seeded uniform" if seeded else "RTN of C"}
+        del L, X
+        torch.cuda.empty_cache()
+    del flush
+    torch.cuda.empty_cache()
+    return out
+
+
+def reconstruction_crossover(fq, wl, torch, dev, stream, peaks):
+    """The weight-reconstruction path against the frame forward on the 7B q and gate shapes
+    at 2048 and 4096 tokens: the one-off fq_reconstruct_weight, then fq_dense_forward per batch,
+    against fq_linear_forward per batch (cold, median of 10).  The crossover is the number of
+    batches after which reconstructing once and running dense products is cheaper."""
+    wk = wl.WORKLOADS["llama2_7b_prefill"]
+    flush = torch.zeros(2 * 129 * 2**20 // 4, dtype=torch.float32, device=dev)
+
+    def cold_us(fn, reps=10):
+        with torch.cuda.stream(stream):
+            fn()
+            fn()
+        torch.cuda.synchronize()
+        evs = []
+        with torch.cuda.stream(stream):
+            for _ in range(reps):
+                flush.add_(1)
+                e0 = torch.cuda.Event(enable_timing=True)
+                e1 = torch.cuda.Event(enable_timing=True)
+                e0.record(stream)
+                fn()
+                e1.record(stream)
+                evs.append((e0, e1))
+        torch.cuda.synchronize()
+        return statistics.median(a.elapsed_time(b) for a, b in evs) * 1e3
+
+    out = {}
+    for name in ("q", "gate"):
+        layer = next(l for l in wk.layers if l.name == name)
+        L = prepare_layer(fq, wl, torch, wk, layer, wk.redundancy[0], dev)
+        d_in, d_out = L["d_in"], L["d_out"]
+        W = torch.empty(d_out, d_in, dtype=torch.bfloat16, device=dev)
+        nr = fq.fq_reconstruct_workspace_bytes(d_in, L["n_in"], L["n_out"], d_out)
+        wsr = torch.zeros(nr, dtype=torch.uint8, device=dev)
+        rec = cold_us(lambda: fq.fq_reconstruct_weight(
+            L["T_in"], L["C"], L["T_out_t"], d_in, d_out, None, W, wsr, nr, stream.cuda_stream),
+            reps=3)
+        if fq.fq_check(wsr) != 0:
+            raise RuntimeError(f"reconstruct {name}: device status")
+        del wsr
+        torch.cuda.empty_cache()
+        for M in (2048, 4096):
+            x = torch.from_numpy(wl.activations(wk, layer, M)).to(dev, torch.bfloat16)
+            y = torch.empty(M, d_out, dtype=torch.bfloat16, device=dev)
+            nf = fq.fq_workspace_bytes(M, d_in, L["n_in"], L["n_out"], d_out, 0)
+            wsf = torch.zeros(nf, dtype=torch.uint8, device=dev)
+            nd = fq.fq_dense_workspace_bytes(M, d_in, d_out)
+            wsd = torch.zeros(nd, dtype=torch.uint8, device=dev)
+            fwd = cold_us(lambda: fq.fq_linear_forward(
+                x, M, d_in, L["T_in"], L["C"], L["T_out_t"], d_out, None, y, wsf, nf, 0,
+                stream.cuda_stream))
+            dense = cold_us(lambda: fq.fq_dense_forward(x, M, d_in, W, d_out, y, wsd, nd,
+                                                        stream.cuda_stream))
+            fl_dense = 2 * M * d_in * d_out
+            out[f"{name} {d_out}x{d_in} M={M}"] = {
+                "forward_us": round(fwd, 1), "dense_us": round(dense, 1),
+                "reconstruct_us": round(rec, 1),
+                "dense_tflops": round(fl_dense / (dense * 1e-6) / 1e12, 1),
+                "dense_frac": round(fl_dense / (dense * 1e-6) / 1e12 / peaks["bf16_tflops"], 3),
+                "crossover_batches": (round(rec / (fwd - dense), 2) if fwd > dense else None),
+            }
+            del x, y, wsf, wsd
+            torch.cuda.empty_cache()
+        del L, W
+        torch.cuda.empty_cache()
+    del flush
+    return out
+
+
 # --------------------------------------------------------------------------- main
 def aggregate(elapsed_ms, steps, layers_per_step, world):
     """Whole-job microseconds per layer from the slowest rank's elapsed time: every rank
@@ -711,6 +880,8 @@ def main(argv=None):
     ap.add_argument("--regime", default="both", choices=["both", "decode", "prefill"],
                     help="decode (the headline), prefill, or both (default)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-summary", action="store_true",
+                    help="skip the per-configuration summary and the reconstruction crossover")
     ap.add_argument("--sweep", action="store_true",
                     help="time every configuration's layer shapes (one JSON line) and exit")
     args = ap.parse_args(argv)
@@ -759,10 +930,18 @@ def main(argv=None):
 
     # ---------------- decode: Llama-2-7B block, M = 16
     dec = Regime(fq, wl, torch, "llama2_7b_decode", 16, dev, rank)
-    step_graph = dec.capture(dec.layers, stream, chain=True)
-    layer_graphs = [dec.capture([L], stream) for L in dec.layers]
-    e2e_graph = dec.capture(dec.layers, stream, host=True, chain=True)
     nL = len(dec.layers)
+    nG = len(dec.groups)
+    step_graph = dec.capture_groups(stream)
+    launch_graphs = []
+    for gi in range(nG):
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, stream=stream):
+            dec.launch_groups(stream, only=gi)
+        launch_graphs.append(g)
+    seq_graph = dec.capture(dec.layers, stream, chain=True)
+    layer_graphs = [dec.capture([L], stream) for L in dec.layers]
+    e2e_graph = dec.capture_groups(stream, host=True)
 
     uuid = None
     try:
@@ -775,60 +954,76 @@ def main(argv=None):
     barrier()
     total_ms = max_over_ranks(total_ms, dist, dev)
     us_layer = aggregate(total_ms, args.steps, nL, world)
+    if fq.fq_check(dec.ws) != 0:
+        raise RuntimeError("decode block: device status after timing")
 
-    # per-layer durations (events between per-layer graphs) for the roofline
+    # per-launch durations (events between per-launch graphs) for the roofline
     rl_steps = max(50, args.steps // 4)
+    _, per_launch = timed_replays(torch, launch_graphs, stream, rl_steps, args.warmup,
+                                  events_between=True)
+    bytes_fl = {L["name"]: dec.bytes_flops(L) for L in dec.layers}
+    launch_bytes = [sum(bytes_fl[L["name"]][0] for L in grp) for grp in dec.groups]
+    dom = max(range(nG), key=lambda i: per_launch[i])
+    achieved = launch_bytes[dom] / (per_launch[dom] * 1e-3) / 1e9
+    step_bytes = sum(launch_bytes)
+    dom_names = "|".join(L["name"] for L in dec.groups[dom])
+
+    # the same block as 7 single-layer launches (each naming the next layer's T_in as its
+    # L2 hint), and each layer alone
+    barrier()
+    seq_ms, _ = timed_replays(torch, [seq_graph], stream, args.steps, args.warmup)
+    seq_ms = max_over_ranks(seq_ms, dist, dev)
+    seq_us = aggregate(seq_ms, args.steps, nL, world)
     _, per_ms = timed_replays(torch, layer_graphs, stream, rl_steps, args.warmup,
                               events_between=True)
-    bytes_fl = [dec.bytes_flops(L) for L in dec.layers]
-    dom = max(range(nL), key=lambda i: per_ms[i])
-    dom_bytes = bytes_fl[dom][0]
-    achieved = dom_bytes / (per_ms[dom] * 1e-3) / 1e9
-    step_bytes = sum(b for b, _ in bytes_fl)
-
-    # the same block with independent layers side by side (q|k|v, o, gate|up, down)
-    sms = torch.cuda.get_device_properties(dev).multi_processor_count
-    groups = [(["q", "k", "v"], sms // 3), (["o"], 0), (["gate", "up"], sms // 2),
-              (["down"], 0)]
-    grouped_graph = dec.capture_grouped(groups, stream)
-    barrier()
-    grp_ms, _ = timed_replays(torch, [grouped_graph], stream, args.steps, args.warmup)
-    grp_ms = max_over_ranks(grp_ms, dist, dev)
-    grp_us = aggregate(grp_ms, args.steps, nL, world)
-    grouped = {
-        "value": round(grp_us, 3), "unit": UNIT, "ms_per_step": round(grp_ms / args.steps, 4),
-        "groups": " ; ".join(f"{'|'.join(n)}@{b or sms} SMs" for n, b in groups),
-        "how": ("fq_linear_forward_sms: the layers of a group run on parallel streams, each "
-                "with its own workspace and SM budget; groups run in order; one CUDA graph "
-                "per step"),
+    sequential = {
+        "value": round(seq_us, 3), "unit": UNIT, "ms_per_step": round(seq_ms / args.steps, 4),
+        "how": "one fq_linear_forward_ex launch per layer (7 per step), one CUDA graph per step",
+        "per_layer": {L["name"]: {"us": round(per_ms[i] * 1e3, 2),
+                                  "GBps": round(bytes_fl[L["name"]][0] / (per_ms[i] * 1e-3) / 1e9,
+                                                1),
+                                  "hbm_frac": round(bytes_fl[L["name"]][0] / (per_ms[i] * 1e-3)
+                                                    / 1e9 / peaks["hbm_gbs"], 3)}
+                      for i, L in enumerate(dec.layers)},
     }
-    del grouped_graph
+    del seq_graph, layer_graphs
 
     # the same block with the frames in structured form (fq_linear_forward_implicit)
     implicit = measure_implicit(args, fq, wl, torch, dec, stream, peaks)
 
-    # end to end through the C ABI with host buffers
+    # end to end through the C ABI with host buffers: plain calls (the API's host work inside
+    # the timed region), and the same step captured once as a CUDA graph
     barrier()
-    e2e_ms, _ = timed_replays(torch, [e2e_graph], stream, max(100, args.steps // 4),
-                              args.warmup)
+    e2e_steps = max(100, args.steps // 4)
+    e2e_ms = eager_e2e(torch, dec, stream, e2e_steps, args.warmup)
     e2e_ms = max_over_ranks(e2e_ms, dist, dev)
-    e2e_us = aggregate(e2e_ms, max(100, args.steps // 4), nL, world)
+    e2e_us = aggregate(e2e_ms, e2e_steps, nL, world)
+    e2eg_ms, _ = timed_replays(torch, [e2e_graph], stream, e2e_steps, args.warmup)
+    e2eg_ms = max_over_ranks(e2eg_ms, dist, dev)
+    e2eg_us = aggregate(e2eg_ms, e2e_steps, nL, world)
     h2d, d2h = dec.host_bytes()
 
-    per_layer = {L["name"]: {"us": round(per_ms[i] * 1e3, 2),
-                             "GBps": round(bytes_fl[i][0] / (per_ms[i] * 1e-3) / 1e9, 1),
-                             "hbm_frac": round(bytes_fl[i][0] / (per_ms[i] * 1e-3) / 1e9
-                                               / peaks["hbm_gbs"], 3)}
-                 for i, L in enumerate(dec.layers)}
+    per_launch_out = {
+        "|".join(L["name"] for L in grp): {
+            "us": round(per_launch[i] * 1e3, 2),
+            "GBps": round(launch_bytes[i] / (per_launch[i] * 1e-3) / 1e9, 1),
+            "hbm_frac": round(launch_bytes[i] / (per_launch[i] * 1e-3) / 1e9 / peaks["hbm_gbs"],
+                              3)}
+        for i, grp in enumerate(dec.groups)}
     roof_us = step_bytes / (peaks["hbm_gbs"] * 1e9) * 1e6 / nL
-    del step_graph, layer_graphs, e2e_graph
+    del step_graph, launch_graphs, e2e_graph
     dec_layers = [(L["name"], L["d_out"], L["d_in"], L["k_in"], L["k_out"]) for L in dec.layers]
+    group_names = " ; ".join("|".join(L["name"] for L in grp) for grp in dec.groups)
     del dec
     torch.cuda.empty_cache()
 
     # ---------------- prefill: same block, M = 2048, de-noising filter on
     prefill = None if args.no_prefill else measure_prefill(args, fq, wl, torch, dev, rank, world,
                                                             dist, stream, peaks)
+    summary = crossover = None
+    if world == 1 and not args.no_summary:
+        summary = config_summary(fq, wl, torch, dev, stream, peaks)
+        crossover = reconstruction_crossover(fq, wl, torch, dev, stream, peaks)
 
     if dist is not None:
         dist.barrier()
@@ -854,29 +1049,39 @@ def main(argv=None):
             "layers": {n: f"{o}x{i} k_in={ki} k_out={ko}" for n, o, i, ki, ko in dec_layers},
             "l2": ("no flush: each step streams 1.2 GB of distinct layer operands (> 126 MB "
                    "L2), so every layer's operands were last touched one step earlier"),
-            "timing": ("one CUDA graph per step (7 layer forwards, each naming the next layer's "
-                       "T_in as its L2 prefetch hint), CUDA events around K replays"),
+            "timing": ("one CUDA graph per step: the block's 4 launches (" + group_names +
+                       "; q|k|v and gate|up each one fq_linear_forward_group call), each naming "
+                       "the next launch's T_in as its L2 prefetch hint; CUDA events around K "
+                       "replays"),
             "parallelism": f"replicas x{world}, no data-path collective",
         },
         "roofline": {
-            "bound": "hbm", "kernel": (f"decode_layer_kernel[{dec_layers[dom][0]}] "
-                                       "(analysis, code product and synthesis fused)"),
+            "bound": "hbm", "kernel": (f"decode_layer_kernel[{dom_names}] (analysis, code "
+                                       "product and synthesis fused, one launch)"),
             "achieved": round(achieved, 1), "peak": peaks["hbm_gbs"], "unit": "GB/s",
             "frac": round(achieved / peaks["hbm_gbs"], 3),
-            "traffic": recorded_traffic(f"decode_{dec_layers[dom][0]}"),
+            "traffic": recorded_traffic(f"decode_{dom_names}"),
             "peak_source": f"{peak_src} (STREAM-style copy)",
             "step_frac": round(roof_us / us_layer, 3),
-            "per_layer": per_layer,
+            "per_launch": per_launch_out,
         },
-        "grouped": grouped,
+        "sequential": sequential,
         "implicit": implicit,
         "e2e": {"value": round(e2e_us, 3), "unit": UNIT, "h2d_bytes_per_step": h2d,
                 "d2h_bytes_per_step": d2h,
                 "copies": ("per step: one host-to-device copy of the 7 layers' inputs from pinned "
-                           "memory, the 7 forwards, one device-to-host copy of their outputs")},
-        "gpu_launches": nL * args.steps,      # one fused kernel per layer forward (M <= 64)
+                           "memory, the block's 4 launches, one device-to-host copy of their "
+                           "outputs"),
+                "how": ("plain calls: each step issues the copies and the 4 forward calls through "
+                        "the C ABI (argument checks, tensor-map encoding and plan lookup on the "
+                        "host inside the timed region); CUDA events around K steps"),
+                "graph_value": round(e2eg_us, 3),
+                "graph_how": "the same step captured once in a CUDA graph and replayed"},
+        "gpu_launches": nG * args.steps,      # one fused kernel per launch (M <= 64)
         "clocks": clocks,
         "prefill": prefill,
+        "configs": summary,
+        "reconstruction": crossover,
         "cpu_baseline": cpu,
     }
     print(json.dumps(line), flush=True)

@@ -192,6 +192,48 @@ fq_status fq_linear_forward_ex(const void* x, int M, int d_in, const void* T_in,
                                const float* gamma, void* y, void* ws, size_t ws_bytes, int mode,
                                const fq_forward_opts* opts, fq_stream_t stream);
 
+/* One layer of fq_linear_forward_group: the arguments of fq_linear_forward for that layer. */
+typedef struct {
+  const void* x;           /* device bf16, M x d_in tokens */
+  int32_t d_in;
+  const void* T_in;        /* device bf16, n_in x d_in */
+  const fq_packed* C;      /* host pointer to the layer's packed descriptor */
+  const void* T_out_t;     /* device bf16, d_out x n_out */
+  int32_t d_out;
+  const float* gamma;      /* device fp32 [n_out] or NULL */
+  void* y;                 /* device bf16, M x d_out output */
+} fq_layer;
+
+/* Most layers one fq_linear_forward_group call takes. */
+#define FQ_MAX_GROUP 4
+
+/* Bytes of workspace fq_linear_forward_group needs for these layers at M tokens (FQ_BF16);
+ * 0 for invalid sizes or counts.  It is at least fq_workspace_bytes of each layer, so the
+ * workspace also serves the layers' single calls. */
+size_t fq_group_workspace_bytes(int M, int n_layers, const fq_layer* layers);
+
+/* The FQ_BF16 forward of up to FQ_MAX_GROUP independent layers in one call: q, k and v of an
+ * attention block, or gate and up of an MLP, which read the same input and whose outputs no
+ * layer of the group reads.  Each layer's result is that of fq_linear_forward on its own
+ * arguments.  For M <= 64 the layers run in one fused launch whose task lists interleave the
+ * layers' phases (analysis, code product, synthesis), so that the point where one layer's
+ * next phase waits for all of its previous phase falls while another layer streams its
+ * weights; larger batches, which are tensor-bound, run the layers one after another.
+ *   layers   host array of n_layers descriptors (1 <= n_layers <= FQ_MAX_GROUP); the layers may
+ *            differ in every size; x may be shared; no y may equal another layer's x or y
+ *   ws       device workspace of fq_group_workspace_bytes(M, n_layers, layers) bytes, with the
+ *            rules of fq_linear_forward (256-byte aligned, zero-filled before its first use,
+ *            reusable, zeroed again after FQ_ERR_TIMEOUT; status word at its head)
+ *   opts     as in fq_linear_forward_ex (NULL: none); inject_timeout_cycles must be 0
+ * Requirements and errors: those of fq_linear_forward for each layer; FQ_ERR_INVALID_ARG for a
+ * bad count or an output that is another layer's input or output; FQ_ERR_UNSUPPORTED when the
+ * layers' ready flags do not fit the workspace header (more than 2016 row tiles of 128 over
+ * the layers' analyses and code products).  This entry point has no counterpart in the
+ * paper. */
+fq_status fq_linear_forward_group(int M, int n_layers, const fq_layer* layers, void* ws,
+                                  size_t ws_bytes, const fq_forward_opts* opts,
+                                  fq_stream_t stream);
+
 /* ------------------------------------------------------------------------------------------
  * Offline preparation of a layer (not on the inference path).  These produce the inputs of
  * fq_linear_forward on the device from a weight matrix W and the frame parameters.

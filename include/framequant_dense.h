@@ -21,7 +21,10 @@
 extern "C" {
 #endif
 
-/* Workspace bytes of fq_reconstruct_weight; 0 for invalid sizes. */
+/* Workspace bytes of fq_reconstruct_weight; 0 for invalid sizes.  It holds the forward's
+ * workspace for M = d_in tokens, the d_in x d_in identity those tokens are, and the d_in x d_out
+ * forward output: about 142 MB for a 4096 x 4096 layer at r = 1.1, 261 MB for 11008 x 4096,
+ * 703 MB for 4096 x 11008, 567 MB for 8192 x 8192 and 4.5 GB for 8192 x 28672. */
 size_t fq_reconstruct_workspace_bytes(int d_in, int n_in, int n_out, int d_out);
 
 /* W_hat = T_out^T diag(gamma) C_hat T_in, bf16 d_out x d_in row-major: the FQ_BF16 forward of

@@ -22,8 +22,10 @@ __all__ = [
     "fq_linear_forward_static", "FQ_STATIC_SCRATCH_BYTES", "Frame", "fq_frame_implicit_bytes",
     "fq_frame_implicit", "fq_implicit_workspace_bytes", "fq_linear_forward_implicit",
     "fq_reconstruct_workspace_bytes", "fq_reconstruct_weight", "fq_dense_workspace_bytes",
-    "fq_dense_forward", "fq_static_check",
+    "fq_dense_forward", "fq_static_check", "fq_group_workspace_bytes",
+    "fq_linear_forward_group", "Layer", "FQ_MAX_GROUP",
 ]
+FQ_MAX_GROUP = 4
 FQ_STATIC_SCRATCH_BYTES = 16 << 20
 
 FQ_BF16 = 0
@@ -38,7 +40,8 @@ EXPORTED = ("fq_packed_words", "fq_pack", "fq_workspace_bytes", "fq_linear_forwa
             "fq_linear_forward_static", "fq_frame_implicit_bytes", "fq_frame_implicit",
             "fq_implicit_workspace_bytes", "fq_linear_forward_implicit",
             "fq_reconstruct_workspace_bytes", "fq_reconstruct_weight", "fq_dense_workspace_bytes",
-            "fq_dense_forward", "fq_static_check")
+            "fq_dense_forward", "fq_static_check", "fq_group_workspace_bytes",
+            "fq_linear_forward_group")
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
 
@@ -68,6 +71,12 @@ class _Rotation(ctypes.Structure):
 class _Opts(ctypes.Structure):
     _fields_ = [("max_sms", ctypes.c_int32), ("l2_prefetch", ctypes.c_void_p),
                 ("l2_prefetch_bytes", ctypes.c_size_t), ("inject_timeout_cycles", ctypes.c_int64)]
+
+
+class _Layer(ctypes.Structure):
+    _fields_ = [("x", ctypes.c_void_p), ("d_in", ctypes.c_int32), ("T_in", ctypes.c_void_p),
+                ("C", ctypes.POINTER(_Packed)), ("T_out_t", ctypes.c_void_p),
+                ("d_out", ctypes.c_int32), ("gamma", ctypes.c_void_p), ("y", ctypes.c_void_p)]
 
 
 class _Frame(ctypes.Structure):
@@ -137,6 +146,12 @@ def lib() -> ctypes.CDLL:
             ctypes.c_void_p, ctypes.c_int, ctypes.c_int, ctypes.c_void_p,
             ctypes.POINTER(_Packed), ctypes.c_void_p, ctypes.c_int, ctypes.c_void_p,
             ctypes.c_void_p, ctypes.c_int, ctypes.c_void_p]
+        L.fq_group_workspace_bytes.restype = ctypes.c_size_t
+        L.fq_group_workspace_bytes.argtypes = [ctypes.c_int, ctypes.c_int, ctypes.POINTER(_Layer)]
+        L.fq_linear_forward_group.restype = ctypes.c_int
+        L.fq_linear_forward_group.argtypes = [ctypes.c_int, ctypes.c_int, ctypes.POINTER(_Layer),
+                                              ctypes.c_void_p, ctypes.c_size_t,
+                                              ctypes.POINTER(_Opts), ctypes.c_void_p]
         L.fq_static_check.restype = ctypes.c_int
         L.fq_static_check.argtypes = [ctypes.c_void_p]
         L.fq_frame_implicit_bytes.restype = ctypes.c_size_t
@@ -282,6 +297,48 @@ def fq_linear_forward_static(x, M: int, d_in: int, T_in, C: Packed, T_out_t, d_o
     _ok(lib().fq_linear_forward_static(_ptr(x), M, d_in, _ptr(T_in), ctypes.byref(pc),
                                        _ptr(T_out_t), d_out, _ptr(gamma), _ptr(y), mode,
                                        _stream(stream)), "fq_linear_forward_static")
+
+
+@dataclass
+class Layer:
+    """One layer of fq_linear_forward_group (the arguments of fq_linear_forward)."""
+    x: object
+    d_in: int
+    T_in: object
+    C: Packed
+    T_out_t: object
+    d_out: int
+    gamma: object
+    y: object
+
+
+def _layers(layers):
+    """C array of fq_layer, and the packed descriptors it points to (kept alive by the caller)."""
+    packs = [L.C._c() for L in layers]
+    arr = (_Layer * len(layers))()
+    for i, (L, pc) in enumerate(zip(layers, packs)):
+        arr[i] = _Layer(_ptr(L.x), L.d_in, _ptr(L.T_in), ctypes.pointer(pc), _ptr(L.T_out_t),
+                        L.d_out, _ptr(L.gamma), _ptr(L.y))
+    return arr, packs
+
+
+def fq_group_workspace_bytes(M: int, layers) -> int:
+    arr, packs = _layers(layers)
+    n = lib().fq_group_workspace_bytes(M, len(layers), arr)
+    del packs
+    return n
+
+
+def fq_linear_forward_group(M: int, layers, ws, ws_bytes: int, max_sms: int = 0, prefetch=None,
+                            stream=None) -> None:
+    """The FQ_BF16 forward of independent layers (list of Layer) in one call."""
+    arr, packs = _layers(layers)
+    nb = 0 if prefetch is None else prefetch.numel() * prefetch.element_size()
+    opts = _Opts(max_sms, _ptr(prefetch), nb, 0)
+    _ok(lib().fq_linear_forward_group(M, len(layers), arr, _ptr(ws), ws_bytes,
+                                      ctypes.byref(opts), _stream(stream)),
+        "fq_linear_forward_group")
+    del packs
 
 
 def fq_static_check(stream=None) -> int:

@@ -2,6 +2,8 @@
 // dispatch to the bf16 tensor-core path (fq_tc.cu) or the fp32 debug path (fq_debug.cu).
 #include <cuda_runtime.h>
 
+#include <algorithm>
+
 #include "fq_internal.h"
 
 using namespace fq;
@@ -75,18 +77,14 @@ size_t fq_workspace_bytes(int M, int d_in, int n_in, int n_out, int d_out, int m
   return 0;
 }
 
-fq_status fq_linear_forward_ex(const void* x, int M, int d_in, const void* T_in,
-                               const fq_packed* C, const void* T_out_t, int d_out,
-                               const float* gamma, void* y, void* ws, size_t ws_bytes, int mode,
-                               const fq_forward_opts* opts, fq_stream_t stream) {
-  const int max_sms = opts ? opts->max_sms : 0;
-  const void* pf = opts ? opts->l2_prefetch : nullptr;
-  const size_t pf_bytes = opts ? (opts->l2_prefetch_bytes & ~static_cast<size_t>(15)) : 0;
-  const int64_t inject = opts ? opts->inject_timeout_cycles : 0;
-  if (max_sms < 0 || (pf_bytes > 0 && !pf) || inject < 0) return FQ_ERR_INVALID_ARG;
-  if (inject > 0 && (mode != FQ_BF16 || M <= 0 || M > kDecodeMaxM || max_sms != 1))
-    return FQ_ERR_INVALID_ARG;
-  if (pf_bytes > 0 && !aligned16(pf)) return FQ_ERR_ALIGNMENT;
+}  // extern "C"
+
+namespace {
+
+// The host-side checks of one layer forward, before anything is launched.
+fq_status check_layer(const void* x, int M, int d_in, const void* T_in, const fq_packed* C,
+                      const void* T_out_t, int d_out, const float* gamma, const void* y,
+                      int mode) {
   if (!x || !T_in || !C || !T_out_t || !y) return FQ_ERR_INVALID_ARG;
   if (mode != FQ_BF16 && mode != FQ_FP32_DEBUG) return FQ_ERR_INVALID_ARG;
   if (M <= 0 || d_in <= 0 || d_out <= 0) return FQ_ERR_INVALID_ARG;
@@ -95,10 +93,56 @@ fq_status fq_linear_forward_ex(const void* x, int M, int d_in, const void* T_in,
   if (!aligned16(x) || !aligned16(T_in) || !aligned16(T_out_t) || !aligned16(y) ||
       (gamma && !aligned16(gamma)))
     return FQ_ERR_ALIGNMENT;
+  return FQ_OK;
+}
+
+fq_status check_opts(const fq_forward_opts* opts, int& max_sms, const void*& pf,
+                     size_t& pf_bytes, int64_t& inject) {
+  max_sms = opts ? opts->max_sms : 0;
+  pf = opts ? opts->l2_prefetch : nullptr;
+  pf_bytes = opts ? (opts->l2_prefetch_bytes & ~static_cast<size_t>(15)) : 0;
+  inject = opts ? opts->inject_timeout_cycles : 0;
+  if (max_sms < 0 || (pf_bytes > 0 && !pf) || inject < 0) return FQ_ERR_INVALID_ARG;
+  if (pf_bytes > 0 && !aligned16(pf)) return FQ_ERR_ALIGNMENT;
+  return FQ_OK;
+}
+
+fq_status check_ws(const void* ws, size_t ws_bytes, size_t need) {
   if (!ws) return FQ_ERR_WORKSPACE;
   if ((reinterpret_cast<uintptr_t>(ws) & 255u) != 0) return FQ_ERR_ALIGNMENT;
-  const size_t need = fq_workspace_bytes(M, d_in, C->n_in, C->n_out, d_out, mode);
   if (ws_bytes < need) return FQ_ERR_WORKSPACE;
+  return FQ_OK;
+}
+
+// The group's layers as the decode kernel takes them.
+bool group_layers(int n, const fq_layer* layers, DecGroupLayer* out) {
+  for (int l = 0; l < n; ++l) {
+    const fq_layer& L = layers[l];
+    if (!L.C) return false;
+    out[l] = DecGroupLayer{L.x, L.d_in, L.T_in, *L.C, L.T_out_t, L.d_out, L.gamma, L.y};
+  }
+  return true;
+}
+
+}  // namespace
+
+extern "C" {
+
+fq_status fq_linear_forward_ex(const void* x, int M, int d_in, const void* T_in,
+                               const fq_packed* C, const void* T_out_t, int d_out,
+                               const float* gamma, void* y, void* ws, size_t ws_bytes, int mode,
+                               const fq_forward_opts* opts, fq_stream_t stream) {
+  int max_sms = 0;
+  const void* pf = nullptr;
+  size_t pf_bytes = 0;
+  int64_t inject = 0;
+  if (const fq_status os = check_opts(opts, max_sms, pf, pf_bytes, inject)) return os;
+  if (inject > 0 && (mode != FQ_BF16 || M <= 0 || M > kDecodeMaxM || max_sms != 1))
+    return FQ_ERR_INVALID_ARG;
+  if (const fq_status ls = check_layer(x, M, d_in, T_in, C, T_out_t, d_out, gamma, y, mode))
+    return ls;
+  const size_t need = fq_workspace_bytes(M, d_in, C->n_in, C->n_out, d_out, mode);
+  if (const fq_status ws_st = check_ws(ws, ws_bytes, need)) return ws_st;
   auto s = reinterpret_cast<cudaStream_t>(stream);
   if (mode == FQ_FP32_DEBUG) {
     if (cudaMemsetAsync(ws, 0, kWsHeader, s) != cudaSuccess) return FQ_ERR_CUDA;
@@ -115,6 +159,66 @@ fq_status fq_linear_forward_ex(const void* x, int M, int d_in, const void* T_in,
                                  s);
   return launch_tc_forward(x, M, d_in, T_in, *C, T_out_t, d_out, gamma, y,
                            static_cast<char*>(ws), ws_bytes, max_sms, s);
+}
+
+size_t fq_group_workspace_bytes(int M, int n_layers, const fq_layer* layers) {
+  if (M <= 0 || n_layers < 1 || n_layers > FQ_MAX_GROUP || !layers) return 0;
+  size_t need = 0;
+  for (int l = 0; l < n_layers; ++l) {
+    const fq_layer& L = layers[l];
+    if (!L.C) return 0;
+    const size_t one = fq_workspace_bytes(M, L.d_in, L.C->n_in, L.C->n_out, L.d_out, FQ_BF16);
+    if (one == 0) return 0;
+    need = std::max(need, one);
+  }
+  if (M <= kDecodeMaxM) {
+    DecGroupLayer g[FQ_MAX_GROUP];
+    if (!group_layers(n_layers, layers, g)) return 0;
+    need = std::max(need, decode_group_workspace_bytes(M, n_layers, g));
+  }
+  return need;
+}
+
+fq_status fq_linear_forward_group(int M, int n_layers, const fq_layer* layers, void* ws,
+                                  size_t ws_bytes, const fq_forward_opts* opts,
+                                  fq_stream_t stream) {
+  int max_sms = 0;
+  const void* pf = nullptr;
+  size_t pf_bytes = 0;
+  int64_t inject = 0;
+  if (const fq_status os = check_opts(opts, max_sms, pf, pf_bytes, inject)) return os;
+  if (inject != 0 || !layers || n_layers < 1 || n_layers > FQ_MAX_GROUP)
+    return FQ_ERR_INVALID_ARG;
+  for (int l = 0; l < n_layers; ++l) {
+    const fq_layer& L = layers[l];
+    if (const fq_status ls = check_layer(L.x, M, L.d_in, L.T_in, L.C, L.T_out_t, L.d_out,
+                                         L.gamma, L.y, FQ_BF16))
+      return ls;
+    // independent layers: no output is another layer's input or output
+    for (int j = 0; j < n_layers; ++j)
+      if (j != l && (layers[j].y == L.y || layers[j].x == L.y)) return FQ_ERR_INVALID_ARG;
+    if (L.x == L.y) return FQ_ERR_INVALID_ARG;
+  }
+  const size_t need = fq_group_workspace_bytes(M, n_layers, layers);
+  if (need == 0) return FQ_ERR_INVALID_ARG;
+  if (const fq_status ws_st = check_ws(ws, ws_bytes, need)) return ws_st;
+  if (current_cc() != 103) return FQ_ERR_UNSUPPORTED;
+  auto s = reinterpret_cast<cudaStream_t>(stream);
+  if (M <= kDecodeMaxM) {
+    DecGroupLayer g[FQ_MAX_GROUP];
+    group_layers(n_layers, layers, g);
+    return launch_decode_group(M, n_layers, g, static_cast<char*>(ws), ws_bytes, max_sms, false,
+                               pf, pf_bytes, 0, s);
+  }
+  // larger batches are tensor-bound: the layers run one after another on the tensor-core path
+  for (int l = 0; l < n_layers; ++l) {
+    const fq_layer& L = layers[l];
+    if (const fq_status st = launch_tc_forward(L.x, M, L.d_in, L.T_in, *L.C, L.T_out_t, L.d_out,
+                                               L.gamma, L.y, static_cast<char*>(ws), ws_bytes,
+                                               max_sms, s))
+      return st;
+  }
+  return FQ_OK;
 }
 
 fq_status fq_linear_forward_sms(const void* x, int M, int d_in, const void* T_in,

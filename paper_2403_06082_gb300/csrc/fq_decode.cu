@@ -101,18 +101,32 @@ struct DecPhase {
   uint32_t* flags;        // [RT][kWsSlices] slice final in this call when == generation + 1
 };
 
-struct DecArgs {
-  int M, S, total;
+// One launch runs up to kMaxGroup independent layers (no layer reads another's output), e.g.
+// q, k and v of an attention block, or gate and up of an MLP; a single layer is a group of 1.
+constexpr int kMaxGroup = FQ_MAX_GROUP;
+
+struct DecLayer {
   DecPhase ph[3];
   const uint32_t* words;
   const __half* scale;
   const __half* zero;
   const float* gamma;
+  int pf_tout;            // prefetch the T_out^T tiles of this CTA's synthesis tasks into L2
+};
+
+// Tensor maps per layer: T_in, x, z, T_out^T, u.
+enum { kMapTin = 0, kMapX = 1, kMapZ = 2, kMapTout = 3, kMapU = 4, kMapsPerLayer = 5 };
+struct DecMaps {
+  CUtensorMap m[kMaxGroup][kMapsPerLayer];
+};
+
+struct DecArgs {
+  int M, S, total, G;
+  DecLayer L[kMaxGroup];
   int32_t* status;
   uint32_t* gen;
   uint32_t* done;
   int pf_codes;           // prefetch this CTA's later code blocks into L2
-  int pf_tout;            // prefetch the T_out^T tiles of its synthesis tasks into L2
   int ext_in;             // bit p: phase p's input was written before the launch (no flags)
   const char* pf_next;    // a range to warm in L2 from the first synthesis task (next layer)
   int64_t pf_next_bytes;  // its length, a multiple of 16 (0: none)
@@ -125,9 +139,10 @@ struct DecArgs {
 // Per-cluster task lists, a kernel parameter: cluster c runs task[off[c]] .. task[off[c+1]-1].
 constexpr int kMaxClusters = 160;
 constexpr int kMaxSched = 3 * kWsMaxTiles;
+constexpr int kTileBits = 12;                  // row tiles per phase < 4096
 struct DecSched {
   uint16_t off[kMaxClusters + 1];
-  uint16_t task[kMaxSched];          // phase << 14 | row tile
+  uint16_t task[kMaxSched];          // layer << 14 | phase << 12 | row tile
 };
 
 template <int BN>
@@ -164,16 +179,17 @@ __device__ __forceinline__ uint4 ldcg_u4(const __nv_bfloat16* p) {
 }
 
 struct Task {
-  int p, tile;
+  int l, p, tile;
 };
 
-__device__ __forceinline__ DecPhase phase_of(const DecArgs& a, int p) {
-  return p == 0 ? a.ph[0] : (p == 1 ? a.ph[1] : a.ph[2]);
+__device__ __forceinline__ const DecPhase& phase_of(const DecArgs& a, int l, int p) {
+  return a.L[l].ph[p];
 }
 
 __device__ __forceinline__ Task task_at(const DecSched& sc, int ti) {
   const uint32_t e = sc.task[ti];
-  return {static_cast<int>(e >> 14), static_cast<int>(e & 0x3FFFu)};
+  return {static_cast<int>(e >> 14), static_cast<int>((e >> kTileBits) & 3u),
+          static_cast<int>(e & ((1u << kTileBits) - 1))};
 }
 
 // q -> bf16(4 + q) (exact: 4 .. 7 need 3 significant bits), one 128-byte row of a K-major tile
@@ -229,11 +245,7 @@ __device__ __forceinline__ void note_timeout(int32_t* status, int role, int task
 
 template <int BN>
 __global__ void __launch_bounds__(DecCfg<BN>::kThreads, 1)
-    decode_layer_kernel(const __grid_constant__ CUtensorMap tmTin,
-                        const __grid_constant__ CUtensorMap tmX,
-                        const __grid_constant__ CUtensorMap tmZ,
-                        const __grid_constant__ CUtensorMap tmTout,
-                        const __grid_constant__ CUtensorMap tmU, const DecArgs a,
+    decode_layer_kernel(const __grid_constant__ DecMaps maps, const __grid_constant__ DecArgs a,
                         const __grid_constant__ DecSched sched) {
   using Lo = DecLayout<BN>;
   constexpr int S_ = Lo::kStages;
@@ -295,12 +307,9 @@ __global__ void __launch_bounds__(DecCfg<BN>::kThreads, 1)
         for (int b = 0; b < 2; ++b)
           if (t_lo + b < t_hi) mbar_arrive_expect_tx(&recv_bar[b], bytes);
       }
-      prefetch_tmap(&tmTin);
-      prefetch_tmap(&tmX);
-      prefetch_tmap(&tmZ);
-      prefetch_tmap(&tmTout);
-      prefetch_tmap(&tmU);
     }
+    if (lane < a.G * kMapsPerLayer)
+      prefetch_tmap(&maps.m[lane / kMapsPerLayer][lane % kMapsPerLayer]);
   }
   if (warp == 1) tmem_alloc(tmem_slot, Lo::kTmemCols);
   tc_fence_before_sync();
@@ -325,7 +334,9 @@ __global__ void __launch_bounds__(DecCfg<BN>::kThreads, 1)
       const uint64_t pol_w = policy_evict_first();
       int stage = 0;
       uint32_t phase = 0;
-      bool first = true, tout_pf = a.pf_tout > 0, next_pf = a.pf_next_bytes > 0;
+      bool tout_pf = false;
+      for (int l = 0; l < a.G; ++l) tout_pf |= a.L[l].pf_tout > 0;
+      bool first = true, next_pf = a.pf_next_bytes > 0;
       // this CTA's share of the next layer's range, into L2 (64 KiB per prefetch)
       auto prefetch_next = [&]() {
         next_pf = false;
@@ -345,23 +356,24 @@ __global__ void __launch_bounds__(DecCfg<BN>::kThreads, 1)
       for (int i = t_lo; i < t_hi && wok; ++i) {
         if (__any_sync(0xffffffffu, *abort_flag != 0)) break;
         const Task t = task_at(sched, i);
-        const DecPhase ph = phase_of(a, t.p);
+        const DecPhase& ph = phase_of(a, t.l, t.p);
         int k0, k1;
         krange(ph, k0, k1);
         if (next_pf && t.p == 2) prefetch_next();
         if (tout_pf && t.p >= 1) {
           tout_pf = false;
-          // this CTA's synthesis tiles, in the order they will be read, into L2
+          // this CTA's synthesis tiles of the layers warmed in L2, in the order they will be
+          // read, into L2
           for (int j = i; j < t_hi && lane == 0; ++j) {
             const Task u = task_at(sched, j);
-            if (u.p != 2) continue;
-            const DecPhase q = phase_of(a, u.p);
+            if (u.p != 2 || !a.L[u.l].pf_tout) continue;
+            const DecPhase& q = phase_of(a, u.l, u.p);
             int u0, u1;
             krange(q, u0, u1);
             for (int kb = u0; kb < u1; ++kb)
               asm volatile(
                   "cp.async.bulk.prefetch.tensor.2d.L2.global.tile [%0, {%1, %2}];" ::"l"(
-                      reinterpret_cast<uint64_t>(&tmTout)),
+                      reinterpret_cast<uint64_t>(&maps.m[u.l][kMapTout])),
                   "r"(kb * kBK), "r"(u.tile * kBM)
                   : "memory");
           }
@@ -382,8 +394,8 @@ __global__ void __launch_bounds__(DecCfg<BN>::kThreads, 1)
             if (lane == 0) {
               mbar_arrive_expect_tx(&cfull[stage], kCodeBytes);
               bulk_load(sC + stage * kCodeBytes,
-                        a.words + (static_cast<int64_t>(t.tile) * ph.KB + kb) * 512, kCodeBytes,
-                        &cfull[stage], pol_w);
+                        a.L[t.l].words + (static_cast<int64_t>(t.tile) * ph.KB + kb) * 512,
+                        kCodeBytes, &cfull[stage], pol_w);
             }
             last_code |= bit;
             last_par = (last_par & ~bit) | (cpar & bit);
@@ -391,8 +403,8 @@ __global__ void __launch_bounds__(DecCfg<BN>::kThreads, 1)
           } else {
             if (lane == 0) {
               mbar_arrive_expect_tx(&fullA[stage], kATile);
-              tma_load_2d(sA + stage * kATile, t.p == 0 ? &tmTin : &tmTout, &fullA[stage],
-                          kb * kBK, t.tile * kBM, pol_w);
+              tma_load_2d(sA + stage * kATile, &maps.m[t.l][t.p == 0 ? kMapTin : kMapTout],
+                          &fullA[stage], kb * kBK, t.tile * kBM, pol_w);
             }
             last_code &= ~bit;
             last_par = (last_par & ~bit) | (phase << stage);
@@ -404,11 +416,12 @@ __global__ void __launch_bounds__(DecCfg<BN>::kThreads, 1)
           // warm L2 with the code blocks of this CTA's later tasks
           for (int j = i + 1; j < t_hi && a.pf_codes && lane == 0; ++j) {
             const Task u = task_at(sched, j);
-            const DecPhase q = phase_of(a, u.p);
+            const DecPhase& q = phase_of(a, u.l, u.p);
             int u0, u1;
             krange(q, u0, u1);
             if (u.p == 1 && u1 > u0) {
-              const uint32_t* src = a.words + (static_cast<int64_t>(u.tile) * q.KB + u0) * 512;
+              const uint32_t* src =
+                  a.L[u.l].words + (static_cast<int64_t>(u.tile) * q.KB + u0) * 512;
               asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(src),
                            "r"(static_cast<uint32_t>((u1 - u0) * kCodeBytes))
                            : "memory");
@@ -445,19 +458,19 @@ __global__ void __launch_bounds__(DecCfg<BN>::kThreads, 1)
     for (int i = t_lo; i < t_hi; ++i) {
       if (__shfl_sync(0xffffffffu, *abort_flag != 0, 0)) break;   // warp-uniform
       const Task t = task_at(sched, i);
-      const DecPhase ph = phase_of(a, t.p);
+      const DecPhase& ph = phase_of(a, t.l, t.p);
       int k0, k1;
       krange(ph, k0, k1);
       // Loads go out in K order as soon as the slices of the previous phase's output that a K
       // block reads are final: the lanes poll the not-yet-final slices of the K range, and
       // the ready prefix decides how far lane 0 may issue.
-      const DecPhase src = phase_of(a, t.p > 0 ? t.p - 1 : 0);
+      const DecPhase& src = phase_of(a, t.l, t.p > 0 ? t.p - 1 : 0);
       const int sl1 = k1 > k0 ? (min(ph.K, k1 * kBK) - 1) / rows_per : 0;
       int ready = k1 > k0 ? (k0 * kBK) / rows_per : 0;   // slices below `ready` are final
       const long long t_start = clock64();
       bool ok = true;
       int kb = k0;
-      const CUtensorMap* tm = t.p == 0 ? &tmX : (t.p == 1 ? &tmZ : &tmU);
+      const CUtensorMap* tm = &maps.m[t.l][t.p == 0 ? kMapX : (t.p == 1 ? kMapZ : kMapU)];
       while (kb < k1 && ok) {
         int kb_end = k1;
         if (t.p > 0 && !((a.ext_in >> t.p) & 1) && ready <= sl1) {
@@ -525,7 +538,7 @@ __global__ void __launch_bounds__(DecCfg<BN>::kThreads, 1)
       bool issued_any = false;
       for (int i = t_lo; i < t_hi && !*abort_flag; ++i) {
         const Task t = task_at(sched, i);
-        const DecPhase ph = phase_of(a, t.p);
+        const DecPhase& ph = phase_of(a, t.l, t.p);
         int k0, k1;
         krange(ph, k0, k1);
         if (!mbar_wait(&tempty[buf], acc_phase ^ 1, abort_flag)) {
@@ -582,7 +595,7 @@ __global__ void __launch_bounds__(DecCfg<BN>::kThreads, 1)
     for (int i = t_lo; i < t_hi && ok; ++i) {
       if (__shfl_sync(0xffffffffu, *abort_flag != 0, 0)) break;   // warp-uniform
       const Task t = task_at(sched, i);
-      const DecPhase ph = phase_of(a, t.p);
+      const DecPhase& ph = phase_of(a, t.l, t.p);
       int k0, k1;
       krange(ph, k0, k1);
       const int n = max(0, k1 - k0);
@@ -636,7 +649,8 @@ __global__ void __launch_bounds__(DecCfg<BN>::kThreads, 1)
     int j = 0;                                    // tasks finished by this CTA
     for (int i = t_lo; i < t_hi; ++i, ++j) {
       const Task t = task_at(sched, i);
-      const DecPhase ph = phase_of(a, t.p);
+      const DecLayer& Ly = a.L[t.l];
+      const DecPhase& ph = Ly.ph[t.p];
       int k0, k1;
       krange(ph, k0, k1);
       const bool has_k = k1 > k0;
@@ -644,9 +658,9 @@ __global__ void __launch_bounds__(DecCfg<BN>::kThreads, 1)
       const bool row_ok = row < ph.R;
       float s_i = 0.f, z_i = 0.f, g_row = 1.f;
       if (t.p == 1 && row_ok) {
-        s_i = __half2float(a.scale[row]);
-        z_i = __half2float(a.zero[row]);
-        if (a.gamma) g_row = a.gamma[row];
+        s_i = __half2float(Ly.scale[row]);
+        z_i = __half2float(Ly.zero[row]);
+        if (Ly.gamma) g_row = Ly.gamma[row];
       }
       const float zb_i = z_i - 4.f * s_i;          // the decoded codes carry an offset of 4
       bool fail = false;
@@ -655,7 +669,7 @@ __global__ void __launch_bounds__(DecCfg<BN>::kThreads, 1)
         if (has_k && !(a.ext_in & 2)) {
           const int sl0 = (k0 * kBK) / rows_per, sl1 = (min(ph.K, k1 * kBK) - 1) / rows_per;
           for (int gs = sl0 + et; gs <= sl1 && !fail; gs += kEpi) {
-            fail = !wait_flag(&a.ph[0].flags[(gs / S) * kWsSlices + gs % S], g, abort_flag);
+            fail = !wait_flag(&Ly.ph[0].flags[(gs / S) * kWsSlices + gs % S], g, abort_flag);
             if (fail && !*abort_flag) note_timeout(a.status, 8, i, gs, 0);
           }
         }
@@ -673,7 +687,7 @@ __global__ void __launch_bounds__(DecCfg<BN>::kThreads, 1)
             // z columns k0 * 64 .. of token q: multiples of 8 (n_in is a multiple of 16), so
             // 16-byte loads from L2, each thread a strided share
             const int c0 = k0 * kBK, c1 = min(ph.K, k1 * kBK);
-            const __nv_bfloat16* zr = a.ph[0].out + static_cast<int64_t>(q) * ph.K;
+            const __nv_bfloat16* zr = Ly.ph[0].out + static_cast<int64_t>(q) * ph.K;
             for (int c = c0 + 8 * part; c < c1; c += 8 * kPer) {
               const uint4 w = ldcg_u4(zr + c);
               const uint32_t wv[4] = {w.x, w.y, w.z, w.w};
@@ -922,31 +936,52 @@ int max_clusters(int dev, int S) {
   return n;
 }
 
-// Task lists for `ncl` clusters of S CTAs: the three phases' tiles, concatenated in phase order,
-// dealt round-robin (each phase spreads evenly and starts on the clusters the previous one
-// left least busy).  Within the analysis and the core phase, tiles are ordered by their offset
-// inside the next phase's K splits, so that every split of the next phase finds its first K
-// blocks among the first tiles produced.
-void build_schedule(const int* R, const int* K, int S, int ncl, DecSched* out) {
-  int RT[3], kbs[3];
-  for (int p = 0; p < 3; ++p) {
-    RT[p] = static_cast<int>(ceil_div(R[p], kBM));
-    kbs[p] = static_cast<int>(ceil_div(ceil_div(K[p], kBK), S));
-  }
+// One phase of one layer of a launch: rows R of its output, reduction length K, and the K of
+// the layer's next phase (0 if none), whose splits its tiles are ordered by.
+struct Block {
+  int l, p, R, K, K_next;
+};
+
+// Launch order of the (layer, phase) blocks.  A single layer runs its three phases in order.  A
+// group runs them along diagonals, block (l, p) at position l + p and lower phases first:
+//     A0 A1 C0 A2 C1 S0 C2 S1 S2   (three layers; A analysis, C code product, S synthesis),
+// so that each layer's phase boundaries have another layer's streaming behind them, and every
+// block still comes after the block it reads (same layer, previous phase).
+std::vector<Block> launch_order(int G, const int (*R)[3], const int (*K)[3]) {
+  std::vector<Block> v;
+  for (int l = 0; l < G; ++l)
+    for (int p = 0; p < 3; ++p)
+      if (R[l][p] > 0) v.push_back({l, p, R[l][p], K[l][p], p < 2 ? K[l][p + 1] : 0});
+  std::stable_sort(v.begin(), v.end(), [](const Block& x, const Block& y) {
+    return x.l + x.p != y.l + y.p ? x.l + x.p < y.l + y.p : x.p < y.p;
+  });
+  return v;
+}
+
+// Task lists for `ncl` clusters of S CTAs: the blocks' tiles, concatenated in launch order, dealt
+// round-robin (each block spreads evenly and starts on the clusters the previous one left least
+// busy).  Within a block whose layer has a next phase, tiles are ordered by their offset inside
+// that phase's K splits, so that every split of the next phase finds its first K blocks among
+// the first tiles produced.
+void build_schedule(const std::vector<Block>& blocks, int S, int ncl, DecSched* out) {
   std::vector<std::vector<uint16_t>> lists(ncl);
   std::vector<int> order;
   int pos = 0;
-  for (int p = 0; p < 3; ++p) {
-    order.resize(RT[p]);
-    for (int t = 0; t < RT[p]; ++t) order[t] = t;
-    if (p < 2 && kbs[p + 1] > 0) {
-      const int64_t split_rows = static_cast<int64_t>(kbs[p + 1]) * kBK;
+  for (const Block& b : blocks) {
+    const int RT = static_cast<int>(ceil_div(b.R, kBM));
+    order.resize(RT);
+    for (int t = 0; t < RT; ++t) order[t] = t;
+    const int kbs_next = static_cast<int>(ceil_div(ceil_div(b.K_next, kBK), S));
+    if (kbs_next > 0) {
+      const int64_t split_rows = static_cast<int64_t>(kbs_next) * kBK;
       std::stable_sort(order.begin(), order.end(), [&](int x, int y) {
         return (static_cast<int64_t>(x) * kBM) % split_rows <
                (static_cast<int64_t>(y) * kBM) % split_rows;
       });
     }
-    for (int t : order) lists[pos++ % ncl].push_back(static_cast<uint16_t>((p << 14) | t));
+    for (int t : order)
+      lists[pos++ % ncl].push_back(
+          static_cast<uint16_t>((b.l << 14) | (b.p << kTileBits) | t));
   }
   int n = 0;
   for (int c = 0; c < ncl; ++c) {
@@ -961,19 +996,20 @@ struct Plan {
   DecSched sched{};
 };
 
-// Cluster size and task lists for a layer shape, cached.  Cluster size: the busiest cluster's
-// K blocks over the three phases, with a fixed cost per task (pipeline fill and drain,
+// Cluster size and task lists for a launch's blocks, cached.  Cluster size: the busiest
+// cluster's K blocks over the blocks, with a fixed cost per task (pipeline fill and drain,
 // reduction) and code blocks weighted by their smaller bytes.
 template <int BN>
-const Plan* plan_for(int dev, int sms, int budget, const int* R, const int* K) {
+const Plan* plan_for(int dev, int sms, int budget, const std::vector<Block>& blocks) {
   static std::mutex mu;
-  static std::map<std::array<int, 8>, Plan> cache;
-  const std::array<int, 8> key{dev, R[0], R[1], R[2], K[0], K[1], K[2], budget};
+  static std::map<std::vector<int>, Plan> cache;
+  std::vector<int> key{dev, budget};
+  for (const Block& b : blocks) key.insert(key.end(), {b.l, b.p, b.R, b.K, b.K_next});
   std::lock_guard<std::mutex> g(mu);
   const auto it = cache.find(key);
   if (it != cache.end()) return &it->second;
   int total = 0;
-  for (int p = 0; p < 3; ++p) total += static_cast<int>(ceil_div(R[p], kBM));
+  for (const Block& b : blocks) total += static_cast<int>(ceil_div(b.R, kBM));
   Plan best;
   double best_cost = 1e30;
   for (int S : {1, 2, 4, 8}) {
@@ -987,10 +1023,10 @@ const Plan* plan_for(int dev, int sms, int budget, const int* R, const int* K) {
     ncl = std::min({ncl, total, kMaxClusters});
     if (ncl <= 0) continue;
     double cost = 0;
-    for (int p = 0; p < 3; ++p) {
-      const int RT = static_cast<int>(ceil_div(R[p], kBM));
-      const int KB = static_cast<int>(ceil_div(K[p], kBK));
-      const double w = p == 1 ? 0.35 : 1.0;
+    for (const Block& b : blocks) {
+      const int RT = static_cast<int>(ceil_div(b.R, kBM));
+      const int KB = static_cast<int>(ceil_div(b.K, kBK));
+      const double w = b.p == 1 ? 0.35 : 1.0;
       cost += static_cast<double>(ceil_div(RT, ncl)) * (w * ceil_div(KB, S) + 4.0);
     }
     if (cost < best_cost - 1e-9) {
@@ -1000,41 +1036,49 @@ const Plan* plan_for(int dev, int sms, int budget, const int* R, const int* K) {
     }
   }
   if (best.S == 0) return nullptr;
-  build_schedule(R, K, best.S, best.ncl, &best.sched);
+  build_schedule(blocks, best.S, best.ncl, &best.sched);
   return &(cache[key] = best);
 }
 
 template <int BN>
-fq_status run(const CUtensorMap* m, DecArgs& a, const int* R, const int* K, int sms,
+fq_status run(const DecMaps& maps, DecArgs& a, const std::vector<Block>& blocks, int sms,
               int budget, cudaStream_t s) {
   int dev = 0;
   cudaGetDevice(&dev);
   if (prepare<BN>(dev) != cudaSuccess) return FQ_ERR_CUDA;
   int total = 0;
-  for (int p = 0; p < 3; ++p) {
-    const int RT = static_cast<int>(ceil_div(R[p], kBM));
-    if (RT > kWsMaxTiles || RT > 0x3FFF) return FQ_ERR_UNSUPPORTED;
-    total += RT;
-  }
+  for (const Block& b : blocks) total += static_cast<int>(ceil_div(b.R, kBM));
   if (total > kMaxSched) return FQ_ERR_UNSUPPORTED;
-  const Plan* plan = plan_for<BN>(dev, sms, budget, R, K);
+  const Plan* plan = plan_for<BN>(dev, sms, budget, blocks);
   if (!plan) return FQ_ERR_CUDA;
   a.S = plan->S;
-  for (int p = 0; p < 3; ++p) {
-    DecPhase& ph = a.ph[p];
-    ph.RT = static_cast<int>(ceil_div(R[p], kBM));
-    ph.KB = static_cast<int>(ceil_div(K[p], kBK));
-    ph.kbs = static_cast<int>(ceil_div(ph.KB, plan->S));
-  }
+  for (int l = 0; l < a.G; ++l)
+    for (int p = 0; p < 3; ++p) {
+      DecPhase& ph = a.L[l].ph[p];
+      ph.RT = static_cast<int>(ceil_div(ph.R, kBM));
+      ph.KB = static_cast<int>(ceil_div(ph.K, kBK));
+      ph.kbs = static_cast<int>(ceil_div(ph.KB, plan->S));
+    }
   a.total = total;
   {
-    const int64_t code_bytes = static_cast<int64_t>(R[1]) * K[1] / 4;
-    const int64_t tout_bytes = static_cast<int64_t>(R[2]) * K[2] * 2;
+    // L2 warming within one budget for the whole launch: the code blocks of every layer, then
+    // the T_out^T of as many layers (in order) as fit with them
+    int64_t code_bytes = 0;
+    for (int l = 0; l < a.G; ++l)
+      code_bytes += static_cast<int64_t>(a.L[l].ph[1].R) * a.L[l].ph[1].K / 4;
     a.pf_codes = code_bytes <= kL2PrefetchBudget;
-    a.pf_tout = code_bytes + tout_bytes <= kL2PrefetchBudget;
-    // the next layer's range only when this synthesis reads from L2 (HBM idle), and at most
-    // the warming budget
-    a.pf_next_bytes = a.pf_tout ? std::min<int64_t>(a.pf_next_bytes, kL2PrefetchBudget) : 0;
+    int64_t warm = code_bytes;
+    bool any_tout = false;
+    for (int l = 0; l < a.G; ++l) {
+      warm += static_cast<int64_t>(a.L[l].ph[2].R) * a.L[l].ph[2].K * 2;
+      a.L[l].pf_tout = a.L[l].ph[2].R > 0 && warm <= kL2PrefetchBudget;
+      any_tout |= a.L[l].pf_tout != 0;
+    }
+    // the next layer's range only when this launch's last synthesis reads from L2 (HBM idle),
+    // and at most the warming budget
+    a.pf_next_bytes = any_tout && a.L[a.G - 1].pf_tout
+                          ? std::min<int64_t>(a.pf_next_bytes, kL2PrefetchBudget)
+                          : 0;
   }
   cudaLaunchConfig_t cfg{};
   cfg.gridDim = dim3(static_cast<unsigned>(plan->ncl * plan->S));
@@ -1050,10 +1094,27 @@ fq_status run(const CUtensorMap* m, DecArgs& a, const int* R, const int* K, int 
   attr[1].val.clusterDim.z = 1;
   cfg.attrs = attr;
   cfg.numAttrs = plan->S > 1 ? 2 : 1;
-  return cudaLaunchKernelEx(&cfg, decode_layer_kernel<BN>, m[0], m[1], m[2], m[3], m[4], a,
-                            plan->sched) == cudaSuccess
+  return cudaLaunchKernelEx(&cfg, decode_layer_kernel<BN>, maps, a, plan->sched) == cudaSuccess
              ? FQ_OK
              : FQ_ERR_CUDA;
+}
+
+// Workspace of a launch: the 64 KiB header, then z and u of every layer.
+struct DecWsGroup {
+  size_t z[kMaxGroup], u[kMaxGroup], total;
+};
+
+DecWsGroup dec_ws_group(int M, int G, const DecGroupLayer* Ls) {
+  DecWsGroup W{};
+  size_t off = kWsHeader;
+  for (int l = 0; l < G; ++l) {
+    W.z[l] = off;
+    off += round_up(static_cast<int64_t>(M) * Ls[l].C.n_in * 2, 256);
+    W.u[l] = off;
+    off += round_up(static_cast<int64_t>(M) * Ls[l].C.n_out * 2, 256);
+  }
+  W.total = off;
+  return W;
 }
 
 }  // namespace
@@ -1064,39 +1125,85 @@ size_t decode_workspace_bytes(int M, int d_in, int n_in, int n_out, int d_out) {
   return dec_ws(M, n_in, n_out).total;
 }
 
-namespace {
+size_t decode_group_workspace_bytes(int M, int G, const DecGroupLayer* layers) {
+  if (G < 1 || G > kMaxGroup) return 0;
+  return dec_ws_group(M, G, layers).total;
+}
 
-// The fused kernel over all three phases, or (core_only) over the code product alone with z
-// already in the workspace and u left there.
-fq_status launch_decode(const void* x, int M, int d_in, const void* T_in, const fq_packed& Cq,
-                        const void* T_out_t, int d_out, const float* gamma, void* y, char* ws,
-                        size_t ws_bytes, int max_sms, bool core_only, const void* pf,
-                        size_t pf_bytes, int64_t inject_wait, cudaStream_t s) {
-  const int n_in = Cq.n_in, n_out = Cq.n_out;
-  const DecWs L = dec_ws(M, n_in, n_out);
-  if (ws_bytes < L.total) return FQ_ERR_WORKSPACE;
+// The fused kernel over a group of G independent layers (G = 1: one layer), or (core_only,
+// G = 1) over the code product alone with z already in the workspace and u left there.
+fq_status launch_decode_group(int M, int G, const DecGroupLayer* Ls, char* ws, size_t ws_bytes,
+                              int max_sms, bool core_only, const void* pf, size_t pf_bytes,
+                              int64_t inject_wait, cudaStream_t s) {
+  if (G < 1 || G > kMaxGroup || (core_only && G != 1)) return FQ_ERR_INVALID_ARG;
+  const DecWsGroup W = dec_ws_group(M, G, Ls);
+  if (ws_bytes < W.total) return FQ_ERR_WORKSPACE;
   const int BN = decode_bn(M);
   int dev = 0, sms = 0;
   cudaGetDevice(&dev);
   cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
   if (sms <= 0) return FQ_ERR_CUDA;
   const int budget = max_sms > 0 ? std::min(sms, max_sms) : sms;
+  if (inject_wait > 0 && budget != 1) return FQ_ERR_INVALID_ARG;   // one CTA, no cluster peers
 
   DecArgs a{};
   a.M = M;
-  const int R[3] = {core_only ? 0 : n_in, n_out, core_only ? 0 : d_out};
-  const int K[3] = {core_only ? 0 : d_in, n_in, core_only ? 0 : n_out};
-  void* outs[3] = {ws + L.z, ws + L.u, core_only ? static_cast<void*>(ws + L.u) : y};
-  for (int p = 0; p < 3; ++p) {
-    a.ph[p].R = R[p];
-    a.ph[p].K = K[p];
-    a.ph[p].out = static_cast<__nv_bfloat16*>(outs[p]);
-    a.ph[p].flags = reinterpret_cast<uint32_t*>(ws + kWsFlags) + p * kWsMaxTiles * kWsSlices;
+  a.G = G;
+  int R[kMaxGroup][3], K[kMaxGroup][3];
+  uint32_t* flag_base = reinterpret_cast<uint32_t*>(ws + kWsFlags);
+  const int64_t flag_words = static_cast<int64_t>(kWsHeader - kWsFlags) / 4;
+  int64_t flag_off = 0;
+  DecMaps maps;
+  for (int l = 0; l < G; ++l) {
+    const DecGroupLayer& Ly = Ls[l];
+    const int n_in = Ly.C.n_in, n_out = Ly.C.n_out;
+    const int Rl[3] = {core_only ? 0 : n_in, n_out, core_only ? 0 : Ly.d_out};
+    const int Kl[3] = {core_only ? 0 : Ly.d_in, n_in, core_only ? 0 : n_out};
+    void* outs[3] = {ws + W.z[l], ws + W.u[l], core_only ? static_cast<void*>(ws + W.u[l]) : Ly.y};
+    for (int p = 0; p < 3; ++p) {
+      R[l][p] = Rl[p];
+      K[l][p] = Kl[p];
+      const int RT = static_cast<int>(ceil_div(Rl[p], kBM));
+      if (RT > kWsMaxTiles || RT >= (1 << kTileBits)) return FQ_ERR_UNSUPPORTED;
+      DecPhase& ph = a.L[l].ph[p];
+      ph.R = Rl[p];
+      ph.K = Kl[p];
+      ph.out = static_cast<__nv_bfloat16*>(outs[p]);
+      if (G == 1) {
+        // one layer: the phases' flags at fixed places of the header
+        ph.flags = flag_base + p * kWsMaxTiles * kWsSlices;
+      } else if (p < 2) {
+        // a group: the flags of the analysis and code-product slices, packed in layer order
+        // (the synthesis publishes none); every flag of the header only ever holds a past
+        // generation, whichever layout wrote it
+        ph.flags = flag_base + flag_off;
+        flag_off += static_cast<int64_t>(RT) * kWsSlices;
+        if (flag_off > flag_words) return FQ_ERR_UNSUPPORTED;
+      } else {
+        ph.flags = flag_base;
+      }
+    }
+    a.L[l].words = Ly.C.words;
+    a.L[l].scale = reinterpret_cast<const __half*>(Ly.C.scale_f16);
+    a.L[l].zero = reinterpret_cast<const __half*>(Ly.C.zero_f16);
+    a.L[l].gamma = Ly.gamma;
+    CUtensorMap* m = maps.m[l];
+    if (!tmap_bf16(&m[kMapZ], ws + W.z[l], M, n_in, BN) ||
+        !tmap_bf16(&m[kMapU], ws + W.u[l], M, n_out, BN))
+      return FQ_ERR_CUDA;
+    if (core_only) {
+      // no analysis or synthesis tasks: their maps are never used for a copy
+      m[kMapTin] = m[kMapZ];
+      m[kMapX] = m[kMapZ];
+      m[kMapTout] = m[kMapU];
+    } else if (!tmap_bf16(&m[kMapTin], Ly.T_in, n_in, Ly.d_in, kBM) ||
+               !tmap_bf16(&m[kMapX], Ly.x, M, Ly.d_in, BN) ||
+               !tmap_bf16(&m[kMapTout], Ly.T_out_t, Ly.d_out, n_out, kBM)) {
+      return FQ_ERR_CUDA;
+    }
   }
-  a.words = Cq.words;
-  a.scale = reinterpret_cast<const __half*>(Cq.scale_f16);
-  a.zero = reinterpret_cast<const __half*>(Cq.zero_f16);
-  a.gamma = gamma;
+  for (int l = G; l < kMaxGroup; ++l)
+    for (int k = 0; k < kMapsPerLayer; ++k) maps.m[l][k] = maps.m[0][k];
   a.status = reinterpret_cast<int32_t*>(ws);
   a.gen = reinterpret_cast<uint32_t*>(ws + kWsGen);
   a.done = reinterpret_cast<uint32_t*>(ws + kWsDone);
@@ -1104,42 +1211,28 @@ fq_status launch_decode(const void* x, int M, int d_in, const void* T_in, const 
   a.pf_next = static_cast<const char*>(pf);
   a.pf_next_bytes = pf ? static_cast<int64_t>(pf_bytes) : 0;
   a.inject_wait = inject_wait;
-
-  CUtensorMap m[5];
-  if (!tmap_bf16(&m[2], ws + L.z, M, n_in, BN) || !tmap_bf16(&m[4], ws + L.u, M, n_out, BN))
-    return FQ_ERR_CUDA;
-  if (core_only) {
-    // no analysis or synthesis tasks: their maps are never used for a copy
-    m[0] = m[2];
-    m[1] = m[2];
-    m[3] = m[4];
-  } else if (!tmap_bf16(&m[0], T_in, n_in, d_in, kBM) || !tmap_bf16(&m[1], x, M, d_in, BN) ||
-             !tmap_bf16(&m[3], T_out_t, d_out, n_out, kBM)) {
-    return FQ_ERR_CUDA;
-  }
-  if (inject_wait > 0 && budget != 1) return FQ_ERR_INVALID_ARG;   // one CTA, no cluster peers
+  const std::vector<Block> blocks = launch_order(G, R, K);
   switch (BN) {
-    case 16: return run<16>(m, a, R, K, sms, budget, s);
-    case 32: return run<32>(m, a, R, K, sms, budget, s);
-    default: return run<64>(m, a, R, K, sms, budget, s);
+    case 16: return run<16>(maps, a, blocks, sms, budget, s);
+    case 32: return run<32>(maps, a, blocks, sms, budget, s);
+    default: return run<64>(maps, a, blocks, sms, budget, s);
   }
 }
-
-}  // namespace
 
 fq_status launch_decode_forward(const void* x, int M, int d_in, const void* T_in,
                                 const fq_packed& Cq, const void* T_out_t, int d_out,
                                 const float* gamma, void* y, char* ws, size_t ws_bytes,
                                 int max_sms, const void* pf, size_t pf_bytes,
                                 int64_t inject_wait, cudaStream_t s) {
-  return launch_decode(x, M, d_in, T_in, Cq, T_out_t, d_out, gamma, y, ws, ws_bytes, max_sms,
-                       false, pf, pf_bytes, inject_wait, s);
+  const DecGroupLayer L{x, d_in, T_in, Cq, T_out_t, d_out, gamma, y};
+  return launch_decode_group(M, 1, &L, ws, ws_bytes, max_sms, false, pf, pf_bytes, inject_wait,
+                             s);
 }
 
 fq_status launch_decode_core(int M, const fq_packed& Cq, const float* gamma, char* ws,
                              size_t ws_bytes, int max_sms, cudaStream_t s) {
-  return launch_decode(nullptr, M, 0, nullptr, Cq, nullptr, 0, gamma, nullptr, ws, ws_bytes,
-                       max_sms, true, nullptr, 0, 0, s);
+  const DecGroupLayer L{nullptr, 0, nullptr, Cq, nullptr, 0, gamma, nullptr};
+  return launch_decode_group(M, 1, &L, ws, ws_bytes, max_sms, true, nullptr, 0, 0, s);
 }
 
 size_t decode_core_z_offset() { return kWsHeader; }

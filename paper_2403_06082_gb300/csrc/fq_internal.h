@@ -63,6 +63,24 @@ fq_status launch_decode_forward(const void* x, int M, int d_in, const void* T_in
                                 int max_sms, const void* pf, size_t pf_bytes,
                                 int64_t inject_wait, cudaStream_t s);
 
+// One layer of a fused launch over independent layers (the M <= 64 kernel).
+struct DecGroupLayer {
+  const void* x;
+  int d_in;
+  const void* T_in;
+  fq_packed C;
+  const void* T_out_t;
+  int d_out;
+  const float* gamma;
+  void* y;
+};
+// Workspace of a launch over G layers (header, then z and u of each layer); 0 for G out of range.
+size_t decode_group_workspace_bytes(int M, int G, const DecGroupLayer* layers);
+// The fused kernel over G <= 4 independent layers; arguments checked by the caller.
+fq_status launch_decode_group(int M, int G, const DecGroupLayer* layers, char* ws,
+                              size_t ws_bytes, int max_sms, bool core_only, const void* pf,
+                              size_t pf_bytes, int64_t inject_wait, cudaStream_t s);
+
 // The code product alone (z already in the workspace at decode_core_z_offset(), u left at
 // decode_core_u_offset()), for the structured-frame forward.
 fq_status launch_decode_core(int M, const fq_packed& C, const float* gamma, char* ws,

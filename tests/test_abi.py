@@ -226,3 +226,37 @@ def test_dense_path_sizes_and_validation_without_gpu(L):
     assert L.fq_dense_forward(None, 8, 256, 0x2000, 256, 0x4000, 0x10000, 1 << 30, None) == 1
     assert L.fq_dense_forward(0x1000, 8, 260, 0x2000, 256, 0x4000, 0x10000, 1 << 30, None) == 2
     assert L.fq_dense_forward(0x1000, 8, 256, 0x2000, 256, 0x4000, 0x10000, 64, None) == 4
+
+
+def test_group_sizes_and_validation_without_gpu(L):
+    C = _P(0x5000, 0x6000, 0x7000, 4512, 4512)
+    Cg = _P(0x5000, 0x6000, 0x7000, 12112, 4512)
+
+    def layer(x=0x1000, y=0x4000, C=C, d_out=4096):
+        return fq._Layer(x, 4096, 0x2000, ctypes.pointer(C), 0x3000, d_out, None, y)
+
+    def arr(*ls):
+        a = (fq._Layer * len(ls))()
+        for i, l_ in enumerate(ls):
+            a[i] = l_
+        return a
+    one = fq.fq_workspace_bytes(16, 4096, 4512, 4512, 4096)
+    g3 = L.fq_group_workspace_bytes(16, 3, arr(layer(), layer(y=0x8000), layer(y=0x9000)))
+    # the header once, then z and u of every layer
+    assert g3 == one + 2 * (one - 64 * 1024)
+    assert L.fq_group_workspace_bytes(16, 0, arr(layer())) == 0
+    assert L.fq_group_workspace_bytes(16, 5, arr(*[layer()] * 5)) == 0
+    # larger batches run the layers in turn: the largest single workspace
+    big = L.fq_group_workspace_bytes(300, 2, arr(layer(), layer(y=0x8000, C=Cg, d_out=11008)))
+    assert big == max(fq.fq_workspace_bytes(300, 4096, 4512, 4512, 4096),
+                      fq.fq_workspace_bytes(300, 4096, 4512, 12112, 11008))
+
+    def fwd(a, n, ws=0x10000, nb=1 << 30, opts=None):
+        return L.fq_linear_forward_group(16, n, a, ws, nb, ctypes.byref(opts) if opts else None,
+                                         None)
+    assert fwd(arr(layer(), layer()), 2) == 1                       # same output twice
+    assert fwd(arr(layer(), layer(x=0x4000, y=0x8000)), 2) == 1     # an output is an input
+    assert fwd(arr(layer(x=0x1002)), 1) == 2
+    assert fwd(arr(layer()), 1, ws=0x10010) == 2
+    assert fwd(arr(layer()), 1, nb=1024) == 4
+    assert fwd(arr(layer()), 1, opts=fq._Opts(1, None, 0, 1000)) == 1   # no timeout hook

@@ -41,6 +41,21 @@ def test_reconstructed_weight(wl_key, name, use_gamma):
     err = assert_parity(W.double().cpu().numpy(), _oracle_w_hat(L, use_gamma), 1e-2)
 
 
+@pytest.mark.parametrize("name,use_gamma", [("q", False), ("gate", True)])
+def test_reconstructed_weight_llama7b_sampled_rows(name, use_gamma):
+    """The 7B shapes (4096 x 4096 and 11008 x 4096 at r = 1.1): the whole W_hat is rebuilt on
+    the GPU; the oracle computes 64 seeded rows of T_out^T diag(gamma) C_hat T_in."""
+    import workloads as wl
+    L = oracle_layer("llama2_7b_prefill", name)
+    W = _w_hat(L, DeviceLayer(L, BF16), use_gamma).double().cpu().numpy()
+    rows = np.sort(wl.rng(3, "w-hat-rows", name).choice(L.d_out, 64, replace=False))
+    C_hat = quant.dequantize(L.codes, L.scale, L.zero)
+    if use_gamma:
+        C_hat = C_hat * L.gamma.astype(np.float64)[:, None]
+    ref = (L.T_out.T[rows] @ C_hat) @ L.T_in
+    assert_parity(W[rows], ref, 1e-2)
+
+
 @pytest.mark.parametrize("M", [1, 8, 100, 300])
 def test_dense_forward_matches_the_layer(M):
     L = oracle_layer("single256", "single")

@@ -56,9 +56,11 @@ def real_codes(name, r):
     W = wl.weight(WK, layer)
     WT = frames.analysis_apply(k_in, RHO, layer.d_in, draws_in, W)          # W T_in^T
     del W
-    C = frames.analysis_apply(k_out, RHO, layer.d_out, draws_out, WT.T).T    # T_out W T_in^T
+    C = np.ascontiguousarray(
+        frames.analysis_apply(k_out, RHO, layer.d_out, draws_out, WT.T).T)   # T_out W T_in^T
     del WT
-    return quant.rtn(C)
+    codes, scale, zero = quant.rtn(C)
+    return np.ascontiguousarray(codes), scale, zero
 
 
 def run_layer(name, r, M, dtype=torch.bfloat16, codes_from_w=False):
