@@ -10,6 +10,7 @@ it and shares no code with it; the two meet only in the seeded input generators 
   forward  analysis -> dequantized product -> synthesis (Sec. 3.2)
   layer    one call that builds a whole quantized layer from a workload
   gptq     the frame-domain GPTQ quantizer of Algorithm 1, step 4 (calibration Hessian)
+  actquant rounding the frame representation of the activations to N-bit integers (App. F)
 
 Parity status: every function is pinned by tests/test_oracle_*.py against brute force, closed
 forms, printed examples or special cases; the de-noising gain (which the paper does not print) is
