@@ -202,10 +202,6 @@ class Regime:
         self.groups = [[by[n] for n in names] for names in GROUPS if all(n in by for n in names)]
         ws_bytes = max(fq.fq_workspace_bytes(M, L["d_in"], L["n_in"], L["n_out"], L["d_out"], 0)
                        for L in self.layers)
-        for grp in self.groups:
-            ws_bytes = max(ws_bytes, fq.fq_group_workspace_bytes(M, self.group_layers(grp)))
-        self.ws_bytes = ws_bytes
-        self.ws = torch.zeros(ws_bytes, dtype=torch.uint8, device=dev)
         # The step's activations and outputs live in one device buffer each (every layer a
         # 256-byte aligned slice), mirrored by one pinned host buffer each, so a step moves its
         # inputs in one host-to-device copy and its results in one device-to-host copy.
@@ -231,12 +227,21 @@ class Regime:
             L["x"].copy_(L["x_host"])
             L["y"] = self.y_all[y0:y0 + M * L["d_out"]].view(M, L["d_out"])
             L["y_host"] = self.y_host_all[y0:y0 + M * L["d_out"]].view(M, L["d_out"])
+        for grp in self.groups:
+            ws_bytes = max(ws_bytes, fq.fq_group_workspace_bytes(M, self.group_layers(grp)))
+        self.ws_bytes = ws_bytes
+        self.ws = torch.zeros(ws_bytes, dtype=torch.uint8, device=dev)
         # one eager call per layer before any capture (sets kernel attributes, checks status)
         for L in self.layers:
             self.forward(L, torch.cuda.current_stream(dev).cuda_stream)
             st = fq.fq_check(self.ws)
             if st != 0:
                 raise RuntimeError(f"{L['name']}: {fq.fq_status_str(st)}")
+        for grp in self.groups:
+            self.forward_group(grp, torch.cuda.current_stream(dev).cuda_stream)
+            st = fq.fq_check(self.ws)
+            if st != 0:
+                raise RuntimeError(f"group {[L['name'] for L in grp]}: {fq.fq_status_str(st)}")
         torch.cuda.synchronize()
 
     def group_layers(self, grp):

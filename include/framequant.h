@@ -58,6 +58,17 @@ enum {
   FQ_FP32_DEBUG = 1   /* x, T_in, T_out^T, y, z, u are fp32 throughout (CUDA cores) */
 };
 
+/* FQ_BF16 | FQ_ACT_BITS(N), 2 <= N <= 8: round the frame representation of the activations to
+ * N-bit integers before the code product (Appendix F: the INT8 form for N = 8).  With
+ * Delta = max |z| / (2^(N-1) - 1) over every token and coefficient of the call (z = T_in x in
+ * fp32) and zbar = nearest integer to z / Delta (ties to even), the layer computes
+ *     u_i = Delta gamma_i (s_i sum_j q_ij zbar_j + zero_i sum_j zbar_j),   y = T_out^T u.
+ * zbar is held exactly in bf16 and sum_j q_ij zbar_j is exact in the tensor cores' fp32
+ * accumulator, so the product is the integer one.  The whole analysis must finish before any
+ * rounding, so every batch size runs the tensor-core path's chain of kernels (an analysis that
+ * writes fp32 z and the maximum, a rounding kernel, the code product, the synthesis). */
+#define FQ_ACT_BITS(n) ((n) << 8)
+
 /* Packed 2-bit frame coefficients with their per-row scale and zero (the paper keeps one scale
  * and one offset per row next to the 2-bit codes, Appendix K).  Code q_ij in {0,1,2,3}
  * dequantizes to s_i q_ij + zero_i.  fq_pack fills this descriptor; it is the one unit every
@@ -131,7 +142,7 @@ size_t fq_workspace_bytes(int M, int d_in, int n_in, int n_out, int d_out, int m
  *            without being cleared again; zero it again after a call reported
  *            FQ_ERR_TIMEOUT.  Its first 4
  *            bytes are the device status word, which each call clears before reporting.
- *   mode     FQ_BF16 or FQ_FP32_DEBUG
+ *   mode     FQ_BF16 or FQ_FP32_DEBUG, or FQ_BF16 | FQ_ACT_BITS(N)
  * Requirements: M, d_in, d_out >= 1; d_in and d_out multiples of 8; C->n_in and C->n_out
  * positive multiples of 16, C->ld_words = 4 * ceil(C->n_in / 64) and C->bits = 2 (as fq_pack
  * sets them); all device pointers 16-byte aligned.

@@ -14,7 +14,7 @@ import os
 from dataclasses import dataclass
 
 __all__ = [
-    "FQ_BF16", "FQ_FP32_DEBUG", "FrameQuantError", "Packed", "ld_words", "lib", "lib_path",
+    "FQ_BF16", "FQ_FP32_DEBUG", "FQ_ACT_BITS", "FrameQuantError", "Packed", "ld_words", "lib", "lib_path",
     "fq_packed_words", "fq_pack", "fq_workspace_bytes", "fq_linear_forward",
     "fq_linear_forward_sms", "fq_linear_forward_ex", "fq_check",
     "fq_status_str", "EXPORTED", "fq_frame_workspace_bytes", "fq_frame_build",
@@ -30,6 +30,12 @@ FQ_STATIC_SCRATCH_BYTES = 16 << 20
 
 FQ_BF16 = 0
 FQ_FP32_DEBUG = 1
+
+
+def FQ_ACT_BITS(n: int) -> int:
+    """Mode flag: round the frame representation of the activations to n-bit integers
+    (FQ_BF16 | FQ_ACT_BITS(n), include/framequant.h)."""
+    return n << 8
 STATUS = {0: "FQ_OK", 1: "FQ_ERR_INVALID_ARG", 2: "FQ_ERR_ALIGNMENT", 3: "FQ_ERR_UNSUPPORTED",
           4: "FQ_ERR_WORKSPACE", 5: "FQ_ERR_CUDA", 6: "FQ_ERR_TIMEOUT",
           7: "FQ_ERR_DEVICE_CHECK"}

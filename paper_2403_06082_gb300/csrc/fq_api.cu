@@ -14,6 +14,16 @@ bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) ==
 
 fq_status cuda_status(cudaError_t e) { return e == cudaSuccess ? FQ_OK : FQ_ERR_CUDA; }
 
+// mode = FQ_BF16 or FQ_FP32_DEBUG, optionally | FQ_ACT_BITS(N) with FQ_BF16 and 2 <= N <= 8
+bool split_mode(int mode, int& base, int& act) {
+  base = mode & 0xFF;
+  act = (mode >> 8) & 0xFF;
+  if ((mode & ~0xFFFF) != 0) return false;
+  if (base != FQ_BF16 && base != FQ_FP32_DEBUG) return false;
+  if (act != 0 && (base != FQ_BF16 || act < 2 || act > 8)) return false;
+  return true;
+}
+
 // Compute capability of the current device, or -1.
 int current_cc() {
   int dev = 0, major = 0, minor = 0;
@@ -70,11 +80,14 @@ fq_status fq_pack(const uint8_t* codes, const uint16_t* scale_f16, const uint16_
 
 size_t fq_workspace_bytes(int M, int d_in, int n_in, int n_out, int d_out, int mode) {
   if (M <= 0 || d_in <= 0 || n_in <= 0 || n_out <= 0 || d_out <= 0) return 0;
-  if (mode == FQ_BF16)
+  int base = 0, act = 0;
+  if (!split_mode(mode, base, act)) return 0;
+  if (base == FQ_BF16) {
+    if (act > 0) return tc_workspace_bytes(M, d_in, n_in, n_out, d_out, act);
     return M <= kDecodeMaxM ? decode_workspace_bytes(M, d_in, n_in, n_out, d_out)
-                            : tc_workspace_bytes(M, d_in, n_in, n_out, d_out);
-  if (mode == FQ_FP32_DEBUG) return debug_workspace_bytes(M, n_in, n_out);
-  return 0;
+                            : tc_workspace_bytes(M, d_in, n_in, n_out, d_out, 0);
+  }
+  return debug_workspace_bytes(M, n_in, n_out);
 }
 
 }  // extern "C"
@@ -86,7 +99,8 @@ fq_status check_layer(const void* x, int M, int d_in, const void* T_in, const fq
                       const void* T_out_t, int d_out, const float* gamma, const void* y,
                       int mode) {
   if (!x || !T_in || !C || !T_out_t || !y) return FQ_ERR_INVALID_ARG;
-  if (mode != FQ_BF16 && mode != FQ_FP32_DEBUG) return FQ_ERR_INVALID_ARG;
+  int base = 0, act = 0;
+  if (!split_mode(mode, base, act)) return FQ_ERR_INVALID_ARG;
   if (M <= 0 || d_in <= 0 || d_out <= 0) return FQ_ERR_INVALID_ARG;
   if (const fq_status cs = check_packed(C)) return cs;
   if (d_in % 8 || d_out % 8) return FQ_ERR_ALIGNMENT;
@@ -139,12 +153,14 @@ fq_status fq_linear_forward_ex(const void* x, int M, int d_in, const void* T_in,
   if (const fq_status os = check_opts(opts, max_sms, pf, pf_bytes, inject)) return os;
   if (inject > 0 && (mode != FQ_BF16 || M <= 0 || M > kDecodeMaxM || max_sms != 1))
     return FQ_ERR_INVALID_ARG;
+  int base = 0, act = 0;
+  if (!split_mode(mode, base, act)) return FQ_ERR_INVALID_ARG;
   if (const fq_status ls = check_layer(x, M, d_in, T_in, C, T_out_t, d_out, gamma, y, mode))
     return ls;
   const size_t need = fq_workspace_bytes(M, d_in, C->n_in, C->n_out, d_out, mode);
   if (const fq_status ws_st = check_ws(ws, ws_bytes, need)) return ws_st;
   auto s = reinterpret_cast<cudaStream_t>(stream);
-  if (mode == FQ_FP32_DEBUG) {
+  if (base == FQ_FP32_DEBUG) {
     if (cudaMemsetAsync(ws, 0, kWsHeader, s) != cudaSuccess) return FQ_ERR_CUDA;
     return cuda_status(launch_debug_forward(
         static_cast<const float*>(x), M, d_in, static_cast<const float*>(T_in), *C,
@@ -152,13 +168,15 @@ fq_status fq_linear_forward_ex(const void* x, int M, int d_in, const void* T_in,
         static_cast<char*>(ws), s));
   }
   if (current_cc() != 103) return FQ_ERR_UNSUPPORTED;
-  // the status word is cleared by the forward's first kernel, in stream order
-  if (M <= kDecodeMaxM)
+  // the status word is cleared by the forward's first kernel, in stream order; rounding the
+  // activations needs the whole analysis before the code product, which the tensor-core
+  // path's chain of three kernels has at any batch size
+  if (M <= kDecodeMaxM && act == 0)
     return launch_decode_forward(x, M, d_in, T_in, *C, T_out_t, d_out, gamma, y,
                                  static_cast<char*>(ws), ws_bytes, max_sms, pf, pf_bytes, inject,
                                  s);
   return launch_tc_forward(x, M, d_in, T_in, *C, T_out_t, d_out, gamma, y,
-                           static_cast<char*>(ws), ws_bytes, max_sms, s);
+                           static_cast<char*>(ws), ws_bytes, max_sms, act, s);
 }
 
 size_t fq_group_workspace_bytes(int M, int n_layers, const fq_layer* layers) {
@@ -215,7 +233,7 @@ fq_status fq_linear_forward_group(int M, int n_layers, const fq_layer* layers, v
     const fq_layer& L = layers[l];
     if (const fq_status st = launch_tc_forward(L.x, M, L.d_in, L.T_in, *L.C, L.T_out_t, L.d_out,
                                                L.gamma, L.y, static_cast<char*>(ws), ws_bytes,
-                                               max_sms, s))
+                                               max_sms, 0, s))
       return st;
   }
   return FQ_OK;

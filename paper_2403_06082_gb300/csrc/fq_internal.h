@@ -19,13 +19,16 @@ inline int64_t round_up(int64_t a, int64_t b) { return ceil_div(a, b) * b; }
 
 // Workspace header (64 KiB, at fixed offsets whatever the layer's sizes, so that one workspace
 // can serve layers of different shapes): [0] device status word, [4] generation counter,
-// [8] end-of-call ticket, [16..31] the first timeout's role, task, stage and detail words
-// (cleared by each call), [kWsFlags] ready flags, kWsSlices per row tile of up to kWsMaxTiles
+// [8] end-of-call ticket, [12] the activation-rounding maximum, [16..31] the first timeout's
+// role, task, stage and detail words (cleared by each call), [32] the activation-rounding step,
+// [kWsFlags] ready flags, kWsSlices per row tile of up to kWsMaxTiles
 // row tiles per phase.  A zero-filled header is a valid initial state and every completed call
 // leaves it valid for the next one.
 constexpr size_t kWsHeader = 64 * 1024;
 constexpr size_t kWsGen = 4;
 constexpr size_t kWsDone = 8;
+constexpr size_t kWsAmax = 12;    // activation rounding: max |z| of the call (float bits)
+constexpr size_t kWsDelta = 32;   // activation rounding: the call's step Delta (float)
 constexpr size_t kWsFlags = 1024;
 constexpr int kWsSlices = 8;
 constexpr int kWsMaxTiles = 640;
@@ -93,10 +96,12 @@ size_t decode_core_u_offset(int M, int n_in);
 void haar_q(const double* G, int a, std::vector<double>& Q);
 
 // ---- fq_tc.cu: bf16 tensor-core path
-size_t tc_workspace_bytes(int M, int d_in, int n_in, int n_out, int d_out);
+// act_bits > 0: the analysis output is rounded to act_bits-bit integers with one step per call
+// (Appendix F) before the code product
+size_t tc_workspace_bytes(int M, int d_in, int n_in, int n_out, int d_out, int act_bits);
 fq_status launch_tc_forward(const void* x, int M, int d_in, const void* T_in,
                             const fq_packed& C, const void* T_out_t, int d_out,
                             const float* gamma, void* y, char* ws, size_t ws_bytes,
-                            int max_sms, cudaStream_t s);
+                            int max_sms, int act_bits, cudaStream_t s);
 
 }  // namespace fq

@@ -68,6 +68,10 @@ struct PhaseArgs {
   const __half* zero;
   const float* gamma;
   int32_t* status;
+  // Rounding of the frame representation of the activations (Appendix F), else all null:
+  float* out32;              // analysis: z in fp32 (the bf16 z is then the rounded one)
+  uint32_t* amax;            // analysis: running max |z| as float bits; the core resets it
+  const float* delta;        // core: the rounding step Delta, which scales the product
 };
 
 template <int PHASE, int BN>
@@ -246,6 +250,8 @@ __global__ void __launch_bounds__(threads_for<PHASE>(), 1)
       }
       pdl_wait();   // the previous kernel is complete and its writes are visible
       if (PHASE == kAnalysis && blockIdx.x == 0) *p.status = 0;   // new call: clear status
+      // the rounding kernel before this one has read the maximum: ready for the next call
+      if (PHASE == kCore && p.amax && blockIdx.x == 0) *p.amax = 0u;
       int stage = 0;
       uint32_t phase = 0;
       int it = 0;
@@ -382,11 +388,27 @@ __global__ void __launch_bounds__(threads_for<PHASE>(), 1)
                              static_cast<uint32_t>(buf * BN);
       const float* zs = zsum_s + buf * BN;
       const float g_i = (PHASE == kCore && row_ok && p.gamma) ? p.gamma[row] : 1.f;
+      // with rounded activations the accumulator is the exact integer sum_j q_ij zbar_j, and
+      // u = Delta gamma (s acc + zero sum_j zbar_j)
+      const float dl = (PHASE == kCore && p.delta) ? ldcg_f32(p.delta) : 1.f;
+      float amax_t = 0.f;                         // analysis with rounding: this row's max |z|
       // the finished values of columns c .. c + 15 of this thread's row
       auto emit = [&](int c, float* v) {
+        if (PHASE == kAnalysis && p.out32) {
+          // fp32 z for the rounding kernel, and the running maximum of |z|
+#pragma unroll
+          for (int q = 0; q < kChunk; ++q) {
+            const int t = t0 + c + q;
+            if (row_ok && t < p.M) {
+              p.out32[static_cast<int64_t>(t) * p.R + row] = v[q];
+              amax_t = fmaxf(amax_t, fabsf(v[q]));
+            }
+          }
+          return;
+        }
 #pragma unroll
         for (int q = 0; q < kChunk; ++q) {
-          if (PHASE == kCore) v[q] = g_i * fmaf(s_i, v[q], z_i * zs[c + q]);
+          if (PHASE == kCore) v[q] = g_i * fmaf(s_i, v[q], z_i * zs[c + q]) * dl;
           const __nv_bfloat16 b = __float2bfloat16_rn(v[q]);
           v[q] = __bfloat162float(b);
           const int t = t0 + c + q;
@@ -468,6 +490,14 @@ __global__ void __launch_bounds__(threads_for<PHASE>(), 1)
         }
         named_barrier_sync(1, kEpi);                 // the flag is read before it is reused
       }
+      if (PHASE == kAnalysis && p.out32) {
+        // one atomic per warp and tile: the tensor's max |z| (non-negative floats order like
+        // their bit patterns)
+#pragma unroll
+        for (int off = 16; off > 0; off >>= 1)
+          amax_t = fmaxf(amax_t, __shfl_xor_sync(0xffffffffu, amax_t, off));
+        if (lane == 0 && amax_t > 0.f) atomicMax(p.amax, __float_as_uint(amax_t));
+      }
       if (++buf == 2) buf = 0, acc_phase ^= 1;
     }
   } else {
@@ -509,6 +539,44 @@ __global__ void __launch_bounds__(threads_for<PHASE>(), 1)
   if (warp == 1) {
     tc_fence_after_sync();
     tmem_dealloc(tmem_base, Lo::kTmemCols);
+  }
+}
+
+// Rounding of the frame representation of the activations (Appendix F): with the tensor's
+// step Delta = max |z| / L, L = 2^(N-1) - 1, zq = nearest integer to z / Delta (ties to even,
+// clamped to [-L, L]) as bf16 (exact: |zq| <= 127 needs 7 significant bits), and the per-token
+// sum of zq for the zero term (exact in fp32: at most 127 * 81920 < 2^24).  One block per
+// token row and round.
+constexpr int kQuantThreads = 256;
+
+__global__ void __launch_bounds__(kQuantThreads) ff_round_kernel(
+    const float* __restrict__ z32, int M, int n, float L, const uint32_t* __restrict__ amax,
+    float* __restrict__ delta, __nv_bfloat16* __restrict__ zq, float* __restrict__ zsum) {
+  __shared__ float red[kQuantThreads / 32];
+  pdl_launch_dependents();
+  pdl_wait();                                   // the analysis is complete
+  const float d = __uint_as_float(*reinterpret_cast<const volatile uint32_t*>(amax)) / L;
+  if (blockIdx.x == 0 && threadIdx.x == 0) *delta = d;
+  for (int t = blockIdx.x; t < M; t += gridDim.x) {
+    const float* zr = z32 + static_cast<int64_t>(t) * n;
+    __nv_bfloat16* qr = zq + static_cast<int64_t>(t) * n;
+    float s = 0.f;
+    for (int j = threadIdx.x; j < n; j += kQuantThreads) {
+      float q = d > 0.f ? rintf(__fdiv_rn(__ldcg(zr + j), d)) : 0.f;
+      q = fminf(fmaxf(q, -L), L);
+      qr[j] = __float2bfloat16_rn(q);
+      s += q;
+    }
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) s += __shfl_xor_sync(0xffffffffu, s, off);
+    if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = s;
+    __syncthreads();
+    if (threadIdx.x == 0) {
+      float tot = 0.f;
+      for (int w = 0; w < kQuantThreads / 32; ++w) tot += red[w];
+      zsum[t] = tot;
+    }
+    __syncthreads();
   }
 }
 
@@ -599,12 +667,12 @@ void plan_phase(PhaseArgs& a, const DeviceInfo& d, int& grid) {
 }
 
 struct WsLayout {
-  size_t z, u, zsum, cnt, part, total;
+  size_t z, u, zsum, cnt, part, z32, total;
 };
 
 // Partial tiles for split K, sized for any device with at most kMaxSplitSms SMs: a phase with
 // t < kMaxSplitSms tiles keeps at most min(kMaxSplitSms, t * kMaxSplits) partial tiles.
-WsLayout ws_layout(int M, int d_in, int n_in, int n_out, int d_out) {
+WsLayout ws_layout(int M, int d_in, int n_in, int n_out, int d_out, int act_bits) {
   WsLayout L{};
   size_t off = kWsHeader;
   L.z = off;
@@ -629,6 +697,8 @@ WsLayout ws_layout(int M, int d_in, int n_in, int n_out, int d_out) {
   off += round_up(max_tiles * 4, 256);
   L.part = off;
   off += static_cast<size_t>(slots) * BN * kBM * 4;
+  L.z32 = off;
+  if (act_bits > 0) off += round_up(static_cast<int64_t>(M) * n_in * 4, 256);
   L.total = off;
   return L;
 }
@@ -651,8 +721,25 @@ cudaError_t launch_phase(const CUtensorMap& tmA, const CUtensorMap& tmB, const P
 
 // maps: {T_in, x, z, T_out^T, u}.  The core phase's A operand is the packed codes, so it gets
 // an unused map in that slot.
+cudaError_t launch_round(const PhaseArgs& an, int n_in, int act_bits, const DeviceInfo& d,
+                         float* delta, __nv_bfloat16* zq, float* zsum, cudaStream_t s) {
+  cudaLaunchConfig_t cfg{};
+  cfg.gridDim = dim3(static_cast<unsigned>(std::max(1, std::min(an.M, 4 * d.sms))));
+  cfg.blockDim = dim3(kQuantThreads);
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  const float L = static_cast<float>((1 << (act_bits - 1)) - 1);
+  return cudaLaunchKernelEx(&cfg, ff_round_kernel, static_cast<const float*>(an.out32), an.M,
+                            n_in, L, static_cast<const uint32_t*>(an.amax), delta, zq, zsum);
+}
+
 template <int BN>
-fq_status run_forward(const CUtensorMap* maps, PhaseArgs* a, int max_sms, cudaStream_t s) {
+fq_status run_forward(const CUtensorMap* maps, PhaseArgs* a, int max_sms, int act_bits,
+                      float* delta, cudaStream_t s) {
   DeviceInfo d = device_info();
   if (max_sms > 0) d.sms = std::min(d.sms, max_sms);
   if (prepare_kernel<kAnalysis, BN>(d.dev) != cudaSuccess ||
@@ -663,9 +750,13 @@ fq_status run_forward(const CUtensorMap* maps, PhaseArgs* a, int max_sms, cudaSt
   plan_phase<kAnalysis, BN>(a[0], d, g[0]);
   plan_phase<kCore, BN>(a[1], d, g[1]);
   plan_phase<kSynthesis, BN>(a[2], d, g[2]);
-  a[1].zsum_tiles = a[0].RT;
-  if (launch_phase<kAnalysis, BN>(maps[0], maps[1], a[0], g[0], s) != cudaSuccess ||
-      launch_phase<kCore, BN>(maps[1], maps[2], a[1], g[1], s) != cudaSuccess ||
+  a[1].zsum_tiles = act_bits > 0 ? 1 : a[0].RT;      // rounded: one exact sum per token
+  if (launch_phase<kAnalysis, BN>(maps[0], maps[1], a[0], g[0], s) != cudaSuccess)
+    return FQ_ERR_CUDA;
+  if (act_bits > 0 && launch_round(a[0], a[1].K, act_bits, d, delta, a[0].out, a[0].zsum_part,
+                                   s) != cudaSuccess)
+    return FQ_ERR_CUDA;
+  if (launch_phase<kCore, BN>(maps[1], maps[2], a[1], g[1], s) != cudaSuccess ||
       launch_phase<kSynthesis, BN>(maps[3], maps[4], a[2], g[2], s) != cudaSuccess)
     return FQ_ERR_CUDA;
   return FQ_OK;
@@ -727,16 +818,16 @@ bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) ==
 
 }  // namespace
 
-size_t tc_workspace_bytes(int M, int d_in, int n_in, int n_out, int d_out) {
-  return ws_layout(M, d_in, n_in, n_out, d_out).total;
+size_t tc_workspace_bytes(int M, int d_in, int n_in, int n_out, int d_out, int act_bits) {
+  return ws_layout(M, d_in, n_in, n_out, d_out, act_bits).total;
 }
 
 fq_status launch_tc_forward(const void* x, int M, int d_in, const void* T_in,
                             const fq_packed& Cq, const void* T_out_t, int d_out,
                             const float* gamma, void* y, char* ws, size_t ws_bytes,
-                            int max_sms, cudaStream_t s) {
+                            int max_sms, int act_bits, cudaStream_t s) {
   const int n_in = Cq.n_in, n_out = Cq.n_out;
-  const WsLayout L = ws_layout(M, d_in, n_in, n_out, d_out);
+  const WsLayout L = ws_layout(M, d_in, n_in, n_out, d_out, act_bits);
   if (ws_bytes < L.total) return FQ_ERR_WORKSPACE;
   const int BN = pick_bn(M);
   auto* status = reinterpret_cast<int32_t*>(ws);
@@ -763,6 +854,14 @@ fq_status launch_tc_forward(const void* x, int M, int d_in, const void* T_in,
   a[1].scale = reinterpret_cast<const __half*>(Cq.scale_f16);
   a[1].zero = reinterpret_cast<const __half*>(Cq.zero_f16);
   a[1].gamma = gamma;
+  float* delta = nullptr;
+  if (act_bits > 0) {
+    a[0].out32 = reinterpret_cast<float*>(ws + L.z32);
+    a[0].amax = reinterpret_cast<uint32_t*>(ws + kWsAmax);
+    delta = reinterpret_cast<float*>(ws + kWsDelta);
+    a[1].amax = a[0].amax;
+    a[1].delta = delta;
+  }
 
   // maps: T_in, x, z, T_out^T, u  (A maps use 128-row boxes, B maps BN-row boxes)
   CUtensorMap maps[5];
@@ -771,7 +870,8 @@ fq_status launch_tc_forward(const void* x, int M, int d_in, const void* T_in,
       !make_tmap(&maps[4], u, M, n_out, BN))
     return FQ_ERR_CUDA;
 
-  return BN == 128 ? run_forward<128>(maps, a, max_sms, s) : run_forward<256>(maps, a, max_sms, s);
+  return BN == 128 ? run_forward<128>(maps, a, max_sms, act_bits, delta, s)
+                   : run_forward<256>(maps, a, max_sms, act_bits, delta, s);
 }
 
 }  // namespace fq

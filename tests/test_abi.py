@@ -260,3 +260,19 @@ def test_group_sizes_and_validation_without_gpu(L):
     assert fwd(arr(layer()), 1, ws=0x10010) == 2
     assert fwd(arr(layer()), 1, nb=1024) == 4
     assert fwd(arr(layer()), 1, opts=fq._Opts(1, None, 0, 1000)) == 1   # no timeout hook
+
+
+def test_activation_rounding_modes_without_gpu(L):
+    A8 = fq.FQ_BF16 | fq.FQ_ACT_BITS(8)
+    # the tensor-core layout at any batch size, plus the fp32 z
+    assert fq.fq_workspace_bytes(16, 4096, 4512, 4512, 4096, A8) >= \
+        fq.fq_workspace_bytes(16, 4096, 4512, 4512, 4096, 0) + 16 * 4512 * 4
+    assert fq.fq_workspace_bytes(300, 4096, 4512, 4512, 4096, A8) == \
+        fq.fq_workspace_bytes(300, 4096, 4512, 4512, 4096, 0) + 300 * 4512 * 4
+    assert fq.fq_workspace_bytes(16, 4096, 4512, 4512, 4096, fq.FQ_ACT_BITS(1)) == 0
+    assert fq.fq_workspace_bytes(16, 4096, 4512, 4512, 4096, fq.FQ_ACT_BITS(9)) == 0
+    assert fq.fq_workspace_bytes(16, 4096, 4512, 4512, 4096,
+                                 fq.FQ_FP32_DEBUG | fq.FQ_ACT_BITS(8)) == 0
+    assert _call(L, mode=fq.FQ_ACT_BITS(9)) == 1
+    assert _call(L, mode=fq.FQ_FP32_DEBUG | fq.FQ_ACT_BITS(4)) == 1
+    assert _call(L, mode=1 << 20) == 1
