@@ -301,6 +301,38 @@ fq_status fq_coefficients(const float* W, int d_out, int d_in, const float* T_in
 fq_status fq_quantize_rtn(const float* C, int n_out, int n_in, uint8_t* codes, uint16_t* scale,
                           uint16_t* zero, float* gamma, fq_stream_t stream);
 
+/* H = Z^T Z (n_in x n_in, fp64): the Hessian of Algorithm 1's proxy loss,
+ * ||D C_prev - D_hat C_prev||_F^2 = tr((D - D_hat) H (D - D_hat)^T) with H = C_prev C_prev^T
+ * (Sec. 3), from Z = C_prev^T, the frame representations T_in a of N calibration tokens a (one
+ * token per row, N x n_in, fp64).  Device pointers, 8-byte aligned; fp64 CUDA-core product.
+ * Errors: FQ_ERR_INVALID_ARG, FQ_ERR_ALIGNMENT, FQ_ERR_CUDA. */
+fq_status fq_gptq_hessian(const double* Z, int N, int n_in, double* H, fq_stream_t stream);
+
+/* Workspace bytes of fq_quantize_gptq: 8 (n_out n_in + 2 n_in^2 + 130 n_out) + n_out n_in
+ * bytes and a few KB (about 0.83 GB for 12112 x 4512); 0 for invalid sizes. */
+size_t fq_gptq_workspace_bytes(int n_out, int n_in);
+
+/* 2-bit codes of C (n_out x n_in, fp64 frame coefficients) by the frame-domain quantizer of
+ * Algorithm 1, steps 2-4, in fp64 on the GPU:
+ *   - clip != 0: C is clipped to [mu - 2 sigma, mu + 2 sigma], mu and sigma over all of C;
+ *   - every row's grid is fixed from the (clipped) row before the iteration, as in
+ *     fq_quantize_rtn: zero = fp16(min), scale = fp16((max - min) / 3) (1 when 0); gamma
+ *     (nullable) receives the de-noising gain P / (P + scale^2 / 12) of the clipped rows;
+ *   - the Hessian H (n_in x n_in, e.g. from fq_gptq_hessian) is damped by damp mean(diag H)
+ *     (0.01 is the usual value) and factored as H^-1 = U^T U, U upper triangular;
+ *   - the columns are rounded in order, in blocks of 128; after column j each row's rounding
+ *     error divided by U_jj is spread over its later columns in proportion to row j of U (the
+ *     optimal-brain-surgeon update of the method GPTQ, which Algorithm 1 cites).
+ *   codes  device uint8 n_out x n_in;  scale, zero  device fp16 bits [n_out];  gamma fp32 or NULL
+ *   ws     device workspace of fq_gptq_workspace_bytes(n_out, n_in) bytes, 256-byte aligned
+ * Synchronizes `stream` before returning.  n_in up to 25600 (the triangular inverse keeps one
+ * column in shared memory).
+ * Errors: FQ_ERR_INVALID_ARG, FQ_ERR_ALIGNMENT, FQ_ERR_WORKSPACE, FQ_ERR_UNSUPPORTED (n_in above
+ * 25600), FQ_ERR_DEVICE_CHECK (the damped H is not positive definite), FQ_ERR_CUDA. */
+fq_status fq_quantize_gptq(const double* C, int n_out, int n_in, const double* H, double damp,
+                           int clip, uint8_t* codes, uint16_t* scale, uint16_t* zero,
+                           float* gamma, void* ws, size_t ws_bytes, fq_stream_t stream);
+
 /* ------------------------------------------------------------------------------------------
  * Frames in structured form (the paper's own deployment form: Sec. 2.2 and Appendix J build T
  * from rho/2 disjoint runs of a spectral-tetris frame, each modulated by k roots of unity;

@@ -23,7 +23,8 @@ __all__ = [
     "fq_frame_implicit", "fq_implicit_workspace_bytes", "fq_linear_forward_implicit",
     "fq_reconstruct_workspace_bytes", "fq_reconstruct_weight", "fq_dense_workspace_bytes",
     "fq_dense_forward", "fq_static_check", "fq_group_workspace_bytes",
-    "fq_linear_forward_group", "Layer", "FQ_MAX_GROUP",
+    "fq_linear_forward_group", "Layer", "FQ_MAX_GROUP", "fq_gptq_hessian",
+    "fq_gptq_workspace_bytes", "fq_quantize_gptq",
 ]
 FQ_MAX_GROUP = 4
 FQ_STATIC_SCRATCH_BYTES = 16 << 20
@@ -47,7 +48,8 @@ EXPORTED = ("fq_packed_words", "fq_pack", "fq_workspace_bytes", "fq_linear_forwa
             "fq_implicit_workspace_bytes", "fq_linear_forward_implicit",
             "fq_reconstruct_workspace_bytes", "fq_reconstruct_weight", "fq_dense_workspace_bytes",
             "fq_dense_forward", "fq_static_check", "fq_group_workspace_bytes",
-            "fq_linear_forward_group")
+            "fq_linear_forward_group", "fq_gptq_hessian", "fq_gptq_workspace_bytes",
+            "fq_quantize_gptq")
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
 
@@ -158,6 +160,16 @@ def lib() -> ctypes.CDLL:
         L.fq_linear_forward_group.argtypes = [ctypes.c_int, ctypes.c_int, ctypes.POINTER(_Layer),
                                               ctypes.c_void_p, ctypes.c_size_t,
                                               ctypes.POINTER(_Opts), ctypes.c_void_p]
+        L.fq_gptq_hessian.restype = ctypes.c_int
+        L.fq_gptq_hessian.argtypes = [ctypes.c_void_p, ctypes.c_int, ctypes.c_int, ctypes.c_void_p,
+                                      ctypes.c_void_p]
+        L.fq_gptq_workspace_bytes.restype = ctypes.c_size_t
+        L.fq_gptq_workspace_bytes.argtypes = [ctypes.c_int, ctypes.c_int]
+        L.fq_quantize_gptq.restype = ctypes.c_int
+        L.fq_quantize_gptq.argtypes = [ctypes.c_void_p, ctypes.c_int, ctypes.c_int, ctypes.c_void_p,
+                                       ctypes.c_double, ctypes.c_int, ctypes.c_void_p,
+                                       ctypes.c_void_p, ctypes.c_void_p, ctypes.c_void_p,
+                                       ctypes.c_void_p, ctypes.c_size_t, ctypes.c_void_p]
         L.fq_static_check.restype = ctypes.c_int
         L.fq_static_check.argtypes = [ctypes.c_void_p]
         L.fq_frame_implicit_bytes.restype = ctypes.c_size_t
@@ -464,6 +476,24 @@ def fq_dense_forward(x, M: int, d_in: int, W_hat, d_out: int, y, ws, ws_bytes: i
     """y = x W_hat^T on the tensor cores (include/framequant_dense.h)."""
     _ok(lib().fq_dense_forward(_ptr(x), M, d_in, _ptr(W_hat), d_out, _ptr(y), _ptr(ws), ws_bytes,
                                _stream(stream)), "fq_dense_forward")
+
+
+def fq_gptq_hessian(Z, N: int, n_in: int, H, stream=None) -> None:
+    """H = Z^T Z for calibration tokens' frame representations Z (N x n_in, fp64)."""
+    _ok(lib().fq_gptq_hessian(_ptr(Z), N, n_in, _ptr(H), _stream(stream)), "fq_gptq_hessian")
+
+
+def fq_gptq_workspace_bytes(n_out: int, n_in: int) -> int:
+    return lib().fq_gptq_workspace_bytes(n_out, n_in)
+
+
+def fq_quantize_gptq(C, n_out: int, n_in: int, H, codes, scale, zero, gamma=None, ws=None,
+                     ws_bytes: int = 0, damp: float = 0.01, clip: bool = False,
+                     stream=None) -> None:
+    """Frame-domain GPTQ of C (fp64) against H (fp64), include/framequant.h."""
+    _ok(lib().fq_quantize_gptq(_ptr(C), n_out, n_in, _ptr(H), damp, int(clip), _ptr(codes),
+                               _ptr(scale), _ptr(zero), _ptr(gamma), _ptr(ws), ws_bytes,
+                               _stream(stream)), "fq_quantize_gptq")
 
 
 def fq_coefficients_workspace_bytes(d_out: int, n_in: int) -> int:

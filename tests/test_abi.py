@@ -276,3 +276,24 @@ def test_activation_rounding_modes_without_gpu(L):
     assert _call(L, mode=fq.FQ_ACT_BITS(9)) == 1
     assert _call(L, mode=fq.FQ_FP32_DEBUG | fq.FQ_ACT_BITS(4)) == 1
     assert _call(L, mode=1 << 20) == 1
+
+
+def test_gptq_validation_without_gpu(L):
+    assert fq.fq_gptq_workspace_bytes(0, 64) == 0
+    n = fq.fq_gptq_workspace_bytes(12112, 4512)
+    assert n >= 8 * (12112 * 4512 + 2 * 4512 * 4512) + 12112 * 4512
+    assert L.fq_gptq_hessian(None, 10, 16, 0x2000, None) == 1
+    assert L.fq_gptq_hessian(0x1004, 10, 16, 0x2000, None) == 2
+
+    def q(C=0x1000, n_out=16, n_in=32, H=0x2000, damp=0.01, codes=0x3000, scale=0x4000,
+          zero=0x5000, gamma=None, ws=0x10000, nb=1 << 30):
+        return L.fq_quantize_gptq(C, n_out, n_in, H, damp, 0, codes, scale, zero, gamma, ws, nb,
+                                  None)
+    assert q(C=None) == 1
+    assert q(damp=-0.5) == 1
+    assert q(damp=float("nan")) == 1
+    assert q(H=0x2004) == 2
+    assert q(scale=0x4001) == 2
+    assert q(ws=None) == 4
+    assert q(ws=0x10010) == 2
+    assert q(nb=1024) == 4
