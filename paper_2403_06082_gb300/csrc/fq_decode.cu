@@ -182,7 +182,9 @@ struct Task {
   int l, p, tile;
 };
 
-__device__ __forceinline__ const DecPhase& phase_of(const DecArgs& a, int l, int p) {
+// by value: the roles keep a task's phase constants in registers (loads from the parameter
+// space with a dynamic index are not free in the flag-polling and copy loops)
+__device__ __forceinline__ DecPhase phase_of(const DecArgs& a, int l, int p) {
   return a.L[l].ph[p];
 }
 
@@ -356,7 +358,9 @@ __global__ void __launch_bounds__(DecCfg<BN>::kThreads, 1)
       for (int i = t_lo; i < t_hi && wok; ++i) {
         if (__any_sync(0xffffffffu, *abort_flag != 0)) break;
         const Task t = task_at(sched, i);
-        const DecPhase& ph = phase_of(a, t.l, t.p);
+        const DecPhase ph = phase_of(a, t.l, t.p);
+        const uint32_t* words = a.L[t.l].words;
+        const CUtensorMap* tmA = &maps.m[t.l][t.p == 0 ? kMapTin : kMapTout];
         int k0, k1;
         krange(ph, k0, k1);
         if (next_pf && t.p == 2) prefetch_next();
@@ -367,7 +371,7 @@ __global__ void __launch_bounds__(DecCfg<BN>::kThreads, 1)
           for (int j = i; j < t_hi && lane == 0; ++j) {
             const Task u = task_at(sched, j);
             if (u.p != 2 || !a.L[u.l].pf_tout) continue;
-            const DecPhase& q = phase_of(a, u.l, u.p);
+            const DecPhase q = phase_of(a, u.l, u.p);
             int u0, u1;
             krange(q, u0, u1);
             for (int kb = u0; kb < u1; ++kb)
@@ -394,7 +398,7 @@ __global__ void __launch_bounds__(DecCfg<BN>::kThreads, 1)
             if (lane == 0) {
               mbar_arrive_expect_tx(&cfull[stage], kCodeBytes);
               bulk_load(sC + stage * kCodeBytes,
-                        a.L[t.l].words + (static_cast<int64_t>(t.tile) * ph.KB + kb) * 512,
+                        words + (static_cast<int64_t>(t.tile) * ph.KB + kb) * 512,
                         kCodeBytes, &cfull[stage], pol_w);
             }
             last_code |= bit;
@@ -403,8 +407,8 @@ __global__ void __launch_bounds__(DecCfg<BN>::kThreads, 1)
           } else {
             if (lane == 0) {
               mbar_arrive_expect_tx(&fullA[stage], kATile);
-              tma_load_2d(sA + stage * kATile, &maps.m[t.l][t.p == 0 ? kMapTin : kMapTout],
-                          &fullA[stage], kb * kBK, t.tile * kBM, pol_w);
+              tma_load_2d(sA + stage * kATile, tmA, &fullA[stage], kb * kBK, t.tile * kBM,
+                          pol_w);
             }
             last_code &= ~bit;
             last_par = (last_par & ~bit) | (phase << stage);
@@ -416,7 +420,7 @@ __global__ void __launch_bounds__(DecCfg<BN>::kThreads, 1)
           // warm L2 with the code blocks of this CTA's later tasks
           for (int j = i + 1; j < t_hi && a.pf_codes && lane == 0; ++j) {
             const Task u = task_at(sched, j);
-            const DecPhase& q = phase_of(a, u.l, u.p);
+            const DecPhase q = phase_of(a, u.l, u.p);
             int u0, u1;
             krange(q, u0, u1);
             if (u.p == 1 && u1 > u0) {
@@ -458,13 +462,13 @@ __global__ void __launch_bounds__(DecCfg<BN>::kThreads, 1)
     for (int i = t_lo; i < t_hi; ++i) {
       if (__shfl_sync(0xffffffffu, *abort_flag != 0, 0)) break;   // warp-uniform
       const Task t = task_at(sched, i);
-      const DecPhase& ph = phase_of(a, t.l, t.p);
+      const DecPhase ph = phase_of(a, t.l, t.p);
       int k0, k1;
       krange(ph, k0, k1);
       // Loads go out in K order as soon as the slices of the previous phase's output that a K
       // block reads are final: the lanes poll the not-yet-final slices of the K range, and
       // the ready prefix decides how far lane 0 may issue.
-      const DecPhase& src = phase_of(a, t.l, t.p > 0 ? t.p - 1 : 0);
+      const DecPhase src = phase_of(a, t.l, t.p > 0 ? t.p - 1 : 0);
       const int sl1 = k1 > k0 ? (min(ph.K, k1 * kBK) - 1) / rows_per : 0;
       int ready = k1 > k0 ? (k0 * kBK) / rows_per : 0;   // slices below `ready` are final
       const long long t_start = clock64();
@@ -538,7 +542,7 @@ __global__ void __launch_bounds__(DecCfg<BN>::kThreads, 1)
       bool issued_any = false;
       for (int i = t_lo; i < t_hi && !*abort_flag; ++i) {
         const Task t = task_at(sched, i);
-        const DecPhase& ph = phase_of(a, t.l, t.p);
+        const DecPhase ph = phase_of(a, t.l, t.p);
         int k0, k1;
         krange(ph, k0, k1);
         if (!mbar_wait(&tempty[buf], acc_phase ^ 1, abort_flag)) {
@@ -595,7 +599,7 @@ __global__ void __launch_bounds__(DecCfg<BN>::kThreads, 1)
     for (int i = t_lo; i < t_hi && ok; ++i) {
       if (__shfl_sync(0xffffffffu, *abort_flag != 0, 0)) break;   // warp-uniform
       const Task t = task_at(sched, i);
-      const DecPhase& ph = phase_of(a, t.l, t.p);
+      const DecPhase ph = phase_of(a, t.l, t.p);
       int k0, k1;
       krange(ph, k0, k1);
       const int n = max(0, k1 - k0);
@@ -649,8 +653,11 @@ __global__ void __launch_bounds__(DecCfg<BN>::kThreads, 1)
     int j = 0;                                    // tasks finished by this CTA
     for (int i = t_lo; i < t_hi; ++i, ++j) {
       const Task t = task_at(sched, i);
-      const DecLayer& Ly = a.L[t.l];
-      const DecPhase& ph = Ly.ph[t.p];
+      const DecPhase ph = phase_of(a, t.l, t.p);
+      const DecPhase ph_z = phase_of(a, t.l, 0);      // the layer's z and its ready flags
+      const __half* l_scale = a.L[t.l].scale;
+      const __half* l_zero = a.L[t.l].zero;
+      const float* l_gamma = a.L[t.l].gamma;
       int k0, k1;
       krange(ph, k0, k1);
       const bool has_k = k1 > k0;
@@ -658,9 +665,9 @@ __global__ void __launch_bounds__(DecCfg<BN>::kThreads, 1)
       const bool row_ok = row < ph.R;
       float s_i = 0.f, z_i = 0.f, g_row = 1.f;
       if (t.p == 1 && row_ok) {
-        s_i = __half2float(Ly.scale[row]);
-        z_i = __half2float(Ly.zero[row]);
-        if (Ly.gamma) g_row = Ly.gamma[row];
+        s_i = __half2float(l_scale[row]);
+        z_i = __half2float(l_zero[row]);
+        if (l_gamma) g_row = l_gamma[row];
       }
       const float zb_i = z_i - 4.f * s_i;          // the decoded codes carry an offset of 4
       bool fail = false;
@@ -669,7 +676,7 @@ __global__ void __launch_bounds__(DecCfg<BN>::kThreads, 1)
         if (has_k && !(a.ext_in & 2)) {
           const int sl0 = (k0 * kBK) / rows_per, sl1 = (min(ph.K, k1 * kBK) - 1) / rows_per;
           for (int gs = sl0 + et; gs <= sl1 && !fail; gs += kEpi) {
-            fail = !wait_flag(&Ly.ph[0].flags[(gs / S) * kWsSlices + gs % S], g, abort_flag);
+            fail = !wait_flag(&ph_z.flags[(gs / S) * kWsSlices + gs % S], g, abort_flag);
             if (fail && !*abort_flag) note_timeout(a.status, 8, i, gs, 0);
           }
         }
@@ -687,7 +694,7 @@ __global__ void __launch_bounds__(DecCfg<BN>::kThreads, 1)
             // z columns k0 * 64 .. of token q: multiples of 8 (n_in is a multiple of 16), so
             // 16-byte loads from L2, each thread a strided share
             const int c0 = k0 * kBK, c1 = min(ph.K, k1 * kBK);
-            const __nv_bfloat16* zr = Ly.ph[0].out + static_cast<int64_t>(q) * ph.K;
+            const __nv_bfloat16* zr = ph_z.out + static_cast<int64_t>(q) * ph.K;
             for (int c = c0 + 8 * part; c < c1; c += 8 * kPer) {
               const uint4 w = ldcg_u4(zr + c);
               const uint32_t wv[4] = {w.x, w.y, w.z, w.w};
