@@ -77,10 +77,13 @@ constexpr int kChunk = 16;
 // into their own accumulator, which the epilogue adds.  Owning stages (not K blocks) keeps
 // every barrier of a stage waited for by one thread, in phase order.  With 64 tokens the
 // epilogue's registers do not leave room for the extra warps: one issuer.
+// With four issuers the code decode also gets a second warp per stage (warps 16-19), each of
+// a stage's two decoders expanding half of its rows; with 64 tokens neither fits.
 template <int BN>
 struct DecCfg {
   static constexpr int NI = BN <= 32 ? 4 : 1;
-  static constexpr int kThreads = NI == 4 ? 512 : 384;
+  static constexpr bool kPairs = NI == 4;
+  static constexpr int kThreads = NI == 4 ? 640 : 384;
 };
 // warp -> issuer index (warps 1, 12, 14, 15: sub-partitions 1, 0, 2, 3), -1 for other roles
 __host__ __device__ constexpr int issuer_of(int warp, int ni) {
@@ -292,11 +295,16 @@ __global__ void __launch_bounds__(DecCfg<BN>::kThreads, 1)
   if (warp == 0) {
     // the barriers, initialised lane-parallel: fullA, fullB, empty, cfull (count 1), tfull[2]
     // (one commit per issuer), tempty[2] (kEpi), mma_done[4] (1), recv_bar[2] (1)
+    // fullA takes two arrivals per round when a stage has two decoders: the weight
+    // producer's two (with the tile's bytes), or one from each decoder
+    constexpr uint32_t kFullA = DecCfg<BN>::kPairs ? 2u : 1u;
     for (int b = lane; b < Lo::kBars; b += 32) {
       const int r = b - 4 * S_;
-      const uint32_t cnt = r < 0 ? 1u
-                                 : (r < 2 ? static_cast<uint32_t>(NI)
-                                          : (r < 4 ? static_cast<uint32_t>(kEpi) : 1u));
+      const uint32_t cnt = b < S_ ? kFullA
+                                  : (r < 0 ? 1u
+                                           : (r < 2 ? static_cast<uint32_t>(NI)
+                                                    : (r < 4 ? static_cast<uint32_t>(kEpi)
+                                                             : 1u)));
       mbar_init(&fullA[b], cnt);
     }
     fence_barrier_init();
@@ -407,6 +415,7 @@ __global__ void __launch_bounds__(DecCfg<BN>::kThreads, 1)
           } else {
             if (lane == 0) {
               mbar_arrive_expect_tx(&fullA[stage], kATile);
+              if (DecCfg<BN>::kPairs) mbar_arrive(&fullA[stage]);
               tma_load_2d(sA + stage * kATile, tmA, &fullA[stage], kb * kBK, t.tile * kBM,
                           pol_w);
             }
@@ -587,12 +596,15 @@ __global__ void __launch_bounds__(DecCfg<BN>::kThreads, 1)
         if (!mbar_wait(&mma_done[q], 0, nullptr)) report(a.status, FQ_ERR_TIMEOUT);
       }
     }
-  } else if (warp >= 7 && warp <= 10) {
+  } else if ((warp >= 7 && warp <= 10) || (DecCfg<BN>::kPairs && warp >= 16 && warp <= 19)) {
     // -------------------------------------------------------------- code decoders
-    // Decoder d (warps 7-10) expands the code blocks of the core rounds that land in
-    // ring stages s = d (mod 4) into the stage's A slot; it waits for nothing else.  All lanes
+    // Decoder d (warps 7-10, and 16-19 with decoder pairs) expands the code blocks of the core
+    // rounds that land in ring stages s = d (mod 4) into the stage's A slot (with pairs, rows
+    // 0-63 by warp 7 + d and rows 64-127 by warp 16 + d); it waits for nothing else.  All lanes
     // wait (measured: one polling lane with the others parked in a shuffle wakes later).
-    const int dw = warp - 7;
+    const int dw = warp <= 10 ? warp - 7 : warp - 16;
+    constexpr int kRR = DecCfg<BN>::kPairs ? 2 : 4;         // 32-row groups per decoder
+    const int rr0 = warp <= 10 ? 0 : 2;
     int stage = 0;
     uint32_t cpar = 0;     // bit s: parity of the next cfull[s] phase
     bool ok = true;
@@ -619,7 +631,7 @@ __global__ void __launch_bounds__(DecCfg<BN>::kThreads, 1)
           const uint4* codes = reinterpret_cast<const uint4*>(sC + stage * kCodeBytes);
           uint8_t* tile_a = sA + stage * kATile;
 #pragma unroll
-          for (int rr = 0; rr < 4; ++rr)
+          for (int rr = rr0; rr < rr0 + kRR; ++rr)
             decode_row_dec(codes[lane + 32 * rr], tile_a, lane + 32 * rr);
           fence_proxy_async_smem();
           __syncwarp();

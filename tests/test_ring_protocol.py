@@ -12,6 +12,9 @@ Roles and barriers (one round = one K block in one stage):
     weight producer   waits empty[s]; loads the T tile onto fullA[s] or the code block onto cfull[s]
     act. producer     waits empty[s]; loads the activation tile onto fullB[s]
     decoder d         owns stages s = d (mod 4); waits cfull[s] in core rounds, arrives fullA[s]
+                      (with decoder pairs two warps own each stage, each expanding half of its
+                      rows: fullA then takes two arrivals, and the weight producer adds a plain
+                      arrival to its tile's in weight rounds)
     issuer q          owns stages s = q (mod NI); waits fullA[s], fullB[s]; commits empty[s]
 """
 import random
@@ -41,11 +44,11 @@ def wait(bar, phase, who):
         yield
 
 
-def run(seed, S, NI, follow_every_round=False):
+def run(seed, S, NI, follow_every_round=False, pairs=False):
     rnd = random.Random(seed)
     tasks = [(p, rnd.randint(0, 12)) for p in (0, 1, 2) for _ in range(rnd.randint(0, 4))]
     rounds = [p for p, n in tasks for _ in range(n)]
-    full_a = [Bar(1, f"fullA{s}") for s in range(S)]
+    full_a = [Bar(2 if pairs else 1, f"fullA{s}") for s in range(S)]
     full_b = [Bar(1, f"fullB{s}") for s in range(S)]
     empty = [Bar(1, f"empty{s}") for s in range(S)]
     cfull = [Bar(1, f"cfull{s}") for s in range(S)]
@@ -63,6 +66,8 @@ def run(seed, S, NI, follow_every_round=False):
                 yield from wait(empty[s], r // S - 1, "weight producer")
             yield from delay()
             landing.append([rnd.randint(1, 20), cfull[s] if p == 1 else full_a[s]])
+            if pairs and p != 1:
+                full_a[s].arrive()          # the producer's second arrival of a weight round
 
     def act_producer():
         for r, _ in enumerate(rounds):
@@ -72,7 +77,7 @@ def run(seed, S, NI, follow_every_round=False):
             yield from delay()
             landing.append([rnd.randint(1, 20), full_b[s]])
 
-    def decoder(d):
+    def decoder(d, half=0):
         seen = [0] * S
         for r, p in enumerate(rounds):
             s = r % S
@@ -84,7 +89,7 @@ def run(seed, S, NI, follow_every_round=False):
                     continue
             elif s % 4 != d or p != 1:
                 continue
-            yield from wait(cfull[s], seen[s], f"decoder {d}")
+            yield from wait(cfull[s], seen[s], f"decoder {d}.{half}")
             seen[s] += 1
             yield from delay()
             full_a[s].arrive()
@@ -102,6 +107,8 @@ def run(seed, S, NI, follow_every_round=False):
 
     alive = [weight_producer(), act_producer()] + [decoder(d) for d in range(4)] + \
             [issuer(q) for q in range(NI)]
+    if pairs:
+        alive += [decoder(d, 1) for d in range(4)]
     steps = 0
     while alive:
         steps += 1
@@ -127,6 +134,13 @@ def run(seed, S, NI, follow_every_round=False):
 def test_stage_owned_ring_is_exact(S, NI):
     for seed in range(150):
         run(seed, S, NI)
+
+
+# four issuers with 16 or 32 tokens run two decoder warps per stage
+@pytest.mark.parametrize("S", [12, 8, 4])
+def test_stage_owned_ring_with_decoder_pairs_is_exact(S):
+    for seed in range(150):
+        run(seed, S, 4, pairs=True)
 
 
 def test_following_every_round_can_be_lapped():
