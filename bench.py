@@ -571,8 +571,11 @@ def measure_implicit(args, fq, wl, torch, dec, stream, peaks):
                                         dev)
         Fi, Fo = fr("in", L["d_in"], L["k_in"]), fr("out", L["d_out"], L["k_out"])
         frames.append((Fi, Fo))
+        # what one forward reads: codes, scale and zero, tokens in and out, the input frame's
+        # analysis tiles and the output frame's synthesis tiles, and both rotations' factors
+        rot = lambda F: 4 * (F.c.a * F.c.a * 2 + F.c.b * F.c.b * 2) + 12 * F.c.d
         bytes_ += (L["n_out"] * L["n_in"] // 4 + 4 * L["n_out"] + 2 * M * (L["d_in"] + L["d_out"])
-                   + Fi.buf.numel() + Fo.buf.numel())
+                   + 16384 * (Fi.c.ana_count + Fo.c.syn_count) + rot(Fi) + rot(Fo))
     nb = max(fq.fq_implicit_workspace_bytes(M, L["d_in"], L["n_in"], L["n_out"], L["d_out"])
              for L in dec.layers)
     ws = torch.zeros(nb, dtype=torch.uint8, device=dev)
@@ -600,9 +603,10 @@ def measure_implicit(args, fq, wl, torch, dec, stream, peaks):
         "value": round(us, 3), "unit": UNIT, "steps": steps,
         "bytes_per_layer": round(bytes_ / len(dec.layers)),
         "hbm_frac": round(roof_us / us, 3),
-        "kernels_per_layer": 5,
-        "how": ("fq_linear_forward_implicit: rotation, run transforms (fp32, CUDA cores) and the "
-                "fused kernel's code product; frames as rotation factors and roots of unity"),
+        "kernels_per_layer": 3,
+        "how": ("fq_linear_forward_implicit: the input rotation (fp32, CUDA cores), the fused "
+                "decode kernel with block-sparse frame operands (analysis, code product and "
+                "synthesis on the tensor cores), the output rotation"),
     }
 
 

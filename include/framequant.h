@@ -345,7 +345,11 @@ fq_status fq_quantize_gptq(const double* C, int n_out, int n_in, const double* H
  * hundred KB per side instead of 2 n d bytes.
  * ---------------------------------------------------------------------------------------- */
 
-/* A frame prepared by fq_frame_implicit: device arrays inside the caller's buffer. */
+/* A frame prepared by fq_frame_implicit: device arrays inside the caller's buffer.
+ * The un-rotated operator T_u is block-diagonal; it is kept in both orientations as
+ * block-sparse tile lists: for every 128-row tile of T_u (n x d, the analysis operand) or of
+ * T_u^T (d x n, the synthesis operand), the 64-column blocks that meet the tile's runs, each a
+ * contiguous 16 KiB bf16 tile laid out as the tensor cores read it from shared memory. */
 typedef struct {
   int32_t k, rho, d;       /* (k, rho, d): rho even, d a multiple of rho, k >= d / rho */
   int32_t a, b;            /* rotation R = Pi (Q_a kron Q_b) D with a * b = d; 0, 0: R = I */
@@ -356,7 +360,12 @@ typedef struct {
   const int32_t* perm;     /* device d: (Pi v)[i] = v[perm[i]] */
   const int32_t* iperm;    /* device d: the inverse permutation */
   const float* signs;      /* device d, the diagonal of D */
-  const float* roots;      /* device 2 k: cos(2 pi m / k), sin(2 pi m / k), m = 0 .. k-1 */
+  const uint8_t* ana_tiles; /* device: the analysis operand's tiles (ana_count x 16 KiB) */
+  const int32_t* ana_idx;  /* device [ceil(n/128)][3]: first K block, end K block, first tile */
+  int32_t ana_count;
+  const uint8_t* syn_tiles; /* device: the synthesis operand's tiles (syn_count x 16 KiB) */
+  const int32_t* syn_idx;  /* device [ceil(d/128)][3], as ana_idx */
+  int32_t syn_count;
 } fq_frame;
 
 /* Bytes of the device buffer fq_frame_implicit fills (a = b = 0 without rotation); 0 for an
@@ -365,10 +374,12 @@ size_t fq_frame_implicit_bytes(int k, int rho, int d, int a, int b);
 
 /* Prepare the structured form of the (k, rho, d) frame with rotation `rot` (NULL: none), the
  * same frame fq_frame_build writes out densely.  Q_a and Q_b are computed on the host in double
- * precision (Householder QR, columns signed as in fq_rotation) and stored as fp32; the roots of
- * unity are computed on the host in double precision and stored as fp32.
+ * precision (Householder QR, columns signed as in fq_rotation) and stored as fp32; the tiles of
+ * T_u are computed on the host in double precision and stored as bf16 (rounded through fp32,
+ * like the dense operator).
  *   buf    device buffer of fq_frame_implicit_bytes(k, rho, d, rot->a, rot->b) bytes, 256-byte
- *          aligned; it must outlive every use of *out
+ *          aligned; it must outlive every use of *out (about 11 MB for (282, 16, 4096), 75 MB
+ *          for (757, 16, 11008))
  *   out    host struct receiving the sizes and the device pointers into buf
  * Synchronizes `stream` before returning.
  * Errors: FQ_ERR_INVALID_ARG (rho odd, d not a multiple of rho, k < d / rho, a bad rotation),
@@ -380,10 +391,11 @@ fq_status fq_frame_implicit(int k, int rho, int d, const fq_rotation* rot, void*
 size_t fq_implicit_workspace_bytes(int M, int d_in, int n_in, int n_out, int d_out);
 
 /* The layer forward of fq_linear_forward (Sec. 3.2) with T_in and T_out given in structured
- * form: z = T_u,in (R_in^T x), the 2-bit code product of fq_linear_forward, then
- * y = R_out (T_u,out^T u).  bf16 tokens in and out; the rotations and the run transforms are
- * computed in fp32 on CUDA cores, z and u are rounded to bf16 as in FQ_BF16, and the code
- * product runs on the tensor cores (the M <= 64 kernel of fq_linear_forward).
+ * form: v = R_in^T x, then the fused decode kernel of fq_linear_forward with block-sparse frame
+ * operands (z = T_u,in v, the 2-bit code product, s = T_u,out^T u, all on the tensor cores; the
+ * analysis and synthesis read only the tiles of each row tile's runs), then y = R_out s.  bf16
+ * tokens in and out; the rotations are computed in fp32 on CUDA cores and v, z, u and s are
+ * rounded to bf16.
  *   x      device bf16, M x F_in->d tokens;  y  device bf16, M x F_out->d
  *   F_in, F_out  host pointers to prepared frames; C->n_in = F_in->k * F_in->rho and
  *          C->n_out = F_out->k * F_out->rho
@@ -391,8 +403,9 @@ size_t fq_implicit_workspace_bytes(int M, int d_in, int n_in, int n_out, int d_o
  *   ws     device workspace of fq_implicit_workspace_bytes(...) bytes, 256-byte aligned and
  *          zero-filled before its first use (the header rules of fq_linear_forward)
  *   max_sms  as in fq_linear_forward_sms (0: the whole device)
- * Requirements: 1 <= M <= 64; for each frame d / rho <= 2560, k <= 4096 and b <= 1024 (the
- * shared-memory footprint of its kernels); sizes and alignment as in fq_linear_forward.
+ * Requirements: 1 <= M <= 64; for each frame at most 640 row tiles of 128 per orientation and,
+ * with a rotation, b <= 1024 and (d + 8 (a + b) + min(b, 128 if b <= 128 else 32) b) * 4
+ * bytes of shared memory at most 227 KiB; sizes and alignment as in fq_linear_forward.
  * Errors: FQ_ERR_INVALID_ARG, FQ_ERR_ALIGNMENT, FQ_ERR_WORKSPACE, FQ_ERR_UNSUPPORTED (M > 64, a
  * frame above those limits, device not compute capability 10.3), FQ_ERR_CUDA. */
 fq_status fq_linear_forward_implicit(const void* x, int M, const fq_frame* F_in,

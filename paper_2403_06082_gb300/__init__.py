@@ -92,7 +92,10 @@ class _Frame(ctypes.Structure):
                 ("a", ctypes.c_int32), ("b", ctypes.c_int32), ("Qa", ctypes.c_void_p),
                 ("QaT", ctypes.c_void_p), ("Qb", ctypes.c_void_p), ("QbT", ctypes.c_void_p),
                 ("perm", ctypes.c_void_p), ("iperm", ctypes.c_void_p),
-                ("signs", ctypes.c_void_p), ("roots", ctypes.c_void_p)]
+                ("signs", ctypes.c_void_p), ("ana_tiles", ctypes.c_void_p),
+                ("ana_idx", ctypes.c_void_p), ("ana_count", ctypes.c_int32),
+                ("syn_tiles", ctypes.c_void_p), ("syn_idx", ctypes.c_void_p),
+                ("syn_count", ctypes.c_int32)]
 
 
 _lib = None

@@ -102,6 +102,12 @@ struct DecPhase {
   int R, K, RT, KB, kbs;
   __nv_bfloat16* out;     // [M][R]
   uint32_t* flags;        // [RT][kWsSlices] slice final in this call when == generation + 1
+  // A block-sparse weight operand (frames in structured form), else null: row tile t reads
+  // only K blocks aidx[3t] .. aidx[3t+1]-1, stored as contiguous pre-swizzled 16 KiB tiles
+  // from tile aidx[3t+2] of atiles on
+  const uint8_t* atiles;
+  const int32_t* aidx;
+  int acount;             // stored tiles of atiles
 };
 
 // One launch runs up to kMaxGroup independent layers (no layer reads another's output), e.g.
@@ -333,9 +339,18 @@ __global__ void __launch_bounds__(DecCfg<BN>::kThreads, 1)
   pdl_launch_dependents();
 
   // this CTA's K range of a task of phase ph
-  auto krange = [&](const DecPhase& ph, int& k0, int& k1) {
-    k0 = ks * ph.kbs;
-    k1 = min(ph.KB, k0 + ph.kbs);
+  // this CTA's K range of row tile `tile` of phase ph (its own range for a block-sparse
+  // operand, split over the cluster like a dense one)
+  auto krange = [&](const DecPhase& ph, int tile, int& k0, int& k1) {
+    if (ph.aidx) {
+      const int lo = __ldg(ph.aidx + 3 * tile), hi = __ldg(ph.aidx + 3 * tile + 1);
+      const int per = (hi - lo + S - 1) / S;
+      k0 = lo + ks * per;
+      k1 = min(hi, k0 + per);
+    } else {
+      k0 = ks * ph.kbs;
+      k1 = min(ph.KB, k0 + ph.kbs);
+    }
   };
 
   if (warp == 0) {
@@ -370,7 +385,10 @@ __global__ void __launch_bounds__(DecCfg<BN>::kThreads, 1)
         const uint32_t* words = a.L[t.l].words;
         const CUtensorMap* tmA = &maps.m[t.l][t.p == 0 ? kMapTin : kMapTout];
         int k0, k1;
-        krange(ph, k0, k1);
+        krange(ph, t.tile, k0, k1);
+        // a block-sparse operand: the tile's first K block and its first stored tile
+        const int a_lo = ph.aidx ? __ldg(ph.aidx + 3 * t.tile) : 0;
+        const int a_off = ph.aidx ? __ldg(ph.aidx + 3 * t.tile + 2) : 0;
         if (next_pf && t.p == 2) prefetch_next();
         if (tout_pf && t.p >= 1) {
           tout_pf = false;
@@ -381,13 +399,22 @@ __global__ void __launch_bounds__(DecCfg<BN>::kThreads, 1)
             if (u.p != 2 || !a.L[u.l].pf_tout) continue;
             const DecPhase q = phase_of(a, u.l, u.p);
             int u0, u1;
-            krange(q, u0, u1);
-            for (int kb = u0; kb < u1; ++kb)
-              asm volatile(
-                  "cp.async.bulk.prefetch.tensor.2d.L2.global.tile [%0, {%1, %2}];" ::"l"(
-                      reinterpret_cast<uint64_t>(&maps.m[u.l][kMapTout])),
-                  "r"(kb * kBK), "r"(u.tile * kBM)
-                  : "memory");
+            krange(q, u.tile, u0, u1);
+            if (q.atiles) {
+              const int lo = __ldg(q.aidx + 3 * u.tile), off = __ldg(q.aidx + 3 * u.tile + 2);
+              if (u1 > u0)
+                asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(
+                                 q.atiles + static_cast<int64_t>(off + u0 - lo) * kATile),
+                             "r"(static_cast<uint32_t>((u1 - u0) * kATile))
+                             : "memory");
+            } else {
+              for (int kb = u0; kb < u1; ++kb)
+                asm volatile(
+                    "cp.async.bulk.prefetch.tensor.2d.L2.global.tile [%0, {%1, %2}];" ::"l"(
+                        reinterpret_cast<uint64_t>(&maps.m[u.l][kMapTout])),
+                    "r"(kb * kBK), "r"(u.tile * kBM)
+                    : "memory");
+            }
           }
         }
         for (int kb = k0; kb < k1; ++kb) {
@@ -416,8 +443,13 @@ __global__ void __launch_bounds__(DecCfg<BN>::kThreads, 1)
             if (lane == 0) {
               mbar_arrive_expect_tx(&fullA[stage], kATile);
               if (DecCfg<BN>::kPairs) mbar_arrive(&fullA[stage]);
-              tma_load_2d(sA + stage * kATile, tmA, &fullA[stage], kb * kBK, t.tile * kBM,
-                          pol_w);
+              if (ph.atiles)
+                bulk_load(sA + stage * kATile,
+                          ph.atiles + static_cast<int64_t>(a_off + kb - a_lo) * kATile, kATile,
+                          &fullA[stage], pol_w);
+              else
+                tma_load_2d(sA + stage * kATile, tmA, &fullA[stage], kb * kBK, t.tile * kBM,
+                            pol_w);
             }
             last_code &= ~bit;
             last_par = (last_par & ~bit) | (phase << stage);
@@ -431,7 +463,7 @@ __global__ void __launch_bounds__(DecCfg<BN>::kThreads, 1)
             const Task u = task_at(sched, j);
             const DecPhase q = phase_of(a, u.l, u.p);
             int u0, u1;
-            krange(q, u0, u1);
+            krange(q, u.tile, u0, u1);
             if (u.p == 1 && u1 > u0) {
               const uint32_t* src =
                   a.L[u.l].words + (static_cast<int64_t>(u.tile) * q.KB + u0) * 512;
@@ -473,7 +505,7 @@ __global__ void __launch_bounds__(DecCfg<BN>::kThreads, 1)
       const Task t = task_at(sched, i);
       const DecPhase ph = phase_of(a, t.l, t.p);
       int k0, k1;
-      krange(ph, k0, k1);
+      krange(ph, t.tile, k0, k1);
       // Loads go out in K order as soon as the slices of the previous phase's output that a K
       // block reads are final: the lanes poll the not-yet-final slices of the K range, and
       // the ready prefix decides how far lane 0 may issue.
@@ -553,7 +585,7 @@ __global__ void __launch_bounds__(DecCfg<BN>::kThreads, 1)
         const Task t = task_at(sched, i);
         const DecPhase ph = phase_of(a, t.l, t.p);
         int k0, k1;
-        krange(ph, k0, k1);
+        krange(ph, t.tile, k0, k1);
         if (!mbar_wait(&tempty[buf], acc_phase ^ 1, abort_flag)) {
           if (!*abort_flag) note_timeout(a.status, 4, i, buf, static_cast<int>(acc_phase));
           *abort_flag = 1;
@@ -613,7 +645,7 @@ __global__ void __launch_bounds__(DecCfg<BN>::kThreads, 1)
       const Task t = task_at(sched, i);
       const DecPhase ph = phase_of(a, t.l, t.p);
       int k0, k1;
-      krange(ph, k0, k1);
+      krange(ph, t.tile, k0, k1);
       const int n = max(0, k1 - k0);
       if (t.p != 1) {
         stage = (stage + n) % S_;
@@ -671,7 +703,7 @@ __global__ void __launch_bounds__(DecCfg<BN>::kThreads, 1)
       const __half* l_zero = a.L[t.l].zero;
       const float* l_gamma = a.L[t.l].gamma;
       int k0, k1;
-      krange(ph, k0, k1);
+      krange(ph, t.tile, k0, k1);
       const bool has_k = k1 > k0;
       const int row = t.tile * kBM + r_in_tile;
       const bool row_ok = row < ph.R;
@@ -1089,7 +1121,9 @@ fq_status run(const DecMaps& maps, DecArgs& a, const std::vector<Block>& blocks,
     int64_t warm = code_bytes;
     bool any_tout = false;
     for (int l = 0; l < a.G; ++l) {
-      warm += static_cast<int64_t>(a.L[l].ph[2].R) * a.L[l].ph[2].K * 2;
+      const DecPhase& sy = a.L[l].ph[2];
+      warm += sy.atiles ? static_cast<int64_t>(sy.acount) * kATile
+                        : static_cast<int64_t>(sy.R) * sy.K * 2;
       a.L[l].pf_tout = a.L[l].ph[2].R > 0 && warm <= kL2PrefetchBudget;
       any_tout |= a.L[l].pf_tout != 0;
     }
@@ -1168,7 +1202,7 @@ fq_status launch_decode_group(int M, int G, const DecGroupLayer* Ls, char* ws, s
   DecArgs a{};
   a.M = M;
   a.G = G;
-  int R[kMaxGroup][3], K[kMaxGroup][3];
+  int R[kMaxGroup][3], K[kMaxGroup][3], Keff[kMaxGroup][3];
   uint32_t* flag_base = reinterpret_cast<uint32_t*>(ws + kWsFlags);
   const int64_t flag_words = static_cast<int64_t>(kWsHeader - kWsFlags) / 4;
   int64_t flag_off = 0;
@@ -1179,15 +1213,24 @@ fq_status launch_decode_group(int M, int G, const DecGroupLayer* Ls, char* ws, s
     const int Rl[3] = {core_only ? 0 : n_in, n_out, core_only ? 0 : Ly.d_out};
     const int Kl[3] = {core_only ? 0 : Ly.d_in, n_in, core_only ? 0 : n_out};
     void* outs[3] = {ws + W.z[l], ws + W.u[l], core_only ? static_cast<void*>(ws + W.u[l]) : Ly.y};
+    const SparseOperand* sp[3] = {&Ly.tin, nullptr, &Ly.tout};
     for (int p = 0; p < 3; ++p) {
       R[l][p] = Rl[p];
       K[l][p] = Kl[p];
+      Keff[l][p] = Kl[p];
       const int RT = static_cast<int>(ceil_div(Rl[p], kBM));
       if (RT > kWsMaxTiles || RT >= (1 << kTileBits)) return FQ_ERR_UNSUPPORTED;
       DecPhase& ph = a.L[l].ph[p];
       ph.R = Rl[p];
       ph.K = Kl[p];
       ph.out = static_cast<__nv_bfloat16*>(outs[p]);
+      if (sp[p] && sp[p]->tiles && Rl[p] > 0) {
+        ph.atiles = sp[p]->tiles;
+        ph.aidx = sp[p]->idx;
+        ph.acount = sp[p]->count;
+        // the cost model's K: the operand's stored K blocks per row tile
+        Keff[l][p] = static_cast<int>(ceil_div(static_cast<int64_t>(sp[p]->count) * kBK, RT));
+      }
       if (G == 1) {
         // one layer: the phases' flags at fixed places of the header
         ph.flags = flag_base + p * kWsMaxTiles * kWsSlices;
@@ -1215,10 +1258,17 @@ fq_status launch_decode_group(int M, int G, const DecGroupLayer* Ls, char* ws, s
       m[kMapTin] = m[kMapZ];
       m[kMapX] = m[kMapZ];
       m[kMapTout] = m[kMapU];
-    } else if (!tmap_bf16(&m[kMapTin], Ly.T_in, n_in, Ly.d_in, kBM) ||
-               !tmap_bf16(&m[kMapX], Ly.x, M, Ly.d_in, BN) ||
-               !tmap_bf16(&m[kMapTout], Ly.T_out_t, Ly.d_out, n_out, kBM)) {
-      return FQ_ERR_CUDA;
+    } else {
+      // block-sparse operands are copied whole tiles at a time: their maps are never used
+      if (!tmap_bf16(&m[kMapX], Ly.x, M, Ly.d_in, BN)) return FQ_ERR_CUDA;
+      if (Ly.tin.tiles)
+        m[kMapTin] = m[kMapX];
+      else if (!tmap_bf16(&m[kMapTin], Ly.T_in, n_in, Ly.d_in, kBM))
+        return FQ_ERR_CUDA;
+      if (Ly.tout.tiles)
+        m[kMapTout] = m[kMapU];
+      else if (!tmap_bf16(&m[kMapTout], Ly.T_out_t, Ly.d_out, n_out, kBM))
+        return FQ_ERR_CUDA;
     }
   }
   for (int l = G; l < kMaxGroup; ++l)
@@ -1230,7 +1280,7 @@ fq_status launch_decode_group(int M, int G, const DecGroupLayer* Ls, char* ws, s
   a.pf_next = static_cast<const char*>(pf);
   a.pf_next_bytes = pf ? static_cast<int64_t>(pf_bytes) : 0;
   a.inject_wait = inject_wait;
-  const std::vector<Block> blocks = launch_order(G, R, K);
+  const std::vector<Block> blocks = launch_order(G, R, Keff);
   switch (BN) {
     case 16: return run<16>(maps, a, blocks, sms, budget, s);
     case 32: return run<32>(maps, a, blocks, sms, budget, s);

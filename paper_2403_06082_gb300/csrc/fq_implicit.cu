@@ -5,25 +5,24 @@
 // c = j w .. (j+1) w - 1 (w = d / rho; complex coordinate c is real coordinates 2c, 2c + 1), and
 // its k frame vectors are the realified rows of exp(2 pi i k_i c / k) / sqrt(k).  The rotated
 // frame is T = T_u R^T, R = Pi (Q_a kron Q_b) D (Appendix K), so
-//     analysis   z = T_u (R^T x):   z_(j,k_i) = k^-1/2 sum_c exp(-2 pi i k_i c / k) v_c
-//     synthesis  y = R (T_u^T u):   y_c = k^-1/2 sum_(k_i) exp(+2 pi i k_i c / k) u_(j,k_i)
-// with complex pairs (real part at the even row or coordinate, imaginary at the odd one).
+//     z = T_u (R^T x),        y = R (T_u^T u).
 //
-// One forward is five kernels chained with programmatic dependent launch:
-//   rotate<analysis>   v = R_in^T x        (fp32, workspace)
-//   run_analysis       z = T_u,in v        (bf16, the fused decode kernel's z slot)
-//   decode core        u = gamma (C_hat z) (the fused decode kernel with its code product only)
-//   run_synthesis      s = T_u,out^T u     (fp32, workspace)
-//   rotate<synthesis>  y = R_out s         (bf16)
-// The rotations and run transforms are fp32 on CUDA cores: at decode batch sizes they are a few
-// MFLOP per token, while the dense operators they replace are 2 n d bytes of HBM traffic.
-// Each kernel triggers its dependents at entry, stages its constant inputs (roots of unity,
-// rotation rows), and waits for its predecessor before touching the workspace or its input.
+// One forward is three kernels chained with programmatic dependent launch:
+//   rotate<analysis>   v = R_in^T x   (bf16)
+//   the fused decode kernel with block-sparse frame operands: z = T_u,in v, the 2-bit code
+//                      product, s = T_u,out^T u, all on the tensor cores (its analysis and
+//                      synthesis read only the K blocks of each row tile's runs, stored as
+//                      contiguous pre-swizzled 16 KiB tiles: about 1/8 of the dense operator
+//                      for rho = 16)
+//   rotate<synthesis>  y = R_out s   (bf16)
+// Without a rotation the fused kernel reads x and writes y itself.  The rotations are two small
+// products per token on CUDA cores (a x a and b x b with a b = d).
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
 
 #include <algorithm>
 #include <cmath>
+#include <cstring>
 #include <mutex>
 #include <set>
 #include <vector>
@@ -34,25 +33,24 @@
 namespace fq {
 namespace {
 
-constexpr int kRunWarps = 8;       // warps of a run-transform CTA: segments of the reduction
-constexpr int kRunTokens = 8;      // tokens per run-transform CTA
-constexpr int kMaxRotRows = 8;     // rows of the a x b rotated block per rotation CTA
-constexpr int kMaxRunW = 2560;     // complex coordinates per run
-constexpr int kMaxK = 4096;        // frame vectors per run
 
 // ------------------------------------------------------------------------------ rotations
 // CTA (token t, rows r0 .. r0 + G - 1 of the a x b block); thread c < b owns column c
-// (b <= 1024; the CTA has at least 256 threads for the loads).
+// (b <= 1024; the CTA has at least 256 threads for the loads).  bf16 in and out.
 //   analysis:  V = Pi^T x (V[perm[i]] = x_i), Y = Q_a^T V Q_b, out = D vec(Y)      A = Q_a^T, B = Q_b
 //   synthesis: V = D s, Y = Q_a V Q_b^T, out = Pi vec(Y) (out[iperm[e]] = vec(Y)_e) A = Q_a, B = Q_b^T
-// B is staged through shared memory kRotChunk rows at a time (coalesced loads, all in flight
-// together), so no thread waits on a chain of dependent L2 loads.
+// The factors do not depend on the previous kernel: A's rows, and all of B when it fits
+// (b <= kRotWholeB), are staged in shared memory before the wait for the input; a larger B is
+// staged kRotChunk rows at a time (coalesced loads, all in flight together).
+constexpr int kMaxRotRows = 8;     // rows of the a x b rotated block per rotation CTA
 constexpr int kRotChunk = 32;
+constexpr int kRotWholeB = 128;
 
 template <bool kSynth>
-__global__ void __launch_bounds__(1024) rotate_kernel(const void* __restrict__ in,
-                                                      void* __restrict__ out, int d, int a,
-                                                      int b, int G, const float* __restrict__ A,
+__global__ void __launch_bounds__(1024) rotate_kernel(const __nv_bfloat16* __restrict__ in,
+                                                      __nv_bfloat16* __restrict__ out, int d,
+                                                      int a, int b, int G,
+                                                      const float* __restrict__ A,
                                                       const float* __restrict__ B,
                                                       const int32_t* __restrict__ perm,
                                                       const int32_t* __restrict__ iperm,
@@ -61,28 +59,32 @@ __global__ void __launch_bounds__(1024) rotate_kernel(const void* __restrict__ i
   float* V = sm;                    // [d]
   float* Ar = V + d;                // [G][a]
   float* T1 = Ar + G * a;           // [G][b]
-  float* Bs = T1 + G * b;           // [kRotChunk][b]
+  float* Bs = T1 + G * b;           // [b][b] when b <= kRotWholeB, else [kRotChunk][b]
   const int t = blockIdx.y, r0 = blockIdx.x * G, nt = blockDim.x;
   const int rows = min(G, a - r0);
   const int c = threadIdx.x;
   const bool col = c < b;
+  const bool whole_b = b <= kRotWholeB;
   pdl_launch_dependents();
   for (int i = threadIdx.x; i < rows * a; i += nt) Ar[i] = A[static_cast<int64_t>(r0) * a + i];
+  if (whole_b)
+#pragma unroll 8
+    for (int i = threadIdx.x; i < b * b; i += nt) Bs[i] = B[i];
   pdl_wait();
+  const __nv_bfloat16* src = in + static_cast<int64_t>(t) * d;
   if (kSynth) {
-    const float* s = static_cast<const float*>(in) + static_cast<int64_t>(t) * d;
 #pragma unroll 8
-    for (int i = threadIdx.x; i < d; i += nt) V[i] = signs[i] * s[i];
+    for (int i = threadIdx.x; i < d; i += nt) V[i] = signs[i] * __bfloat162float(src[i]);
   } else {
-    const __nv_bfloat16* x = static_cast<const __nv_bfloat16*>(in) + static_cast<int64_t>(t) * d;
 #pragma unroll 8
-    for (int i = threadIdx.x; i < d; i += nt) V[perm[i]] = __bfloat162float(x[i]);
+    for (int i = threadIdx.x; i < d; i += nt) V[perm[i]] = __bfloat162float(src[i]);
   }
   __syncthreads();
   float acc[kMaxRotRows];
 #pragma unroll
   for (int g = 0; g < kMaxRotRows; ++g) acc[g] = 0.f;
   if (col) {
+#pragma unroll 4
     for (int r = 0; r < a; ++r) {
       const float v = V[r * b + c];
 #pragma unroll
@@ -95,15 +97,20 @@ __global__ void __launch_bounds__(1024) rotate_kernel(const void* __restrict__ i
   }
 #pragma unroll
   for (int g = 0; g < kMaxRotRows; ++g) acc[g] = 0.f;
-  for (int k0 = 0; k0 < b; k0 += kRotChunk) {
-    const int kn = min(kRotChunk, b - k0);
+  const int chunk = whole_b ? b : kRotChunk;
+  for (int k0 = 0; k0 < b; k0 += chunk) {
+    const int kn = min(chunk, b - k0);
     __syncthreads();            // T1 written (first chunk), the previous chunk consumed
+    if (!whole_b) {
 #pragma unroll 8
-    for (int i = threadIdx.x; i < kn * b; i += nt) Bs[i] = B[static_cast<int64_t>(k0) * b + i];
-    __syncthreads();
+      for (int i = threadIdx.x; i < kn * b; i += nt) Bs[i] = B[static_cast<int64_t>(k0) * b + i];
+      __syncthreads();
+    }
+    const float* Bk = whole_b ? Bs + static_cast<int64_t>(k0) * b : Bs;
     if (col) {
+#pragma unroll 4
       for (int kk = 0; kk < kn; ++kk) {
-        const float w = Bs[kk * b + c];
+        const float w = Bk[kk * b + c];
 #pragma unroll
         for (int g = 0; g < kMaxRotRows; ++g)
           if (g < rows) acc[g] = fmaf(T1[g * b + k0 + kk], w, acc[g]);
@@ -111,171 +118,108 @@ __global__ void __launch_bounds__(1024) rotate_kernel(const void* __restrict__ i
     }
   }
   if (!col) return;
+  __nv_bfloat16* dst = out + static_cast<int64_t>(t) * d;
 #pragma unroll
   for (int g = 0; g < kMaxRotRows; ++g) {
     if (g >= rows) continue;
     const int e = (r0 + g) * b + c;
-    if (kSynth) {
-      static_cast<__nv_bfloat16*>(out)[static_cast<int64_t>(t) * d + iperm[e]] =
-          __float2bfloat16_rn(acc[g]);
-    } else {
-      static_cast<float*>(out)[static_cast<int64_t>(t) * d + e] = signs[e] * acc[g];
-    }
-  }
-}
-
-// Without a rotation: a copy that converts (bf16 -> fp32 for the analysis, fp32 -> bf16 for the
-// synthesis).
-template <bool kSynth>
-__global__ void __launch_bounds__(256) copy_kernel(const void* __restrict__ in,
-                                                   void* __restrict__ out, int64_t n) {
-  pdl_launch_dependents();
-  pdl_wait();
-  for (int64_t i = blockIdx.x * 256ll + threadIdx.x; i < n; i += gridDim.x * 256ll) {
     if (kSynth)
-      static_cast<__nv_bfloat16*>(out)[i] = __float2bfloat16_rn(static_cast<const float*>(in)[i]);
+      dst[iperm[e]] = __float2bfloat16_rn(acc[g]);
     else
-      static_cast<float*>(out)[i] = __bfloat162float(static_cast<const __nv_bfloat16*>(in)[i]);
-  }
-}
-
-// -------------------------------------------------------------------------- run transforms
-// Analysis of run j for frame vectors k_i = kc .. kc + 31 (lane) and tokens t0 .. t0 + 7: warp q
-// sums over its segment of the run's w complex coordinates, the segments are added in warp
-// order.  The root index (k_i c) mod k advances by k_i per coordinate.
-__global__ void __launch_bounds__(kRunWarps * 32) run_analysis_kernel(
-    const float* __restrict__ v, __nv_bfloat16* __restrict__ z, int M, int d, int n, int k,
-    int w, int kchunks, float rk, const float2* __restrict__ roots) {
-  extern __shared__ float sm[];
-  float2* rt = reinterpret_cast<float2*>(sm);                     // [k]
-  float2* xs = rt + k;                                            // [kRunTokens][w]
-  float2* red = xs + kRunTokens * w;                              // [warps][tokens][32]
-  const int j = blockIdx.x / kchunks, kc = (blockIdx.x % kchunks) * 32;
-  const int t0 = blockIdx.y * kRunTokens, nt = min(kRunTokens, M - t0);
-  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  pdl_launch_dependents();
-#pragma unroll 4
-  for (int i = threadIdx.x; i < k; i += blockDim.x) rt[i] = roots[i];
-  pdl_wait();
-#pragma unroll 8
-  for (int i = threadIdx.x; i < kRunTokens * w; i += blockDim.x) {
-    const int tt = i / w, c = i % w;
-    xs[i] = tt < nt ? *reinterpret_cast<const float2*>(
-                          v + static_cast<int64_t>(t0 + tt) * d + 2 * (static_cast<int64_t>(j) * w + c))
-                    : make_float2(0.f, 0.f);
-  }
-  __syncthreads();
-  const int ki = kc + lane;
-  const int seg = (w + kRunWarps - 1) / kRunWarps;
-  const int c0 = warp * seg, c1 = min(w, c0 + seg);
-  float re[kRunTokens], im[kRunTokens];
-#pragma unroll
-  for (int tt = 0; tt < kRunTokens; ++tt) re[tt] = im[tt] = 0.f;
-  if (ki < k && c0 < c1) {
-    int idx = static_cast<int>((static_cast<int64_t>(ki) * (static_cast<int64_t>(j) * w + c0)) % k);
-    for (int c = c0; c < c1; ++c) {
-      const float2 r = rt[idx];
-#pragma unroll
-      for (int tt = 0; tt < kRunTokens; ++tt) {
-        const float2 x = xs[tt * w + c];
-        re[tt] = fmaf(x.x, r.x, fmaf(x.y, r.y, re[tt]));
-        im[tt] = fmaf(x.y, r.x, fmaf(-x.x, r.y, im[tt]));
-      }
-      idx += ki;
-      if (idx >= k) idx -= k;
-    }
-  }
-#pragma unroll
-  for (int tt = 0; tt < kRunTokens; ++tt)
-    red[(warp * kRunTokens + tt) * 32 + lane] = make_float2(re[tt], im[tt]);
-  __syncthreads();
-  for (int i = threadIdx.x; i < kRunTokens * 32; i += blockDim.x) {
-    const int tt = i / 32, l = i % 32, kk = kc + l;
-    if (tt >= nt || kk >= k) continue;
-    float sr = 0.f, si = 0.f;
-    for (int q = 0; q < kRunWarps; ++q) {
-      const float2 p = red[(q * kRunTokens + tt) * 32 + l];
-      sr += p.x;
-      si += p.y;
-    }
-    *reinterpret_cast<__nv_bfloat162*>(z + static_cast<int64_t>(t0 + tt) * n +
-                                        2 * (static_cast<int64_t>(j) * k + kk)) =
-        __floats2bfloat162_rn(sr * rk, si * rk);
-  }
-}
-
-// Synthesis of run j for complex coordinates c = j w + cc .. + 31 (lane) and tokens t0 .. t0 + 7:
-// warp q sums over its segment of the k frame vectors; the root index (k_i c) mod k advances by
-// c mod k per frame vector.
-__global__ void __launch_bounds__(kRunWarps * 32) run_synthesis_kernel(
-    const __nv_bfloat16* __restrict__ u, float* __restrict__ s, int M, int d, int n, int k,
-    int w, int cchunks, float rk, const float2* __restrict__ roots) {
-  extern __shared__ float sm[];
-  float2* rt = reinterpret_cast<float2*>(sm);                             // [k]
-  float2* red = rt + k;                                                   // [warps][tokens][32]
-  __nv_bfloat162* us = reinterpret_cast<__nv_bfloat162*>(red + kRunWarps * kRunTokens * 32);  // [tokens][k]
-  const int j = blockIdx.x / cchunks, cc = (blockIdx.x % cchunks) * 32;
-  const int t0 = blockIdx.y * kRunTokens, nt = min(kRunTokens, M - t0);
-  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  pdl_launch_dependents();
-#pragma unroll 4
-  for (int i = threadIdx.x; i < k; i += blockDim.x) rt[i] = roots[i];
-  pdl_wait();
-#pragma unroll 8
-  for (int i = threadIdx.x; i < kRunTokens * k; i += blockDim.x) {
-    const int tt = i / k, q = i % k;
-    us[i] = tt < nt ? *reinterpret_cast<const __nv_bfloat162*>(
-                          u + static_cast<int64_t>(t0 + tt) * n + 2 * (static_cast<int64_t>(j) * k + q))
-                    : __floats2bfloat162_rn(0.f, 0.f);
-  }
-  __syncthreads();
-  const int c = cc + lane;                       // complex coordinate within the run
-  const int seg = (k + kRunWarps - 1) / kRunWarps;
-  const int q0 = warp * seg, q1 = min(k, q0 + seg);
-  float yr[kRunTokens], yi[kRunTokens];
-#pragma unroll
-  for (int tt = 0; tt < kRunTokens; ++tt) yr[tt] = yi[tt] = 0.f;
-  if (c < w && q0 < q1) {
-    const int64_t cabs = static_cast<int64_t>(j) * w + c;
-    const int step = static_cast<int>(cabs % k);
-    int idx = static_cast<int>((static_cast<int64_t>(q0) * cabs) % k);
-    for (int q = q0; q < q1; ++q) {
-      const float2 r = rt[idx];
-#pragma unroll
-      for (int tt = 0; tt < kRunTokens; ++tt) {
-        const float2 p = __bfloat1622float2(us[tt * k + q]);
-        yr[tt] = fmaf(p.x, r.x, fmaf(-p.y, r.y, yr[tt]));
-        yi[tt] = fmaf(p.y, r.x, fmaf(p.x, r.y, yi[tt]));
-      }
-      idx += step;
-      if (idx >= k) idx -= k;
-    }
-  }
-#pragma unroll
-  for (int tt = 0; tt < kRunTokens; ++tt)
-    red[(warp * kRunTokens + tt) * 32 + lane] = make_float2(yr[tt], yi[tt]);
-  __syncthreads();
-  for (int i = threadIdx.x; i < kRunTokens * 32; i += blockDim.x) {
-    const int tt = i / 32, l = i % 32, cl = cc + l;
-    if (tt >= nt || cl >= w) continue;
-    float sr = 0.f, si = 0.f;
-    for (int q = 0; q < kRunWarps; ++q) {
-      const float2 p = red[(q * kRunTokens + tt) * 32 + l];
-      sr += p.x;
-      si += p.y;
-    }
-    *reinterpret_cast<float2*>(s + static_cast<int64_t>(t0 + tt) * d +
-                               2 * (static_cast<int64_t>(j) * w + cl)) =
-        make_float2(sr * rk, si * rk);
+      dst[e] = __float2bfloat16_rn(signs[e] * acc[g]);
   }
 }
 
 // ------------------------------------------------------------------------------ host side
-struct FrameBuf {
-  size_t Qa, QaT, Qb, QbT, perm, iperm, signs, roots, total;
+constexpr int kTR = 128, kTK = 64;            // operand tile: 128 rows x 64 bf16 (16 KiB)
+constexpr int kTileBytes = kTR * kTK * 2;
+
+// The row tiles of a block-sparse frame operand and the K blocks each one touches.
+//   analysis  (T_u, n x d):   row tile t covers frame rows [128 t, +128); run j owns frame rows
+//             [2 k j, 2 k (j+1)) and real coordinates [2 w j, 2 w (j+1)) (the K range)
+//   synthesis (T_u^T, d x n): row tile t covers coordinates [128 t, +128); run j owns them in
+//             [2 w j, 2 w (j+1)) and frame rows [2 k j, 2 k (j+1)) (the K range)
+struct SparseShape {
+  int rows, cols, RT, KB;
+  int run_rows, run_cols;        // rows and columns of one run in this orientation
+  std::vector<int32_t> idx;      // [RT][3]: kb_lo, kb_hi, first stored tile
+  int count = 0;
 };
 
-FrameBuf frame_buf(int k, int d, int a, int b) {
+SparseShape sparse_shape(int k, int rho, int d, bool synthesis) {
+  const int n = k * rho, w = d / rho;
+  SparseShape S;
+  S.rows = synthesis ? d : n;
+  S.cols = synthesis ? n : d;
+  S.run_rows = synthesis ? 2 * w : 2 * k;
+  S.run_cols = synthesis ? 2 * k : 2 * w;
+  S.RT = static_cast<int>(ceil_div(S.rows, kTR));
+  S.KB = static_cast<int>(ceil_div(S.cols, kTK));
+  S.idx.resize(3 * static_cast<size_t>(S.RT));
+  for (int t = 0; t < S.RT; ++t) {
+    const int r0 = t * kTR, r1 = std::min(S.rows, r0 + kTR);
+    const int j0 = r0 / S.run_rows, j1 = (r1 - 1) / S.run_rows;
+    const int lo = static_cast<int>((static_cast<int64_t>(j0) * S.run_cols) / kTK);
+    const int hi = static_cast<int>(std::min<int64_t>(
+        S.KB, ceil_div(static_cast<int64_t>(j1 + 1) * S.run_cols, kTK)));
+    S.idx[3 * t] = lo;
+    S.idx[3 * t + 1] = hi;
+    S.idx[3 * t + 2] = S.count;
+    S.count += hi - lo;
+  }
+  return S;
+}
+
+// bf16 bit pattern of a float, rounding to nearest even (the operands are finite)
+uint16_t bf16_bits(float f) {
+  uint32_t u;
+  std::memcpy(&u, &f, 4);
+  u += 0x7FFFu + ((u >> 16) & 1u);
+  return static_cast<uint16_t>(u >> 16);
+}
+
+// The stored tiles of one orientation: entry (r, c) of the un-rotated analysis operator is,
+// for frame row r = 2 (j k + k_i) + e and real coordinate c = 2 q + f with q in run j,
+// v = exp(2 pi i k_i q / k) / sqrt(k) realified as (e, f) = (0,0) Re v, (0,1) Im v,
+// (1,0) -Im v, (1,1) Re v (Appendix J; 0 outside the run), computed in double, rounded to fp32
+// and then to bf16 like the dense operator.  Each tile is written in the 128-byte-swizzled
+// shared-memory image of a K-major 128 x 64 tile: row r's 16-byte chunk h at chunk h ^ (r mod 8).
+void fill_tiles(int k, int rho, int d, const SparseShape& S, bool synthesis,
+                const std::vector<double>& cs, const std::vector<double>& sn,
+                std::vector<uint16_t>& out) {
+  const int w = d / rho;
+  const double rk = 1.0 / std::sqrt(static_cast<double>(k));
+  out.assign(static_cast<size_t>(S.count) * kTR * kTK, 0);
+  for (int t = 0; t < S.RT; ++t) {
+    const int lo = S.idx[3 * t], hi = S.idx[3 * t + 1], first = S.idx[3 * t + 2];
+    for (int kb = lo; kb < hi; ++kb) {
+      uint16_t* tile = out.data() + static_cast<size_t>(first + kb - lo) * kTR * kTK;
+      for (int r = 0; r < kTR; ++r) {
+        const int gr = t * kTR + r;
+        if (gr >= S.rows) continue;
+        for (int cc = 0; cc < kTK; ++cc) {
+          const int gc = kb * kTK + cc;
+          if (gc >= S.cols) continue;
+          const int frow = synthesis ? gc : gr, coord = synthesis ? gr : gc;
+          const int b2 = frow >> 1, e = frow & 1, f = coord & 1, q = coord >> 1;
+          const int j = b2 / k, ki = b2 % k;
+          if (q < j * w || q >= (j + 1) * w) continue;
+          const int m = static_cast<int>((static_cast<int64_t>(ki) * q) % k);
+          const double re = cs[m] * rk, im = sn[m] * rk;
+          const double v = e == 0 ? (f == 0 ? re : im) : (f == 0 ? -im : re);
+          const int pos = r * kTK + ((((cc >> 3) ^ (r & 7)) << 3) | (cc & 7));
+          tile[pos] = bf16_bits(static_cast<float>(v));
+        }
+      }
+    }
+  }
+}
+
+struct FrameBuf {
+  size_t Qa, QaT, Qb, QbT, perm, iperm, signs, ana_tiles, ana_idx, syn_tiles, syn_idx, total;
+};
+
+FrameBuf frame_buf(int k, int rho, int d, int a, int b) {
   FrameBuf L{};
   size_t off = 0;
   auto take = [&](size_t bytes) {
@@ -291,7 +235,11 @@ FrameBuf frame_buf(int k, int d, int a, int b) {
   L.perm = take(static_cast<size_t>(d) * 4);
   L.iperm = take(static_cast<size_t>(d) * 4);
   L.signs = take(static_cast<size_t>(d) * 4);
-  L.roots = take(static_cast<size_t>(k) * 8);
+  const SparseShape A = sparse_shape(k, rho, d, false), S = sparse_shape(k, rho, d, true);
+  L.ana_tiles = take(static_cast<size_t>(A.count) * kTileBytes);
+  L.ana_idx = take(A.idx.size() * 4);
+  L.syn_tiles = take(static_cast<size_t>(S.count) * kTileBytes);
+  L.syn_idx = take(S.idx.size() * 4);
   L.total = off;
   return L;
 }
@@ -301,7 +249,10 @@ bool valid_triple(int k, int rho, int d) {
 }
 
 bool valid_frame(const fq_frame* f) {
-  if (!f || !valid_triple(f->k, f->rho, f->d) || !f->roots) return false;
+  if (!f || !valid_triple(f->k, f->rho, f->d)) return false;
+  if (!f->ana_tiles || !f->ana_idx || !f->syn_tiles || !f->syn_idx || f->ana_count <= 0 ||
+      f->syn_count <= 0)
+    return false;
   if (f->a == 0 && f->b == 0) return true;
   return f->a > 0 && f->b > 0 && static_cast<int64_t>(f->a) * f->b == f->d && f->Qa && f->QaT &&
          f->Qb && f->QbT && f->perm && f->iperm && f->signs;
@@ -310,42 +261,34 @@ bool valid_frame(const fq_frame* f) {
 bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 
 struct ImplWs {
-  size_t z, u, v, s, total;
+  size_t v, s, total, group;
 };
 
+// the fused kernel's workspace (header, z, u), then the rotated tokens and the un-rotated output
 ImplWs impl_ws(int M, int d_in, int n_in, int n_out, int d_out) {
   ImplWs L{};
-  L.z = decode_core_z_offset();
-  L.u = decode_core_u_offset(M, n_in);
   size_t off = decode_workspace_bytes(M, d_in, n_in, n_out, d_out);
+  L.group = off;
   L.v = off;
-  off += static_cast<size_t>(round_up(static_cast<int64_t>(M) * d_in * 4, 256));
+  off += static_cast<size_t>(round_up(static_cast<int64_t>(M) * d_in * 2, 256));
   L.s = off;
-  off += static_cast<size_t>(round_up(static_cast<int64_t>(M) * d_out * 4, 256));
+  off += static_cast<size_t>(round_up(static_cast<int64_t>(M) * d_out * 2, 256));
   L.total = off;
   return L;
 }
 
 size_t rot_smem(const fq_frame& f, int G) {
-  return (static_cast<size_t>(f.d) + static_cast<size_t>(G) * (f.a + f.b) +
-          static_cast<size_t>(kRotChunk) * f.b) * 4;
-}
-size_t ana_smem(const fq_frame& f) {
-  const int w = f.d / f.rho;
-  return (static_cast<size_t>(f.k) + kRunTokens * w + kRunWarps * kRunTokens * 32) * 8;
-}
-size_t syn_smem(const fq_frame& f) {
-  return (static_cast<size_t>(f.k) + kRunWarps * kRunTokens * 32) * 8 +
-         static_cast<size_t>(kRunTokens) * f.k * 4;
+  const size_t brows = f.b <= kRotWholeB ? static_cast<size_t>(f.b) : kRotChunk;
+  return (static_cast<size_t>(f.d) + static_cast<size_t>(G) * (f.a + f.b) + brows * f.b) * 4;
 }
 
 constexpr size_t kMaxSmem = 227 * 1024;
 
 bool frame_fits(const fq_frame& f) {
-  const int w = f.d / f.rho;
-  if (w > kMaxRunW || f.k > kMaxK) return false;
-  if (f.a > 0 && (f.b > 1024 || rot_smem(f, kMaxRotRows) > kMaxSmem)) return false;
-  return ana_smem(f) <= kMaxSmem && syn_smem(f) <= kMaxSmem;
+  if (ceil_div(static_cast<int64_t>(f.k) * f.rho, kTR) > kWsMaxTiles ||
+      ceil_div(f.d, kTR) > kWsMaxTiles)
+    return false;
+  return f.a == 0 || (f.b <= 1024 && rot_smem(f, kMaxRotRows) <= kMaxSmem);
 }
 
 cudaError_t set_smem_attributes() {
@@ -360,12 +303,6 @@ cudaError_t set_smem_attributes() {
                                        cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
   if (e == cudaSuccess)
     e = cudaFuncSetAttribute(rotate_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             bytes);
-  if (e == cudaSuccess)
-    e = cudaFuncSetAttribute(run_analysis_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             bytes);
-  if (e == cudaSuccess)
-    e = cudaFuncSetAttribute(run_synthesis_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                              bytes);
   if (e == cudaSuccess) done.insert(dev);
   return e;
@@ -393,20 +330,16 @@ int rot_rows_per_cta(int a, int M) {
   return std::max(1, std::min(kMaxRotRows, static_cast<int>(ceil_div(static_cast<int64_t>(a) * M, 296))));
 }
 
-// R^T x (analysis, bf16 in, fp32 out) or R s (synthesis, fp32 in, bf16 out) for M tokens
+// R^T x (analysis) or R s (synthesis) for M tokens, bf16 in and out
 template <bool kSynth>
 cudaError_t rotate(const fq_frame& f, int M, const void* in, void* out, cudaStream_t s) {
-  if (f.a == 0) {
-    const int64_t n = static_cast<int64_t>(M) * f.d;
-    const unsigned grid = static_cast<unsigned>(std::min<int64_t>(ceil_div(n, 256), 1184));
-    return launch_pdl(copy_kernel<kSynth>, dim3(grid), dim3(256), 0, s, in, out, n);
-  }
   const int G = rot_rows_per_cta(f.a, M);
   // one thread per column of the a x b block, at least 256 for the loads
   const int threads = static_cast<int>(std::min<int64_t>(1024, std::max<int64_t>(256, round_up(f.b, 32))));
   return launch_pdl(rotate_kernel<kSynth>, dim3(static_cast<unsigned>(ceil_div(f.a, G)), M),
-                    dim3(threads), rot_smem(f, G), s, in, out, f.d, f.a, f.b, G,
-                    kSynth ? f.Qa : f.QaT, kSynth ? f.QbT : f.Qb, f.perm, f.iperm, f.signs);
+                    dim3(threads), rot_smem(f, G), s, static_cast<const __nv_bfloat16*>(in),
+                    static_cast<__nv_bfloat16*>(out), f.d, f.a, f.b, G, kSynth ? f.Qa : f.QaT,
+                    kSynth ? f.QbT : f.Qb, f.perm, f.iperm, f.signs);
 }
 
 }  // namespace
@@ -419,7 +352,7 @@ extern "C" {
 size_t fq_frame_implicit_bytes(int k, int rho, int d, int a, int b) {
   if (!valid_triple(k, rho, d) || a < 0 || b < 0) return 0;
   if ((a == 0) != (b == 0) || (a > 0 && static_cast<int64_t>(a) * b != d)) return 0;
-  return frame_buf(k, d, a, b).total;
+  return frame_buf(k, rho, d, a, b).total;
 }
 
 fq_status fq_frame_implicit(int k, int rho, int d, const fq_rotation* rot, void* buf,
@@ -438,19 +371,22 @@ fq_status fq_frame_implicit(int k, int rho, int d, const fq_rotation* rot, void*
       seen[p] = 1;
     }
   }
-  const FrameBuf L = frame_buf(k, d, a, b);
+  const FrameBuf L = frame_buf(k, rho, d, a, b);
   if (!buf || bytes < L.total) return FQ_ERR_WORKSPACE;
   if ((reinterpret_cast<uintptr_t>(buf) & 255u) != 0) return FQ_ERR_ALIGNMENT;
   auto s = reinterpret_cast<cudaStream_t>(stream);
   char* base = static_cast<char*>(buf);
-  // roots of unity exp(2 pi i m / k), m = 0 .. k-1 (host, double precision)
-  std::vector<float> roots(2 * static_cast<size_t>(k));
+  // the two orientations of the un-rotated operator, tile by tile (host, double precision)
+  std::vector<double> cs(k), sn(k);
   const double two_pi = 6.283185307179586476925286766559;
   for (int m = 0; m < k; ++m) {
-    const double th = two_pi * m / k;
-    roots[2 * m] = static_cast<float>(std::cos(th));
-    roots[2 * m + 1] = static_cast<float>(std::sin(th));
+    cs[m] = std::cos(two_pi * m / k);
+    sn[m] = std::sin(two_pi * m / k);
   }
+  const SparseShape SA = sparse_shape(k, rho, d, false), SS = sparse_shape(k, rho, d, true);
+  std::vector<uint16_t> ta, ts;
+  fill_tiles(k, rho, d, SA, false, cs, sn, ta);
+  fill_tiles(k, rho, d, SS, true, cs, sn, ts);
   std::vector<float> qa, qat, qb, qbt, sg;
   std::vector<int32_t> pm, ipm;
   if (rot) {
@@ -483,10 +419,12 @@ fq_status fq_frame_implicit(int k, int rho, int d, const fq_rotation* rot, void*
   auto up = [&](size_t off, const void* src, size_t n) {
     return n == 0 || cudaMemcpyAsync(base + off, src, n, cudaMemcpyHostToDevice, s) == cudaSuccess;
   };
-  if (!up(L.roots, roots.data(), roots.size() * 4) || !up(L.Qa, qa.data(), qa.size() * 4) ||
-      !up(L.QaT, qat.data(), qat.size() * 4) || !up(L.Qb, qb.data(), qb.size() * 4) ||
-      !up(L.QbT, qbt.data(), qbt.size() * 4) || !up(L.signs, sg.data(), sg.size() * 4) ||
-      !up(L.perm, pm.data(), pm.size() * 4) || !up(L.iperm, ipm.data(), ipm.size() * 4))
+  if (!up(L.ana_tiles, ta.data(), ta.size() * 2) || !up(L.ana_idx, SA.idx.data(), SA.idx.size() * 4) ||
+      !up(L.syn_tiles, ts.data(), ts.size() * 2) || !up(L.syn_idx, SS.idx.data(), SS.idx.size() * 4) ||
+      !up(L.Qa, qa.data(), qa.size() * 4) || !up(L.QaT, qat.data(), qat.size() * 4) ||
+      !up(L.Qb, qb.data(), qb.size() * 4) || !up(L.QbT, qbt.data(), qbt.size() * 4) ||
+      !up(L.signs, sg.data(), sg.size() * 4) || !up(L.perm, pm.data(), pm.size() * 4) ||
+      !up(L.iperm, ipm.data(), ipm.size() * 4))
     return FQ_ERR_CUDA;
   // the host vectors are released on return: the copies from them must be complete
   if (cudaStreamSynchronize(s) != cudaSuccess) return FQ_ERR_CUDA;
@@ -496,7 +434,12 @@ fq_status fq_frame_implicit(int k, int rho, int d, const fq_rotation* rot, void*
   f.d = d;
   f.a = a;
   f.b = b;
-  f.roots = reinterpret_cast<const float*>(base + L.roots);
+  f.ana_tiles = reinterpret_cast<const uint8_t*>(base + L.ana_tiles);
+  f.ana_idx = reinterpret_cast<const int32_t*>(base + L.ana_idx);
+  f.ana_count = SA.count;
+  f.syn_tiles = reinterpret_cast<const uint8_t*>(base + L.syn_tiles);
+  f.syn_idx = reinterpret_cast<const int32_t*>(base + L.syn_idx);
+  f.syn_count = SS.count;
   if (rot) {
     f.Qa = reinterpret_cast<const float*>(base + L.Qa);
     f.QaT = reinterpret_cast<const float*>(base + L.QaT);
@@ -526,8 +469,8 @@ fq_status fq_linear_forward_implicit(const void* x, int M, const fq_frame* F_in,
   const int n_in = fi.k * fi.rho, n_out = fo.k * fo.rho;
   if (C->n_in != n_in || C->n_out != n_out) return FQ_ERR_INVALID_ARG;
   if (n_in % 16 || n_out % 16 || fi.d % 8 || fo.d % 8) return FQ_ERR_ALIGNMENT;
-  if (!aligned16(x) || !aligned16(y) || (gamma && !aligned16(gamma)) || !aligned16(fi.roots) ||
-      !aligned16(fo.roots))
+  if (!aligned16(x) || !aligned16(y) || (gamma && !aligned16(gamma)) ||
+      !aligned16(fi.ana_tiles) || !aligned16(fo.syn_tiles))
     return FQ_ERR_ALIGNMENT;
   if (!ws) return FQ_ERR_WORKSPACE;
   if ((reinterpret_cast<uintptr_t>(ws) & 255u) != 0) return FQ_ERR_ALIGNMENT;
@@ -545,32 +488,15 @@ fq_status fq_linear_forward_implicit(const void* x, int M, const fq_frame* F_in,
   if (set_smem_attributes() != cudaSuccess) return FQ_ERR_CUDA;
   auto s = reinterpret_cast<cudaStream_t>(stream);
   char* w = static_cast<char*>(ws);
-  float* v = reinterpret_cast<float*>(w + L.v);
-  float* sy = reinterpret_cast<float*>(w + L.s);
-  auto* z = reinterpret_cast<__nv_bfloat16*>(w + L.z);
-  auto* u = reinterpret_cast<__nv_bfloat16*>(w + L.u);
-  const unsigned tchunks = static_cast<unsigned>(ceil_div(M, kRunTokens));
-
-  if (rotate<false>(fi, M, x, v, s) != cudaSuccess) return FQ_ERR_CUDA;
-  {
-    const int wi = fi.d / fi.rho, kch = static_cast<int>(ceil_div(fi.k, 32));
-    const float rk = static_cast<float>(1.0 / std::sqrt(static_cast<double>(fi.k)));
-    if (launch_pdl(run_analysis_kernel, dim3(static_cast<unsigned>(fi.rho / 2 * kch), tchunks),
-                   dim3(kRunWarps * 32), ana_smem(fi), s, v, z, M, fi.d, n_in, fi.k, wi, kch, rk,
-                   reinterpret_cast<const float2*>(fi.roots)) != cudaSuccess)
-      return FQ_ERR_CUDA;
-  }
-  const fq_status st = launch_decode_core(M, *C, gamma, w, ws_bytes, max_sms, s);
+  void* v = fi.a > 0 ? static_cast<void*>(w + L.v) : const_cast<void*>(x);
+  void* sy = fo.a > 0 ? static_cast<void*>(w + L.s) : y;
+  if (fi.a > 0 && rotate<false>(fi, M, x, v, s) != cudaSuccess) return FQ_ERR_CUDA;
+  DecGroupLayer g{v, fi.d, nullptr, *C, nullptr, fo.d, gamma, sy};
+  g.tin = SparseOperand{fi.ana_tiles, fi.ana_idx, fi.ana_count};
+  g.tout = SparseOperand{fo.syn_tiles, fo.syn_idx, fo.syn_count};
+  const fq_status st = launch_decode_group(M, 1, &g, w, L.group, max_sms, false, nullptr, 0, 0, s);
   if (st != FQ_OK) return st;
-  {
-    const int wo = fo.d / fo.rho, cch = static_cast<int>(ceil_div(wo, 32));
-    const float rk = static_cast<float>(1.0 / std::sqrt(static_cast<double>(fo.k)));
-    if (launch_pdl(run_synthesis_kernel, dim3(static_cast<unsigned>(fo.rho / 2 * cch), tchunks),
-                   dim3(kRunWarps * 32), syn_smem(fo), s, u, sy, M, fo.d, n_out, fo.k, wo, cch, rk,
-                   reinterpret_cast<const float2*>(fo.roots)) != cudaSuccess)
-      return FQ_ERR_CUDA;
-  }
-  if (rotate<true>(fo, M, sy, y, s) != cudaSuccess) return FQ_ERR_CUDA;
+  if (fo.a > 0 && rotate<true>(fo, M, sy, y, s) != cudaSuccess) return FQ_ERR_CUDA;
   return FQ_OK;
 }
 

@@ -66,7 +66,19 @@ fq_status launch_decode_forward(const void* x, int M, int d_in, const void* T_in
                                 int max_sms, const void* pf, size_t pf_bytes,
                                 int64_t inject_wait, cudaStream_t s);
 
-// One layer of a fused launch over independent layers (the M <= 64 kernel).
+// A block-sparse frame operand (frames in structured form): for every 128-row tile of the
+// operand, the K blocks [idx[3t], idx[3t+1]) it has non-zero entries in, stored from tile
+// idx[3t+2] of `tiles` on as contiguous 16 KiB tiles already in the 128-byte-swizzled shared
+// memory image; `count` stored tiles in all.
+struct SparseOperand {
+  const uint8_t* tiles;
+  const int32_t* idx;
+  int count;
+};
+
+// One layer of a fused launch over independent layers (the M <= 64 kernel).  With tin.tiles
+// (tout.tiles) set, the analysis (synthesis) reads that block-sparse operand instead of T_in
+// (T_out_t).
 struct DecGroupLayer {
   const void* x;
   int d_in;
@@ -76,6 +88,8 @@ struct DecGroupLayer {
   int d_out;
   const float* gamma;
   void* y;
+  SparseOperand tin{};
+  SparseOperand tout{};
 };
 // Workspace of a launch over G layers (header, then z and u of each layer); 0 for G out of range.
 size_t decode_group_workspace_bytes(int M, int G, const DecGroupLayer* layers);

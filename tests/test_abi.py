@@ -122,8 +122,9 @@ def test_valid_bf16_request_needs_sm103(L):
     assert _call(L) == 3
 
 
-def _frame(k=18, rho=16, d=256, roots=0x8000):
-    return fq._Frame(k, rho, d, 0, 0, None, None, None, None, None, None, None, roots)
+def _frame(k=18, rho=16, d=256, tiles=0x8000):
+    return fq._Frame(k, rho, d, 0, 0, None, None, None, None, None, None, None, tiles, 0x9000, 6,
+                     tiles, 0xA000, 6)
 
 
 def _call_implicit(L, x=0x1000, M=8, Fi=None, C=None, Fo=None, gamma=None, y=0x4000,
@@ -157,7 +158,7 @@ def test_implicit_host_validation_without_gpu(L):
     assert _call_implicit(L, M=0) == 1
     assert _call_implicit(L, max_sms=-1) == 1
     assert _call_implicit(L, Fi=_frame(k=15)) == 1                  # not a tight frame
-    assert _call_implicit(L, Fi=_frame(roots=None)) == 1
+    assert _call_implicit(L, Fi=_frame(tiles=None)) == 1
     assert _call_implicit(L, C=_P(0x5000, 0x6000, 0x7000, 288, 304)) == 1   # n_in != k rho
     assert _call_implicit(L, x=0x1002) == 2
     assert _call_implicit(L, ws=None) == 4
