@@ -413,6 +413,30 @@ fq_status fq_linear_forward_implicit(const void* x, int M, const fq_frame* F_in,
                                      const float* gamma, void* y, void* ws, size_t ws_bytes,
                                      int max_sms, fq_stream_t stream);
 
+/* One layer of fq_linear_forward_implicit_group: the arguments of fq_linear_forward_implicit
+ * for that layer. */
+typedef struct {
+  const void* x;            /* device bf16, M x F_in->d */
+  const fq_frame* F_in;     /* host pointers to prepared frames */
+  const fq_packed* C;
+  const fq_frame* F_out;
+  const float* gamma;       /* device fp32 [C->n_out] or NULL */
+  void* y;                  /* device bf16, M x F_out->d */
+} fq_implicit_layer;
+
+/* Workspace bytes of fq_linear_forward_implicit_group (0 for invalid sizes or counts). */
+size_t fq_implicit_group_workspace_bytes(int M, int n_layers, const fq_implicit_layer* layers);
+
+/* fq_linear_forward_implicit for up to FQ_MAX_GROUP independent layers: each layer's input
+ * rotation, then one fused launch over all the layers (as fq_linear_forward_group does with
+ * dense operators), then each layer's output rotation.  Requirements and errors: those of
+ * fq_linear_forward_implicit for each layer, and those of fq_linear_forward_group for the
+ * group (no y may be another layer's x or y).  This entry point has no counterpart in the
+ * paper. */
+fq_status fq_linear_forward_implicit_group(int M, int n_layers, const fq_implicit_layer* layers,
+                                           void* ws, size_t ws_bytes, int max_sms,
+                                           fq_stream_t stream);
+
 /* ------------------------------------------------------------------------------------------
  * Forward pass without a caller-provided workspace.  The paper has no counterpart: this is a
  * convenience of the library for callers that cannot allocate device memory.

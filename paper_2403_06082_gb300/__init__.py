@@ -24,7 +24,8 @@ __all__ = [
     "fq_reconstruct_workspace_bytes", "fq_reconstruct_weight", "fq_dense_workspace_bytes",
     "fq_dense_forward", "fq_static_check", "fq_group_workspace_bytes",
     "fq_linear_forward_group", "Layer", "FQ_MAX_GROUP", "fq_gptq_hessian",
-    "fq_gptq_workspace_bytes", "fq_quantize_gptq",
+    "fq_gptq_workspace_bytes", "fq_quantize_gptq", "fq_implicit_group_workspace_bytes",
+    "fq_linear_forward_implicit_group", "ImplicitLayer",
 ]
 FQ_MAX_GROUP = 4
 FQ_STATIC_SCRATCH_BYTES = 16 << 20
@@ -49,7 +50,8 @@ EXPORTED = ("fq_packed_words", "fq_pack", "fq_workspace_bytes", "fq_linear_forwa
             "fq_reconstruct_workspace_bytes", "fq_reconstruct_weight", "fq_dense_workspace_bytes",
             "fq_dense_forward", "fq_static_check", "fq_group_workspace_bytes",
             "fq_linear_forward_group", "fq_gptq_hessian", "fq_gptq_workspace_bytes",
-            "fq_quantize_gptq")
+            "fq_quantize_gptq", "fq_implicit_group_workspace_bytes",
+            "fq_linear_forward_implicit_group")
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
 
@@ -85,6 +87,11 @@ class _Layer(ctypes.Structure):
     _fields_ = [("x", ctypes.c_void_p), ("d_in", ctypes.c_int32), ("T_in", ctypes.c_void_p),
                 ("C", ctypes.POINTER(_Packed)), ("T_out_t", ctypes.c_void_p),
                 ("d_out", ctypes.c_int32), ("gamma", ctypes.c_void_p), ("y", ctypes.c_void_p)]
+
+
+class _ImplLayer(ctypes.Structure):
+    _fields_ = [("x", ctypes.c_void_p), ("F_in", ctypes.c_void_p), ("C", ctypes.c_void_p),
+                ("F_out", ctypes.c_void_p), ("gamma", ctypes.c_void_p), ("y", ctypes.c_void_p)]
 
 
 class _Frame(ctypes.Structure):
@@ -173,6 +180,13 @@ def lib() -> ctypes.CDLL:
                                        ctypes.c_double, ctypes.c_int, ctypes.c_void_p,
                                        ctypes.c_void_p, ctypes.c_void_p, ctypes.c_void_p,
                                        ctypes.c_void_p, ctypes.c_size_t, ctypes.c_void_p]
+        L.fq_implicit_group_workspace_bytes.restype = ctypes.c_size_t
+        L.fq_implicit_group_workspace_bytes.argtypes = [ctypes.c_int, ctypes.c_int,
+                                                        ctypes.POINTER(_ImplLayer)]
+        L.fq_linear_forward_implicit_group.restype = ctypes.c_int
+        L.fq_linear_forward_implicit_group.argtypes = [
+            ctypes.c_int, ctypes.c_int, ctypes.POINTER(_ImplLayer), ctypes.c_void_p,
+            ctypes.c_size_t, ctypes.c_int, ctypes.c_void_p]
         L.fq_static_check.restype = ctypes.c_int
         L.fq_static_check.argtypes = [ctypes.c_void_p]
         L.fq_frame_implicit_bytes.restype = ctypes.c_size_t
@@ -455,6 +469,42 @@ def fq_linear_forward_implicit(x, M: int, F_in: Frame, C: Packed, F_out: Frame, 
                                          ctypes.byref(F_out.c), _ptr(gamma), _ptr(y), _ptr(ws),
                                          ws_bytes, max_sms, _stream(stream)),
         "fq_linear_forward_implicit")
+
+
+@dataclass
+class ImplicitLayer:
+    """One layer of fq_linear_forward_implicit_group."""
+    x: object
+    F_in: Frame
+    C: Packed
+    F_out: Frame
+    gamma: object
+    y: object
+
+
+def _impl_layers(layers):
+    keep = [L.C._c() for L in layers]
+    arr = (_ImplLayer * len(layers))()
+    for i, (L, pc) in enumerate(zip(layers, keep)):
+        arr[i] = _ImplLayer(_ptr(L.x), ctypes.addressof(L.F_in.c), ctypes.addressof(pc),
+                            ctypes.addressof(L.F_out.c), _ptr(L.gamma), _ptr(L.y))
+    return arr, keep
+
+
+def fq_implicit_group_workspace_bytes(M: int, layers) -> int:
+    arr, keep = _impl_layers(layers)
+    n = lib().fq_implicit_group_workspace_bytes(M, len(layers), arr)
+    del keep
+    return n
+
+
+def fq_linear_forward_implicit_group(M: int, layers, ws, ws_bytes: int, max_sms: int = 0,
+                                     stream=None) -> None:
+    arr, keep = _impl_layers(layers)
+    _ok(lib().fq_linear_forward_implicit_group(M, len(layers), arr, _ptr(ws), ws_bytes, max_sms,
+                                               _stream(stream)),
+        "fq_linear_forward_implicit_group")
+    del keep
 
 
 def fq_reconstruct_workspace_bytes(d_in: int, n_in: int, n_out: int, d_out: int) -> int:

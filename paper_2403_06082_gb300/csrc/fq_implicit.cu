@@ -46,15 +46,37 @@ constexpr int kMaxRotRows = 8;     // rows of the a x b rotated block per rotati
 constexpr int kRotChunk = 32;
 constexpr int kRotWholeB = 128;
 
+// One launch rotates the tokens of up to FQ_MAX_GROUP layers (blockIdx.z = layer).
+struct RotLayer {
+  const __nv_bfloat16* in;
+  __nv_bfloat16* out;
+  int d, a, b, G;
+  const float* A;
+  const float* B;
+  const int32_t* perm;
+  const int32_t* iperm;
+  const float* signs;
+};
+struct RotBatch {
+  RotLayer L[FQ_MAX_GROUP];
+};
+
 template <bool kSynth>
-__global__ void __launch_bounds__(1024) rotate_kernel(const __nv_bfloat16* __restrict__ in,
-                                                      __nv_bfloat16* __restrict__ out, int d,
-                                                      int a, int b, int G,
-                                                      const float* __restrict__ A,
-                                                      const float* __restrict__ B,
-                                                      const int32_t* __restrict__ perm,
-                                                      const int32_t* __restrict__ iperm,
-                                                      const float* __restrict__ signs) {
+__global__ void __launch_bounds__(1024) rotate_kernel(const __grid_constant__ RotBatch rb) {
+  const RotLayer& ly = rb.L[blockIdx.z];
+  const __nv_bfloat16* __restrict__ in = ly.in;
+  __nv_bfloat16* __restrict__ out = ly.out;
+  const int d = ly.d, a = ly.a, b = ly.b, G = ly.G;
+  const float* __restrict__ A = ly.A;
+  const float* __restrict__ B = ly.B;
+  const int32_t* __restrict__ perm = ly.perm;
+  const int32_t* __restrict__ iperm = ly.iperm;
+  const float* __restrict__ signs = ly.signs;
+  pdl_launch_dependents();
+  if (static_cast<int>(blockIdx.x) * G >= a) {
+    pdl_wait();
+    return;
+  }
   extern __shared__ float sm[];
   float* V = sm;                    // [d]
   float* Ar = V + d;                // [G][a]
@@ -65,7 +87,6 @@ __global__ void __launch_bounds__(1024) rotate_kernel(const __nv_bfloat16* __res
   const int c = threadIdx.x;
   const bool col = c < b;
   const bool whole_b = b <= kRotWholeB;
-  pdl_launch_dependents();
   for (int i = threadIdx.x; i < rows * a; i += nt) Ar[i] = A[static_cast<int64_t>(r0) * a + i];
   if (whole_b)
 #pragma unroll 8
@@ -330,16 +351,36 @@ int rot_rows_per_cta(int a, int M) {
   return std::max(1, std::min(kMaxRotRows, static_cast<int>(ceil_div(static_cast<int64_t>(a) * M, 296))));
 }
 
-// R^T x (analysis) or R s (synthesis) for M tokens, bf16 in and out
+// R^T x (analysis) or R s (synthesis) for M tokens of n layers in one launch, bf16 in and out;
+// layers without a rotation are skipped
+template <bool kSynth>
+cudaError_t rotate_batch(int n, const fq_frame* const* f, const void* const* in,
+                         void* const* out, int M, cudaStream_t s) {
+  RotBatch rb{};
+  int nb = 0, gx = 1, threads = 256;
+  size_t smem = 0;
+  for (int l = 0; l < n; ++l) {
+    if (f[l]->a == 0) continue;
+    const fq_frame& F = *f[l];
+    const int G = rot_rows_per_cta(F.a, M);
+    rb.L[nb] = RotLayer{static_cast<const __nv_bfloat16*>(in[l]), static_cast<__nv_bfloat16*>(out[l]),
+                        F.d, F.a, F.b, G, kSynth ? F.Qa : F.QaT, kSynth ? F.QbT : F.Qb, F.perm,
+                        F.iperm, F.signs};
+    gx = std::max(gx, static_cast<int>(ceil_div(F.a, G)));
+    // one thread per column of the a x b block, at least 256 for the loads
+    threads = std::max(threads, static_cast<int>(std::min<int64_t>(1024, round_up(F.b, 32))));
+    smem = std::max(smem, rot_smem(F, G));
+    ++nb;
+  }
+  if (nb == 0) return cudaSuccess;
+  return launch_pdl(rotate_kernel<kSynth>, dim3(static_cast<unsigned>(gx), M, nb), dim3(threads),
+                    smem, s, rb);
+}
+
 template <bool kSynth>
 cudaError_t rotate(const fq_frame& f, int M, const void* in, void* out, cudaStream_t s) {
-  const int G = rot_rows_per_cta(f.a, M);
-  // one thread per column of the a x b block, at least 256 for the loads
-  const int threads = static_cast<int>(std::min<int64_t>(1024, std::max<int64_t>(256, round_up(f.b, 32))));
-  return launch_pdl(rotate_kernel<kSynth>, dim3(static_cast<unsigned>(ceil_div(f.a, G)), M),
-                    dim3(threads), rot_smem(f, G), s, static_cast<const __nv_bfloat16*>(in),
-                    static_cast<__nv_bfloat16*>(out), f.d, f.a, f.b, G, kSynth ? f.Qa : f.QaT,
-                    kSynth ? f.QbT : f.Qb, f.perm, f.iperm, f.signs);
+  const fq_frame* fp = &f;
+  return rotate_batch<kSynth>(1, &fp, &in, &out, M, s);
 }
 
 }  // namespace
@@ -497,6 +538,102 @@ fq_status fq_linear_forward_implicit(const void* x, int M, const fq_frame* F_in,
   const fq_status st = launch_decode_group(M, 1, &g, w, L.group, max_sms, false, nullptr, 0, 0, s);
   if (st != FQ_OK) return st;
   if (fo.a > 0 && rotate<true>(fo, M, sy, y, s) != cudaSuccess) return FQ_ERR_CUDA;
+  return FQ_OK;
+}
+
+
+size_t fq_implicit_group_workspace_bytes(int M, int n_layers, const fq_implicit_layer* layers) {
+  if (M <= 0 || M > kDecodeMaxM || n_layers < 1 || n_layers > FQ_MAX_GROUP || !layers) return 0;
+  DecGroupLayer g[FQ_MAX_GROUP];
+  size_t extra = 0;
+  for (int l = 0; l < n_layers; ++l) {
+    const fq_implicit_layer& L = layers[l];
+    if (!L.C || !L.F_in || !L.F_out) return 0;
+    g[l] = DecGroupLayer{nullptr, L.F_in->d, nullptr, *L.C, nullptr, L.F_out->d, nullptr, nullptr};
+    extra += static_cast<size_t>(round_up(static_cast<int64_t>(M) * L.F_in->d * 2, 256)) +
+             static_cast<size_t>(round_up(static_cast<int64_t>(M) * L.F_out->d * 2, 256));
+  }
+  const size_t base = decode_group_workspace_bytes(M, n_layers, g);
+  return base == 0 ? 0 : base + extra;
+}
+
+fq_status fq_linear_forward_implicit_group(int M, int n_layers, const fq_implicit_layer* layers,
+                                           void* ws, size_t ws_bytes, int max_sms,
+                                           fq_stream_t stream) {
+  if (!layers || n_layers < 1 || n_layers > FQ_MAX_GROUP || max_sms < 0 || M <= 0)
+    return FQ_ERR_INVALID_ARG;
+  for (int l = 0; l < n_layers; ++l) {
+    const fq_implicit_layer& L = layers[l];
+    if (!L.x || !L.y || !L.C) return FQ_ERR_INVALID_ARG;
+    if (const fq_status cs = check_packed(L.C)) return cs;
+    if (!valid_frame(L.F_in) || !valid_frame(L.F_out)) return FQ_ERR_INVALID_ARG;
+    const fq_frame &fi = *L.F_in, &fo = *L.F_out;
+    if (L.C->n_in != fi.k * fi.rho || L.C->n_out != fo.k * fo.rho) return FQ_ERR_INVALID_ARG;
+    if (fi.d % 8 || fo.d % 8) return FQ_ERR_ALIGNMENT;
+    if (!aligned16(L.x) || !aligned16(L.y) || (L.gamma && !aligned16(L.gamma)) ||
+        !aligned16(fi.ana_tiles) || !aligned16(fo.syn_tiles))
+      return FQ_ERR_ALIGNMENT;
+    if (!frame_fits(fi) || !frame_fits(fo)) return FQ_ERR_UNSUPPORTED;
+    for (int j = 0; j < n_layers; ++j)
+      if (j != l && (layers[j].y == L.y || layers[j].x == L.y)) return FQ_ERR_INVALID_ARG;
+    if (L.x == L.y) return FQ_ERR_INVALID_ARG;
+  }
+  if (M > kDecodeMaxM) return FQ_ERR_UNSUPPORTED;
+  if (!ws) return FQ_ERR_WORKSPACE;
+  if ((reinterpret_cast<uintptr_t>(ws) & 255u) != 0) return FQ_ERR_ALIGNMENT;
+  const size_t need = fq_implicit_group_workspace_bytes(M, n_layers, layers);
+  if (need == 0) return FQ_ERR_INVALID_ARG;
+  if (ws_bytes < need) return FQ_ERR_WORKSPACE;
+  {
+    int dev = 0, major = 0, minor = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess ||
+        cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, dev) != cudaSuccess ||
+        cudaDeviceGetAttribute(&minor, cudaDevAttrComputeCapabilityMinor, dev) != cudaSuccess)
+      return FQ_ERR_CUDA;
+    if (major * 10 + minor != 103) return FQ_ERR_UNSUPPORTED;
+  }
+  if (set_smem_attributes() != cudaSuccess) return FQ_ERR_CUDA;
+  auto s = reinterpret_cast<cudaStream_t>(stream);
+  char* w = static_cast<char*>(ws);
+  // the fused kernel's workspace first, then every layer's rotated tokens and output
+  DecGroupLayer g[FQ_MAX_GROUP];
+  for (int l = 0; l < n_layers; ++l) {
+    const fq_implicit_layer& L = layers[l];
+    g[l] = DecGroupLayer{nullptr, L.F_in->d, nullptr, *L.C, nullptr, L.F_out->d, L.gamma, nullptr};
+  }
+  size_t off = decode_group_workspace_bytes(M, n_layers, g);
+  const size_t group_bytes = off;
+  for (int l = 0; l < n_layers; ++l) {
+    const fq_implicit_layer& L = layers[l];
+    const fq_frame &fi = *L.F_in, &fo = *L.F_out;
+    void* v = fi.a > 0 ? static_cast<void*>(w + off) : const_cast<void*>(L.x);
+    off += static_cast<size_t>(round_up(static_cast<int64_t>(M) * fi.d * 2, 256));
+    void* sy = fo.a > 0 ? static_cast<void*>(w + off) : L.y;
+    off += static_cast<size_t>(round_up(static_cast<int64_t>(M) * fo.d * 2, 256));
+    g[l].x = v;
+    g[l].y = sy;
+    g[l].tin = SparseOperand{fi.ana_tiles, fi.ana_idx, fi.ana_count};
+    g[l].tout = SparseOperand{fo.syn_tiles, fo.syn_idx, fo.syn_count};
+  }
+  const fq_frame* fin[FQ_MAX_GROUP];
+  const fq_frame* fout[FQ_MAX_GROUP];
+  const void* xin[FQ_MAX_GROUP];
+  void* vout[FQ_MAX_GROUP];
+  const void* sin_[FQ_MAX_GROUP];
+  void* yout[FQ_MAX_GROUP];
+  for (int l = 0; l < n_layers; ++l) {
+    fin[l] = layers[l].F_in;
+    fout[l] = layers[l].F_out;
+    xin[l] = layers[l].x;
+    vout[l] = const_cast<void*>(g[l].x);
+    sin_[l] = g[l].y;
+    yout[l] = layers[l].y;
+  }
+  if (rotate_batch<false>(n_layers, fin, xin, vout, M, s) != cudaSuccess) return FQ_ERR_CUDA;
+  const fq_status st =
+      launch_decode_group(M, n_layers, g, w, group_bytes, max_sms, false, nullptr, 0, 0, s);
+  if (st != FQ_OK) return st;
+  if (rotate_batch<true>(n_layers, fout, sin_, yout, M, s) != cudaSuccess) return FQ_ERR_CUDA;
   return FQ_OK;
 }
 

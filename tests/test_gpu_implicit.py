@@ -160,3 +160,57 @@ def test_errors_launch_nothing():
         fq.fq_frame_implicit(15, RHO, 256, None, DEV)   # k < d / rho: not tight
     torch.cuda.synchronize()
     assert (y == 7.0).all()
+
+
+def _run_group(specs, M, max_sms=0):
+    """specs: [(workload, layer name, use_gamma, rotate)] in one fq_linear_forward_implicit_group
+    call; returns [(got, oracle)] per layer."""
+    keep, layers, out = [], [], []
+    for wl_key, name, use_gamma, rotate in specs:
+        L = oracle_layer(wl_key, name, rotate=rotate)
+        D = DeviceLayer(L, BF16)
+        Fi, Fo = _frames(wl_key, name, L, rotate)
+        X = activations(wl_key, name, M)
+        x = torch.from_numpy(X).to(DEV, BF16)
+        y = torch.full((M, L.d_out), float("nan"), dtype=BF16, device=DEV)
+        keep.append((D, Fi, Fo, x))
+        layers.append(fq.ImplicitLayer(x, Fi, D.C, Fo, D.gamma if use_gamma else None, y))
+        out.append((L, X, use_gamma, y))
+    nb = fq.fq_implicit_group_workspace_bytes(M, layers)
+    assert nb > 0
+    ws = torch.zeros(nb, dtype=torch.uint8, device=DEV)
+    fq.fq_linear_forward_implicit_group(M, layers, ws, nb, max_sms)
+    assert fq.fq_check(ws) == 0
+    return [(y.double().cpu().numpy(), reference(L, X, g)) for L, X, g, y in out]
+
+
+@pytest.mark.parametrize("M", [1, 16])
+def test_group_qkv(M):
+    for got, ref in _run_group([("llama2_7b_decode", n, False, True) for n in ("q", "k", "v")], M):
+        assert_parity(got, ref, 1e-2)
+
+
+def test_group_gate_up_and_mixed():
+    for got, ref in _run_group([("llama2_7b_decode", "gate", True, True),
+                                ("llama2_7b_decode", "up", False, True)], 4):
+        assert_parity(got, ref, 1e-2)
+    # different widths, one layer without rotation, and a budget
+    for got, ref in _run_group([("single256", "single", True, False),
+                                ("llama2_7b_decode", "down", False, True),
+                                ("vit_b16_mlp", "fc1", True, True)], 33, max_sms=100):
+        assert_parity(got, ref, 1e-2)
+
+
+def test_group_refusals():
+    L = oracle_layer("single256", "single")
+    D = DeviceLayer(L, BF16)
+    Fi, Fo = _frames("single256", "single", L)
+    x = torch.zeros(8, L.d_in, dtype=BF16, device=DEV)
+    y = torch.zeros(8, L.d_out, dtype=BF16, device=DEV)
+    one = fq.ImplicitLayer(x, Fi, D.C, Fo, None, y)
+    nb = fq.fq_implicit_group_workspace_bytes(8, [one, one])
+    ws = torch.zeros(nb, dtype=torch.uint8, device=DEV)
+    with pytest.raises(fq.FrameQuantError) as e:
+        fq.fq_linear_forward_implicit_group(8, [one, one], ws, nb)      # one output twice
+    assert e.value.status == 1
+    assert fq.fq_implicit_group_workspace_bytes(65, [one]) == 0         # decode batches only
