@@ -227,6 +227,17 @@ class Regime:
             L["x"].copy_(L["x_host"])
             L["y"] = self.y_all[y0:y0 + M * L["d_out"]].view(M, L["d_out"])
             L["y_host"] = self.y_host_all[y0:y0 + M * L["d_out"]].view(M, L["d_out"])
+        # the decode launches read the frames as pre-swizzled tiles (fq_frame_tile): the same
+        # values, one contiguous 16 KiB copy per 128 x 64 block
+        self.use_tiles = M <= 64
+        if self.use_tiles:
+            for L in self.layers:
+                for src, rows, cols, key in ((L["T_in"], L["n_in"], L["d_in"], "T_in_tiles"),
+                                             (L["T_out_t"], L["d_out"], L["n_out"],
+                                              "T_out_tiles")):
+                    nb = fq.fq_frame_tiles_bytes(rows, cols)
+                    L[key] = torch.empty(nb, dtype=torch.uint8, device=dev)
+                    fq.fq_frame_tile(src, rows, cols, L[key], nb)
         for grp in self.groups:
             ws_bytes = max(ws_bytes, fq.fq_group_workspace_bytes(M, self.group_layers(grp)))
         self.ws_bytes = ws_bytes
@@ -246,13 +257,17 @@ class Regime:
 
     def group_layers(self, grp):
         fq = self.fq
+        t = self.use_tiles
         return [fq.Layer(L["x"], L["d_in"], L["T_in"], L["C"], L["T_out_t"], L["d_out"],
-                         L["gamma"] if self.use_gamma else None, L["y"]) for L in grp]
+                         L["gamma"] if self.use_gamma else None, L["y"],
+                         L["T_in_tiles"] if t else None, L["T_out_tiles"] if t else None)
+                for L in grp]
 
     def forward_group(self, grp, stream, prefetch=None):
-        """One launch for the group's layers (fq_linear_forward_group; a single layer through
-        fq_linear_forward_ex), naming `prefetch` as the L2 hint."""
-        if len(grp) == 1:
+        """One launch for the group's layers (fq_linear_forward_group, which takes the tiled
+        frames; a single layer on row-major frames through fq_linear_forward_ex), naming
+        `prefetch` as the L2 hint."""
+        if len(grp) == 1 and not self.use_tiles:
             self.forward(grp[0], stream, prefetch)
             return
         self.fq.fq_linear_forward_group(self.M, self.group_layers(grp), self.ws, self.ws_bytes,
@@ -277,7 +292,9 @@ class Regime:
         for i, grp in enumerate(self.groups):
             if only is not None and i != only:
                 continue
-            self.forward_group(grp, stream.cuda_stream, self.groups[(i + 1) % n][0]["T_in"])
+            nxt = self.groups[(i + 1) % n][0]
+            self.forward_group(grp, stream.cuda_stream,
+                               nxt["T_in_tiles"] if self.use_tiles else nxt["T_in"])
 
     def forward(self, L, stream, prefetch=None):
         fq = self.fq
@@ -961,6 +978,10 @@ def main(argv=None):
         with torch.cuda.graph(g, stream=stream):
             dec.launch_groups(stream, only=gi)
         launch_graphs.append(g)
+    # the same 4 launches reading the row-major frames through 2-D tensor-map boxes
+    dec.use_tiles = False
+    rm_graph = dec.capture_groups(stream)
+    dec.use_tiles = True
     seq_graph = dec.capture(dec.layers, stream, chain=True)
     layer_graphs = [dec.capture([L], stream) for L in dec.layers]
     e2e_graph = dec.capture_groups(stream, host=True)
@@ -1009,6 +1030,16 @@ def main(argv=None):
                       for i, L in enumerate(dec.layers)},
     }
     del seq_graph, layer_graphs
+    barrier()
+    rm_ms, _ = timed_replays(torch, [rm_graph], stream, args.steps, args.warmup)
+    rm_ms = max_over_ranks(rm_ms, dist, dev)
+    row_major = {
+        "value": round(aggregate(rm_ms, args.steps, nL, world), 3), "unit": UNIT,
+        "ms_per_step": round(rm_ms / args.steps, 4),
+        "how": ("the headline's 4 launches with the frames read row-major (T_in, T_out_t "
+                "through 2-D tensor-map boxes of 128 rows x 128 bytes) instead of as tiles"),
+    }
+    del rm_graph
 
     # the same block with the frames in structured form (fq_linear_forward_implicit)
     implicit = measure_implicit(args, fq, wl, torch, dec, stream, peaks)
@@ -1088,6 +1119,7 @@ def main(argv=None):
             "per_launch": per_launch_out,
         },
         "sequential": sequential,
+        "row_major": row_major,
         "implicit": implicit,
         "e2e": {"value": round(e2e_us, 3), "unit": UNIT, "h2d_bytes_per_step": h2d,
                 "d2h_bytes_per_step": d2h,

@@ -213,6 +213,13 @@ typedef struct {
   int32_t d_out;
   const float* gamma;      /* device fp32 [n_out] or NULL */
   void* y;                 /* device bf16, M x d_out output */
+  /* Optional tiled copies of the frame operands, written by fq_frame_tile from this layer's
+   * T_in (rows n_in, cols d_in) and T_out_t (rows d_out, cols n_out), or NULL.  For M <= 64
+   * the fused launch reads a tiled operand instead of its row-major matrix, one contiguous
+   * 16 KiB copy per 128 x 64 block (the same values, so the same result); batches above 64
+   * read T_in and T_out_t, which stay required.  16-byte aligned. */
+  const void* T_in_tiles;
+  const void* T_out_tiles;
 } fq_layer;
 
 /* Most layers one fq_linear_forward_group call takes. */
@@ -244,6 +251,23 @@ size_t fq_group_workspace_bytes(int M, int n_layers, const fq_layer* layers);
 fq_status fq_linear_forward_group(int M, int n_layers, const fq_layer* layers, void* ws,
                                   size_t ws_bytes, const fq_forward_opts* opts,
                                   fq_stream_t stream);
+
+/* Bytes of the tiled copy of a rows x cols frame operand (fq_frame_tile): ceil(rows/128) x
+ * ceil(cols/64) tiles of 16 KiB, then a row-tile index of 12 bytes per row tile rounded up to
+ * 256; 0 for non-positive sizes or cols not a multiple of 8. */
+size_t fq_frame_tiles_bytes(int rows, int cols);
+
+/* Tiled copy of a dense frame operand for fq_layer's T_in_tiles / T_out_tiles: the bf16
+ * rows x cols row-major T (T_in, or T_out_t) as 128 x 64 blocks, row-block major then column
+ * block, each block 128 rows of 128 bytes with the 16-byte groups of row r stored in the
+ * order g ^ (r mod 8) (the 128-byte swizzle the tensor-core operand expects), zero padded
+ * past rows and cols.  A layout of the same values, not a change of the operator (the frame
+ * of Sec. 2.2 as T_in and T_out_t hold it).  Runs on the stream; T is read, out written.
+ * Errors: FQ_ERR_INVALID_ARG for NULL pointers, non-positive sizes or out overlapping T;
+ * FQ_ERR_ALIGNMENT for cols % 8 != 0 or a pointer not 16-byte aligned; FQ_ERR_WORKSPACE when
+ * out_bytes < fq_frame_tiles_bytes(rows, cols); FQ_ERR_CUDA for a launch failure. */
+fq_status fq_frame_tile(const void* T, int rows, int cols, void* out, size_t out_bytes,
+                        fq_stream_t stream);
 
 /* ------------------------------------------------------------------------------------------
  * Offline preparation of a layer (not on the inference path).  These produce the inputs of

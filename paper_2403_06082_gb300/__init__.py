@@ -25,7 +25,7 @@ __all__ = [
     "fq_dense_forward", "fq_static_check", "fq_group_workspace_bytes",
     "fq_linear_forward_group", "Layer", "FQ_MAX_GROUP", "fq_gptq_hessian",
     "fq_gptq_workspace_bytes", "fq_quantize_gptq", "fq_implicit_group_workspace_bytes",
-    "fq_linear_forward_implicit_group", "ImplicitLayer",
+    "fq_linear_forward_implicit_group", "ImplicitLayer", "fq_frame_tiles_bytes", "fq_frame_tile",
 ]
 FQ_MAX_GROUP = 4
 FQ_STATIC_SCRATCH_BYTES = 16 << 20
@@ -51,7 +51,7 @@ EXPORTED = ("fq_packed_words", "fq_pack", "fq_workspace_bytes", "fq_linear_forwa
             "fq_dense_forward", "fq_static_check", "fq_group_workspace_bytes",
             "fq_linear_forward_group", "fq_gptq_hessian", "fq_gptq_workspace_bytes",
             "fq_quantize_gptq", "fq_implicit_group_workspace_bytes",
-            "fq_linear_forward_implicit_group")
+            "fq_linear_forward_implicit_group", "fq_frame_tiles_bytes", "fq_frame_tile")
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
 
@@ -86,7 +86,8 @@ class _Opts(ctypes.Structure):
 class _Layer(ctypes.Structure):
     _fields_ = [("x", ctypes.c_void_p), ("d_in", ctypes.c_int32), ("T_in", ctypes.c_void_p),
                 ("C", ctypes.POINTER(_Packed)), ("T_out_t", ctypes.c_void_p),
-                ("d_out", ctypes.c_int32), ("gamma", ctypes.c_void_p), ("y", ctypes.c_void_p)]
+                ("d_out", ctypes.c_int32), ("gamma", ctypes.c_void_p), ("y", ctypes.c_void_p),
+                ("T_in_tiles", ctypes.c_void_p), ("T_out_tiles", ctypes.c_void_p)]
 
 
 class _ImplLayer(ctypes.Structure):
@@ -117,6 +118,11 @@ def lib() -> ctypes.CDLL:
             raise ImportError(f"libframequant.so is missing ({path}); build it with "
                               "`python -m paper_2403_06082_gb300._build`")
         L = ctypes.CDLL(path)
+        L.fq_frame_tiles_bytes.restype = ctypes.c_size_t
+        L.fq_frame_tiles_bytes.argtypes = [ctypes.c_int, ctypes.c_int]
+        L.fq_frame_tile.restype = ctypes.c_int
+        L.fq_frame_tile.argtypes = [ctypes.c_void_p, ctypes.c_int, ctypes.c_int, ctypes.c_void_p,
+                                    ctypes.c_size_t, ctypes.c_void_p]
         L.fq_packed_words.restype = ctypes.c_size_t
         L.fq_packed_words.argtypes = [ctypes.c_int, ctypes.c_int]
         L.fq_pack.restype = ctypes.c_int
@@ -270,6 +276,17 @@ class Packed:
                        self.n_in, self.ld_words, self.bits)
 
 
+def fq_frame_tiles_bytes(rows: int, cols: int) -> int:
+    return lib().fq_frame_tiles_bytes(rows, cols)
+
+
+def fq_frame_tile(T, rows: int, cols: int, out, out_bytes: int, stream=None) -> None:
+    """Tiled copy of a dense bf16 frame operand (T_in or T_out_t) for Layer.T_in_tiles /
+    Layer.T_out_tiles."""
+    _ok(lib().fq_frame_tile(_ptr(T), rows, cols, _ptr(out), out_bytes, _stream(stream)),
+        "fq_frame_tile")
+
+
 def fq_packed_words(n_out: int, n_in: int) -> int:
     return lib().fq_packed_words(n_out, n_in)
 
@@ -345,6 +362,8 @@ class Layer:
     d_out: int
     gamma: object
     y: object
+    T_in_tiles: object = None     # fq_frame_tile(T_in, n_in, d_in), or None
+    T_out_tiles: object = None    # fq_frame_tile(T_out_t, d_out, n_out), or None
 
 
 def _layers(layers):
@@ -353,7 +372,8 @@ def _layers(layers):
     arr = (_Layer * len(layers))()
     for i, (L, pc) in enumerate(zip(layers, packs)):
         arr[i] = _Layer(_ptr(L.x), L.d_in, _ptr(L.T_in), ctypes.pointer(pc), _ptr(L.T_out_t),
-                        L.d_out, _ptr(L.gamma), _ptr(L.y))
+                        L.d_out, _ptr(L.gamma), _ptr(L.y), _ptr(L.T_in_tiles),
+                        _ptr(L.T_out_tiles))
     return arr, packs
 
 

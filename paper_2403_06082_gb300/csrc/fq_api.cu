@@ -78,6 +78,27 @@ fq_status fq_pack(const uint8_t* codes, const uint16_t* scale_f16, const uint16_
   return FQ_OK;
 }
 
+size_t fq_frame_tiles_bytes(int rows, int cols) {
+  if (rows <= 0 || cols <= 0 || cols % 8 != 0) return 0;
+  return frame_tiles_index_offset(rows, cols) +
+         static_cast<size_t>(round_up(ceil_div(rows, kRowTile) * 12, 256));
+}
+
+fq_status fq_frame_tile(const void* T, int rows, int cols, void* out, size_t out_bytes,
+                        fq_stream_t stream) {
+  if (!T || !out || rows <= 0 || cols <= 0) return FQ_ERR_INVALID_ARG;
+  if (cols % 8 != 0 || !aligned16(T) || !aligned16(out)) return FQ_ERR_ALIGNMENT;
+  if (out_bytes < fq_frame_tiles_bytes(rows, cols)) return FQ_ERR_WORKSPACE;
+  if (static_cast<const char*>(out) < static_cast<const char*>(T) +
+          static_cast<size_t>(rows) * cols * 2 &&
+      static_cast<const char*>(T) < static_cast<const char*>(out) + out_bytes)
+    return FQ_ERR_INVALID_ARG;   // the copy may not overlap its source
+  return launch_frame_tile(T, rows, cols, out, reinterpret_cast<cudaStream_t>(stream)) ==
+                 cudaSuccess
+             ? FQ_OK
+             : FQ_ERR_CUDA;
+}
+
 size_t fq_workspace_bytes(int M, int d_in, int n_in, int n_out, int d_out, int mode) {
   if (M <= 0 || d_in <= 0 || n_in <= 0 || n_out <= 0 || d_out <= 0) return 0;
   int base = 0, act = 0;
@@ -134,6 +155,17 @@ bool group_layers(int n, const fq_layer* layers, DecGroupLayer* out) {
     const fq_layer& L = layers[l];
     if (!L.C) return false;
     out[l] = DecGroupLayer{L.x, L.d_in, L.T_in, *L.C, L.T_out_t, L.d_out, L.gamma, L.y};
+    // tiled copies of the frame operands (fq_frame_tile), read whole tiles at a time
+    auto tiled = [](const void* p, int rows, int cols) {
+      if (!p) return SparseOperand{};
+      const auto* b = static_cast<const uint8_t*>(p);
+      const int64_t RT = ceil_div(rows, kRowTile), KB = ceil_div(cols, kColBlock);
+      return SparseOperand{b, reinterpret_cast<const int32_t*>(
+                                  b + frame_tiles_index_offset(rows, cols)),
+                           static_cast<int>(RT * KB)};
+    };
+    out[l].tin = tiled(L.T_in_tiles, L.C->n_in, L.d_in);
+    out[l].tout = tiled(L.T_out_tiles, L.d_out, L.C->n_out);
   }
   return true;
 }
@@ -216,6 +248,7 @@ fq_status fq_linear_forward_group(int M, int n_layers, const fq_layer* layers, v
     for (int j = 0; j < n_layers; ++j)
       if (j != l && (layers[j].y == L.y || layers[j].x == L.y)) return FQ_ERR_INVALID_ARG;
     if (L.x == L.y) return FQ_ERR_INVALID_ARG;
+    if (!aligned16(L.T_in_tiles) || !aligned16(L.T_out_tiles)) return FQ_ERR_ALIGNMENT;
   }
   const size_t need = fq_group_workspace_bytes(M, n_layers, layers);
   if (need == 0) return FQ_ERR_INVALID_ARG;

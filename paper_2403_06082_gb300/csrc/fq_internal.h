@@ -45,6 +45,11 @@ namespace fq {
 fq_status check_packed(const fq_packed* C);
 
 // ---- fq_pack.cu
+// Dense frame operand (rows x cols bf16, row-major, cols % 8 == 0) -> out: ceil(rows/128) x
+// ceil(cols/64) pre-swizzled 16 KiB tiles (row tile major, zero padded), then the block-sparse
+// index {0, KB, t * KB} of each row tile at frame_tiles_index_offset().
+size_t frame_tiles_index_offset(int rows, int cols);
+cudaError_t launch_frame_tile(const void* T, int rows, int cols, void* out, cudaStream_t s);
 cudaError_t launch_pack(const uint8_t* codes, const uint16_t* scale, const uint16_t* zero,
                         int n_out, int n_in, uint32_t* words, int32_t* status, cudaStream_t s);
 

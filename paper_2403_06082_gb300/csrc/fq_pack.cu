@@ -1,6 +1,9 @@
 // fq_pack: 2-bit codes (uint8, row-major) -> the tiled packed layout of framequant.h, with a
 // check of the per-row scale and zero the descriptor will carry.
 // Memory-bound: one thread writes one 16-byte group of 4 words (64 codes of one row).
+// fq_frame_tile (below): a dense frame operand -> pre-swizzled contiguous tiles.
+#include <algorithm>
+
 #include "fq_device.cuh"
 #include "fq_internal.h"
 
@@ -57,6 +60,65 @@ cudaError_t launch_pack(const uint8_t* codes, const uint16_t* scale, const uint1
   const int64_t blocks = ceil_div(groups, threads);
   pack_kernel<<<static_cast<unsigned>(blocks), threads, 0, s>>>(
       codes, scale, zero, n_out, n_in, KB, groups, reinterpret_cast<uint4*>(words), status);
+  return cudaGetLastError();
+}
+
+}  // namespace fq
+
+// ------------------------------------------------------------------------------------------
+// fq_frame_tile: a dense bf16 frame operand (rows x cols, row-major) -> contiguous pre-swizzled
+// 128 x 64 tiles, the layout the M <= 64 kernel's weight copies read whole (one 16 KiB bulk
+// copy per K block instead of a 2-D box of 128 rows of 128 bytes).  Memory-bound: one thread
+// moves one 16-byte chunk (8 elements of one row).
+namespace fq {
+namespace {
+
+constexpr int kTileRows = 128, kTileCols = 64;
+
+__global__ void __launch_bounds__(256) frame_tile_kernel(const uint4* __restrict__ T, int rows,
+                                                         int cols, int KB, int64_t chunks,
+                                                         uint4* __restrict__ tiles,
+                                                         int32_t* __restrict__ idx, int RT) {
+  const int64_t g = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
+  if (g < 3ll * RT) {
+    // row tile t reads K blocks 0 .. KB-1 from tile t * KB on (the block-sparse index form)
+    const int t = static_cast<int>(g / 3), f = static_cast<int>(g % 3);
+    idx[g] = f == 0 ? 0 : (f == 1 ? KB : t * KB);
+  }
+  if (g >= chunks) return;
+  // chunk g of the output = (tile t, K block kb, row r, stored position h); it holds the
+  // row's 16-byte group c = h ^ (r & 7) (128-byte swizzle within each 8-row group)
+  const int h = static_cast<int>(g & 7);
+  const int r = static_cast<int>((g >> 3) % kTileRows);
+  const int64_t tk = g / (8 * kTileRows);
+  const int kb = static_cast<int>(tk % KB);
+  const int t = static_cast<int>(tk / KB);
+  const int row = t * kTileRows + r;
+  const int c = h ^ (r & 7);
+  const int col = kb * kTileCols + c * 8;
+  uint4 v = make_uint4(0u, 0u, 0u, 0u);
+  if (row < rows && col < cols) v = __ldg(T + (static_cast<int64_t>(row) * cols + col) / 8);
+  tiles[g] = v;
+}
+
+}  // namespace
+
+size_t frame_tiles_index_offset(int rows, int cols) {
+  return static_cast<size_t>(ceil_div(rows, kTileRows) * ceil_div(cols, kTileCols)) *
+         (kTileRows * kTileCols * 2);
+}
+
+cudaError_t launch_frame_tile(const void* T, int rows, int cols, void* out, cudaStream_t s) {
+  const int RT = static_cast<int>(ceil_div(rows, kTileRows));
+  const int KB = static_cast<int>(ceil_div(cols, kTileCols));
+  const int64_t chunks = static_cast<int64_t>(RT) * KB * kTileRows * 8;
+  auto* tiles = static_cast<uint4*>(out);
+  auto* idx = reinterpret_cast<int32_t*>(static_cast<char*>(out) +
+                                         frame_tiles_index_offset(rows, cols));
+  const int threads = 256;
+  const int64_t blocks = ceil_div(std::max<int64_t>(chunks, 3ll * RT), threads);
+  frame_tile_kernel<<<static_cast<unsigned>(blocks), threads, 0, s>>>(
+      static_cast<const uint4*>(T), rows, cols, KB, chunks, tiles, idx, RT);
   return cudaGetLastError();
 }
 

@@ -233,8 +233,8 @@ def test_group_sizes_and_validation_without_gpu(L):
     C = _P(0x5000, 0x6000, 0x7000, 4512, 4512)
     Cg = _P(0x5000, 0x6000, 0x7000, 12112, 4512)
 
-    def layer(x=0x1000, y=0x4000, C=C, d_out=4096):
-        return fq._Layer(x, 4096, 0x2000, ctypes.pointer(C), 0x3000, d_out, None, y)
+    def layer(x=0x1000, y=0x4000, C=C, d_out=4096, ti=None, to=None):
+        return fq._Layer(x, 4096, 0x2000, ctypes.pointer(C), 0x3000, d_out, None, y, ti, to)
 
     def arr(*ls):
         a = (fq._Layer * len(ls))()
@@ -261,6 +261,29 @@ def test_group_sizes_and_validation_without_gpu(L):
     assert fwd(arr(layer()), 1, ws=0x10010) == 2
     assert fwd(arr(layer()), 1, nb=1024) == 4
     assert fwd(arr(layer()), 1, opts=fq._Opts(1, None, 0, 1000)) == 1   # no timeout hook
+    assert fwd(arr(layer(ti=0x20008)), 1) == 2                       # tiles not 16-byte aligned
+    assert fwd(arr(layer(to=0x20004)), 1) == 2
+    # tiled operands do not change the workspace
+    assert L.fq_group_workspace_bytes(16, 1, arr(layer(ti=0x20000, to=0x30000))) == \
+        L.fq_group_workspace_bytes(16, 1, arr(layer()))
+
+
+def test_frame_tiles_sizes_and_validation_without_gpu(L):
+    # ceil(rows/128) x ceil(cols/64) tiles of 16 KiB, then 12 bytes per row tile (256-rounded)
+    assert fq.fq_frame_tiles_bytes(4512, 4096) == 36 * 64 * 16384 + 512
+    assert fq.fq_frame_tiles_bytes(4096, 4512) == 32 * 71 * 16384 + 512
+    assert fq.fq_frame_tiles_bytes(1, 8) == 16384 + 256
+    assert fq.fq_frame_tiles_bytes(12112, 11008) == 95 * 172 * 16384 + 1280
+    assert fq.fq_frame_tiles_bytes(0, 64) == 0
+    assert fq.fq_frame_tiles_bytes(64, 60) == 0
+    nb = fq.fq_frame_tiles_bytes(64, 64)
+    tile = L.fq_frame_tile
+    assert tile(None, 64, 64, 0x100000, nb, None) == 1
+    assert tile(0x1000, 0, 64, 0x100000, nb, None) == 1
+    assert tile(0x1000, 64, 60, 0x100000, nb, None) == 2
+    assert tile(0x1008, 64, 64, 0x100000, nb, None) == 2
+    assert tile(0x1000, 64, 64, 0x100000, nb - 16, None) == 4
+    assert tile(0x1000, 64, 64, 0x1000 + 4096, nb, None) == 1   # overlaps the source
 
 
 def test_activation_rounding_modes_without_gpu(L):
