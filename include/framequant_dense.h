@@ -21,15 +21,18 @@
 extern "C" {
 #endif
 
-/* Workspace bytes of fq_reconstruct_weight; 0 for invalid sizes.  It holds the forward's
- * workspace for M = d_in tokens, the d_in x d_in identity those tokens are, and the d_in x d_out
- * forward output: about 142 MB for a 4096 x 4096 layer at r = 1.1, 261 MB for 11008 x 4096,
- * 703 MB for 4096 x 11008, 567 MB for 8192 x 8192 and 4.5 GB for 8192 x 28672. */
+/* Workspace bytes of fq_reconstruct_weight; 0 for invalid sizes.  It holds the tensor-core
+ * chain's workspace for M = d_in tokens (z and u of the d_in unit vectors) and the d_in x d_out
+ * output before its transpose: about 108 MB for a 4096 x 4096 layer at r = 1.1, 227 MB for
+ * 11008 x 4096, 460 MB for 4096 x 11008, 432 MB for 8192 x 8192, 1.14 GB for 28672 x 8192 and
+ * 2.8 GB for 8192 x 28672. */
 size_t fq_reconstruct_workspace_bytes(int d_in, int n_in, int n_out, int d_out);
 
 /* W_hat = T_out^T diag(gamma) C_hat T_in, bf16 d_out x d_in row-major: the FQ_BF16 forward of
  * fq_linear_forward applied to the d_in unit vectors (so z and u are rounded to bf16 as in the
- * forward), then transposed.
+ * forward), then transposed.  The analysis of unit vector e_j is column j of T_in, exact in
+ * bf16, so it is taken as a transpose rather than a product; the code product and the synthesis
+ * run on the tensor cores.
  *   T_in, C, T_out_t, gamma  as in fq_linear_forward
  *   W_hat  device bf16 d_out x d_in output
  *   ws     device workspace of fq_reconstruct_workspace_bytes(...) bytes, 256-byte aligned,

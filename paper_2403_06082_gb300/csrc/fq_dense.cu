@@ -1,6 +1,8 @@
 // Weight reconstruction (include/framequant_dense.h): W_hat = T_out^T diag(gamma) C_hat T_in
 // as the FQ_BF16 forward of the d_in unit vectors, then a transpose.  The forward of unit
-// vector e_j is column j of W_hat, so the d_in x d_out output of the forward is W_hat^T.
+// vector e_j is column j of W_hat, so the d_in x d_out output of the forward is W_hat^T.  The
+// analysis of e_j is column j of T_in, exact in bf16, so the chain starts from that transpose
+// and runs only the code product and the synthesis on the tensor cores.
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
 
@@ -11,13 +13,6 @@
 
 namespace fq {
 namespace {
-
-// I (n x n bf16), grid-stride
-__global__ void eye_bf16_kernel(__nv_bfloat16* __restrict__ I, int n) {
-  const int64_t total = static_cast<int64_t>(n) * n;
-  for (int64_t i = blockIdx.x * 256ll + threadIdx.x; i < total; i += gridDim.x * 256ll)
-    I[i] = __float2bfloat16_rn(i / n == i % n ? 1.f : 0.f);
-}
 
 // out (cols x rows) = in (rows x cols)^T through 32 x 32 shared-memory tiles
 __global__ void transpose_bf16_kernel(const __nv_bfloat16* __restrict__ in,
@@ -36,17 +31,15 @@ __global__ void transpose_bf16_kernel(const __nv_bfloat16* __restrict__ in,
 }
 
 struct RecWs {
-  size_t fwd_bytes, eye, yt, total;
+  size_t fwd_bytes, yt, total;
 };
 
+// the tensor-core chain's workspace for M = d_in tokens, then the d_in x d_out output
 RecWs rec_ws(int d_in, int n_in, int n_out, int d_out) {
   RecWs L{};
   L.fwd_bytes = static_cast<size_t>(
-      round_up(static_cast<int64_t>(fq_workspace_bytes(d_in, d_in, n_in, n_out, d_out, FQ_BF16)),
-               256));
+      round_up(static_cast<int64_t>(tc_workspace_bytes(d_in, d_in, n_in, n_out, d_out, 0)), 256));
   size_t off = L.fwd_bytes;
-  L.eye = off;
-  off += static_cast<size_t>(round_up(static_cast<int64_t>(d_in) * d_in * 2, 256));
   L.yt = off;
   off += static_cast<size_t>(round_up(static_cast<int64_t>(d_in) * d_out * 2, 256));
   L.total = off;
@@ -64,7 +57,6 @@ extern "C" {
 
 size_t fq_reconstruct_workspace_bytes(int d_in, int n_in, int n_out, int d_out) {
   if (d_in <= 0 || n_in <= 0 || n_out <= 0 || d_out <= 0) return 0;
-  if (fq_workspace_bytes(d_in, d_in, n_in, n_out, d_out, FQ_BF16) == 0) return 0;
   return rec_ws(d_in, n_in, n_out, d_out).total;
 }
 
@@ -92,15 +84,10 @@ fq_status fq_reconstruct_weight(const void* T_in, const fq_packed* C, const void
   const RecWs L = rec_ws(d_in, C->n_in, C->n_out, d_out);
   auto s = reinterpret_cast<cudaStream_t>(stream);
   char* w = static_cast<char*>(ws);
-  auto* I = reinterpret_cast<__nv_bfloat16*>(w + L.eye);
   auto* Yt = reinterpret_cast<__nv_bfloat16*>(w + L.yt);
-  const int64_t n2 = static_cast<int64_t>(d_in) * d_in;
-  const unsigned g = static_cast<unsigned>(std::min<int64_t>(ceil_div(n2, 256), 4096));
-  eye_bf16_kernel<<<g, 256, 0, s>>>(I, d_in);
-  if (cudaGetLastError() != cudaSuccess) return FQ_ERR_CUDA;
-  // every check of the forward passed above (sizes, alignment, workspace, device)
-  const fq_status st = fq_linear_forward_ex(I, d_in, d_in, T_in, C, T_out_t, d_out, gamma, Yt,
-                                            w, L.fwd_bytes, FQ_BF16, nullptr, stream);
+  // every check of the chain passed above (sizes, alignment, workspace, device)
+  const fq_status st =
+      launch_tc_unit_forward(T_in, d_in, *C, T_out_t, d_out, gamma, Yt, w, L.fwd_bytes, s);
   if (st != FQ_OK) return st;
   transpose_bf16_kernel<<<dim3(static_cast<unsigned>(ceil_div(d_out, 32)),
                                static_cast<unsigned>(ceil_div(d_in, 32))),

@@ -122,5 +122,11 @@ fq_status launch_tc_forward(const void* x, int M, int d_in, const void* T_in,
                             const fq_packed& C, const void* T_out_t, int d_out,
                             const float* gamma, void* y, char* ws, size_t ws_bytes,
                             int max_sms, int act_bits, cudaStream_t s);
+// The same chain for the d_in unit vectors as tokens (M = d_in; y is d_in x d_out, row t the
+// forward of e_t), with the analysis product replaced by its exact result: z[t] = column t of
+// T_in (a transpose) and sum_j z[t][j] (column sums).  Workspace: tc_workspace_bytes(d_in, ...).
+fq_status launch_tc_unit_forward(const void* T_in, int d_in, const fq_packed& C,
+                                 const void* T_out_t, int d_out, const float* gamma, void* y,
+                                 char* ws, size_t ws_bytes, cudaStream_t s);
 
 }  // namespace fq

@@ -580,6 +580,48 @@ __global__ void __launch_bounds__(kQuantThreads) ff_round_kernel(
   }
 }
 
+// The analysis of the d_in unit vectors, for the weight reconstruction: unit vector e_t has
+// z = T_in e_t = column t of T_in, exact in bf16, so the analysis product is a transpose,
+// z[t][j] = T_in[j][t], through 32 x 32 shared-memory tiles.
+__global__ void unit_analysis_kernel(const __nv_bfloat16* __restrict__ T_in, int n_in, int d_in,
+                                     __nv_bfloat16* __restrict__ z) {
+  __shared__ __nv_bfloat16 tile[32][34];
+  const int t0 = blockIdx.x * 32, j0 = blockIdx.y * 32;
+  for (int dy = threadIdx.y; dy < 32; dy += 8) {
+    const int j = j0 + dy, t = t0 + threadIdx.x;
+    if (j < n_in && t < d_in) tile[dy][threadIdx.x] = T_in[static_cast<int64_t>(j) * d_in + t];
+  }
+  __syncthreads();
+  for (int dy = threadIdx.y; dy < 32; dy += 8) {
+    const int t = t0 + dy, j = j0 + threadIdx.x;
+    if (t < d_in && j < n_in) z[static_cast<int64_t>(t) * n_in + j] = tile[threadIdx.x][dy];
+  }
+}
+
+// sum_j z[t][j] of unit vector t (the column sums of T_in), for the code product's zero term.
+// Block of 32 columns x 32 row groups: thread (x, y) adds rows j = y, y + 32, ... of column
+// t0 + x (coalesced across the warp), then the 32 partial sums of a column are added in row
+// group order.  Block 0 clears the status word of the new call.
+__global__ void __launch_bounds__(1024) unit_zsum_kernel(const __nv_bfloat16* __restrict__ T_in,
+                                                         int n_in, int d_in,
+                                                         float* __restrict__ zsum,
+                                                         int32_t* __restrict__ status) {
+  __shared__ float part[32][33];
+  if (blockIdx.x == 0 && threadIdx.x == 0 && threadIdx.y == 0) *status = 0;
+  const int t = blockIdx.x * 32 + threadIdx.x;
+  float s = 0.f;
+  if (t < d_in)
+    for (int j = threadIdx.y; j < n_in; j += 32)
+      s += __bfloat162float(T_in[static_cast<int64_t>(j) * d_in + t]);
+  part[threadIdx.y][threadIdx.x] = s;
+  __syncthreads();
+  if (threadIdx.y == 0 && t < d_in) {
+    float tot = 0.f;
+    for (int y = 0; y < 32; ++y) tot += part[y][threadIdx.x];
+    zsum[t] = tot;
+  }
+}
+
 // ---------------------------------------------------------------------------------------------
 // host side
 // ---------------------------------------------------------------------------------------------
@@ -872,6 +914,75 @@ fq_status launch_tc_forward(const void* x, int M, int d_in, const void* T_in,
 
   return BN == 128 ? run_forward<128>(maps, a, max_sms, act_bits, delta, s)
                    : run_forward<256>(maps, a, max_sms, act_bits, delta, s);
+}
+
+namespace {
+// The code product and the synthesis of the tensor-core chain, after z and one sum of z per
+// token have been written to the workspace (a[1].zsum_tiles = 1).
+template <int BN>
+fq_status run_core_synthesis(const CUtensorMap* maps, PhaseArgs* a, cudaStream_t s) {
+  const DeviceInfo d = device_info();
+  if (prepare_kernel<kCore, BN>(d.dev) != cudaSuccess ||
+      prepare_kernel<kSynthesis, BN>(d.dev) != cudaSuccess)
+    return FQ_ERR_CUDA;
+  int g[2];
+  plan_phase<kCore, BN>(a[1], d, g[0]);
+  plan_phase<kSynthesis, BN>(a[2], d, g[1]);
+  a[1].zsum_tiles = 1;
+  if (launch_phase<kCore, BN>(maps[0], maps[0], a[1], g[0], s) != cudaSuccess ||
+      launch_phase<kSynthesis, BN>(maps[1], maps[2], a[2], g[1], s) != cudaSuccess)
+    return FQ_ERR_CUDA;
+  return FQ_OK;
+}
+}  // namespace
+
+fq_status launch_tc_unit_forward(const void* T_in, int d_in, const fq_packed& Cq,
+                                 const void* T_out_t, int d_out, const float* gamma, void* y,
+                                 char* ws, size_t ws_bytes, cudaStream_t s) {
+  const int M = d_in, n_in = Cq.n_in, n_out = Cq.n_out;
+  const WsLayout L = ws_layout(M, d_in, n_in, n_out, d_out, 0);
+  if (ws_bytes < L.total) return FQ_ERR_WORKSPACE;
+  const int BN = pick_bn(M);
+  auto* status = reinterpret_cast<int32_t*>(ws);
+  auto* z = reinterpret_cast<__nv_bfloat16*>(ws + L.z);
+  auto* u = reinterpret_cast<__nv_bfloat16*>(ws + L.u);
+  auto* zsum = reinterpret_cast<float*>(ws + L.zsum);
+  const auto* Tin = static_cast<const __nv_bfloat16*>(T_in);
+
+  PhaseArgs a[3];
+  const int R[3] = {n_in, n_out, d_out};
+  const int K[3] = {d_in, n_in, n_out};
+  __nv_bfloat16* outs[3] = {z, u, reinterpret_cast<__nv_bfloat16*>(y)};
+  for (int ph = 1; ph < 3; ++ph) {
+    a[ph] = PhaseArgs{};
+    a[ph].R = R[ph];
+    a[ph].K = K[ph];
+    a[ph].M = M;
+    a[ph].out = outs[ph];
+    a[ph].zsum_part = zsum;
+    a[ph].status = status;
+    a[ph].cnt = reinterpret_cast<uint32_t*>(ws + L.cnt);
+    a[ph].part = reinterpret_cast<float*>(ws + L.part);
+  }
+  a[1].words = Cq.words;
+  a[1].scale = reinterpret_cast<const __half*>(Cq.scale_f16);
+  a[1].zero = reinterpret_cast<const __half*>(Cq.zero_f16);
+  a[1].gamma = gamma;
+
+  // maps: z (the code product's B; also the unused A slot), T_out^T, u
+  CUtensorMap maps[3];
+  if (!make_tmap(&maps[0], z, M, n_in, BN) || !make_tmap(&maps[1], T_out_t, d_out, n_out, kBM) ||
+      !make_tmap(&maps[2], u, M, n_out, BN))
+    return FQ_ERR_CUDA;
+
+  unit_analysis_kernel<<<dim3(static_cast<unsigned>(ceil_div(d_in, 32)),
+                              static_cast<unsigned>(ceil_div(n_in, 32))),
+                         dim3(32, 8), 0, s>>>(Tin, n_in, d_in, z);
+  if (cudaGetLastError() != cudaSuccess) return FQ_ERR_CUDA;
+  unit_zsum_kernel<<<static_cast<unsigned>(ceil_div(d_in, 32)), dim3(32, 32), 0, s>>>(
+      Tin, n_in, d_in, zsum, status);
+  if (cudaGetLastError() != cudaSuccess) return FQ_ERR_CUDA;
+  return BN == 128 ? run_core_synthesis<128>(maps, a, s) : run_core_synthesis<256>(maps, a, s);
 }
 
 }  // namespace fq
