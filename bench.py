@@ -66,12 +66,13 @@ def load_peaks():
 
 
 def source_hash():
-    """Hash of the sources that define the decode kernel (its traffic record is only valid for
-    these exact sources)."""
+    """Hash of the sources that define the decode kernel: its code, the device helpers and the
+    workspace constants it is built with (its traffic record is only valid for these exact
+    sources)."""
     h = hashlib.sha256()
     pkg = os.path.join(ROOT, "paper_2403_06082_gb300", "csrc")
     for path in (os.path.join(pkg, "fq_decode.cu"), os.path.join(pkg, "fq_device.cuh"),
-                 os.path.join(pkg, "fq_internal.h"), os.path.join(ROOT, "include", "framequant.h")):
+                 os.path.join(pkg, "fq_internal.h")):
         with open(path, "rb") as f:
             h.update(os.path.basename(path).encode())
             h.update(f.read())

@@ -35,22 +35,29 @@ namespace {
 
 
 // ------------------------------------------------------------------------------ rotations
-// CTA (token t, rows r0 .. r0 + G - 1 of the a x b block); thread c < b owns column c
-// (b <= 1024; the CTA has at least 256 threads for the loads).  bf16 in and out.
+// CTA (token t, rows r0 .. r0 + 7 of the a x b block); bf16 in and out.
 //   analysis:  V = Pi^T x (V[perm[i]] = x_i), Y = Q_a^T V Q_b, out = D vec(Y)      A = Q_a^T, B = Q_b
 //   synthesis: V = D s, Y = Q_a V Q_b^T, out = Pi vec(Y) (out[iperm[e]] = vec(Y)_e) A = Q_a, B = Q_b^T
-// The factors do not depend on the previous kernel: A's rows, and all of B when it fits
-// (b <= kRotWholeB), are staged in shared memory before the wait for the input; a larger B is
-// staged kRotChunk rows at a time (coalesced loads, all in flight together).
-constexpr int kMaxRotRows = 8;     // rows of the a x b rotated block per rotation CTA
-constexpr int kRotChunk = 32;
-constexpr int kRotWholeB = 128;
+// The CTA is KG groups of r threads (r = b rounded up to a warp): thread (c, g) owns column c and
+// the reduction indices g, g + KG, ... of both products, for all eight rows at once (eight
+// accumulators; the eight row values of a reduction index are one 32-byte broadcast read of a
+// row-interleaved copy).  The KG partial sums of an entry are added in group order through
+// shared memory.  The factors do not depend on the previous kernel: A's rows, and all of B
+// when b <= kRotStageB, are staged in shared memory before the wait for the input; a larger B
+// streams through kRotBufs buffers of kRotChunk rows with asynchronous copies, so that its
+// loads overlap the products (the first chunks are requested before the wait).
+constexpr int kRotRows = 8;        // rows of the a x b block per rotation CTA
+constexpr int kRotStageB = 128;
+constexpr int kRotChunk = 16;
+constexpr int kRotBufs = 4;
+constexpr int kRotMaxGroups = 4;
 
 // One launch rotates the tokens of up to FQ_MAX_GROUP layers (blockIdx.z = layer).
 struct RotLayer {
   const __nv_bfloat16* in;
   __nv_bfloat16* out;
-  int d, a, b, G;
+  int d, a, b;
+  int bp, KG;             // column slots (b rounded up to 32) and reduction groups
   const float* A;
   const float* B;
   const int32_t* perm;
@@ -61,93 +68,152 @@ struct RotBatch {
   RotLayer L[FQ_MAX_GROUP];
 };
 
+__device__ __forceinline__ void cp_async16(float* smem_dst, const float* gsrc) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(smem_u32(smem_dst)), "l"(gsrc)
+               : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() {
+  asm volatile("cp.async.commit_group;" ::: "memory");
+}
+__device__ __forceinline__ void cp_async_wait_pending() {
+  asm volatile("cp.async.wait_group %0;" ::"n"(kRotBufs - 1) : "memory");
+}
+
+__device__ __forceinline__ void fma8(float (&acc)[kRotRows], const float* r8, float v) {
+  const float4 u0 = *reinterpret_cast<const float4*>(r8);
+  const float4 u1 = *reinterpret_cast<const float4*>(r8 + 4);
+  acc[0] = fmaf(u0.x, v, acc[0]);
+  acc[1] = fmaf(u0.y, v, acc[1]);
+  acc[2] = fmaf(u0.z, v, acc[2]);
+  acc[3] = fmaf(u0.w, v, acc[3]);
+  acc[4] = fmaf(u1.x, v, acc[4]);
+  acc[5] = fmaf(u1.y, v, acc[5]);
+  acc[6] = fmaf(u1.z, v, acc[6]);
+  acc[7] = fmaf(u1.w, v, acc[7]);
+}
+
 template <bool kSynth>
 __global__ void __launch_bounds__(1024) rotate_kernel(const __grid_constant__ RotBatch rb) {
   const RotLayer& ly = rb.L[blockIdx.z];
   const __nv_bfloat16* __restrict__ in = ly.in;
   __nv_bfloat16* __restrict__ out = ly.out;
-  const int d = ly.d, a = ly.a, b = ly.b, G = ly.G;
+  const int d = ly.d, a = ly.a, b = ly.b, bp = ly.bp, KG = ly.KG;
   const float* __restrict__ A = ly.A;
   const float* __restrict__ B = ly.B;
   const int32_t* __restrict__ perm = ly.perm;
   const int32_t* __restrict__ iperm = ly.iperm;
   const float* __restrict__ signs = ly.signs;
   pdl_launch_dependents();
-  if (static_cast<int>(blockIdx.x) * G >= a) {
+  const int r0 = static_cast<int>(blockIdx.x) * kRotRows;
+  if (r0 >= a) {
     pdl_wait();
     return;
   }
-  extern __shared__ float sm[];
-  float* V = sm;                    // [d]
-  float* Ar = V + d;                // [G][a]
-  float* T1 = Ar + G * a;           // [G][b]
-  float* Bs = T1 + G * b;           // [b][b] when b <= kRotWholeB, else [kRotChunk][b]
-  const int t = blockIdx.y, r0 = blockIdx.x * G, nt = blockDim.x;
-  const int rows = min(G, a - r0);
-  const int c = threadIdx.x;
-  const bool col = c < b;
-  const bool whole_b = b <= kRotWholeB;
-  for (int i = threadIdx.x; i < rows * a; i += nt) Ar[i] = A[static_cast<int64_t>(r0) * a + i];
-  if (whole_b)
-#pragma unroll 8
-    for (int i = threadIdx.x; i < b * b; i += nt) Bs[i] = B[i];
+  extern __shared__ float4 rot_smem4[];
+  float* V = reinterpret_cast<float*>(rot_smem4);   // [d], d rounded up to 4
+  float* At = V + ((d + 3) & ~3);                   // [a][8]: At[i][g] = A[r0 + g][i]
+  float* T1t = At + a * kRotRows;                   // [b][8]: T1t[k][g] = (A V)[r0 + g][k]
+  float* P = T1t + b * kRotRows;                    // [KG][8][bp] partial sums
+  float* Bs = P + KG * kRotRows * bp;               // all of B, or kRotBufs chunks of it
+  const int t = blockIdx.y, nt = blockDim.x, tid = threadIdx.x;
+  const int rows = min(kRotRows, a - r0);
+  const int c = tid % bp, kg = tid / bp;
+  const bool active = c < b && kg < KG;
+  const bool staged = b <= kRotStageB;
+  const bool async = !staged && (b & 3) == 0;
+  const int nch = (b + kRotChunk - 1) / kRotChunk;
+  // chunk ch of B (rows ch * kRotChunk ..) into buffer ch mod kRotBufs; every thread commits a
+  // group per call, so that the group count stays uniform
+  auto stage_chunk = [&](int ch) {
+    if (ch < nch) {
+      const int k0 = ch * kRotChunk, kn = min(kRotChunk, b - k0);
+      const float* src = B + static_cast<int64_t>(k0) * b;
+      float* dst = Bs + (ch % kRotBufs) * kRotChunk * b;
+      for (int i = tid; i < kn * b / 4; i += nt) cp_async16(dst + 4 * i, src + 4 * i);
+    }
+    cp_async_commit();
+  };
+  for (int i = tid; i < a * kRotRows; i += nt) {
+    const int ii = i / kRotRows, g = i % kRotRows;
+    At[i] = g < rows ? A[static_cast<int64_t>(r0 + g) * a + ii] : 0.f;
+  }
+  if (staged) {
+#pragma unroll 4
+    for (int i = tid; i < b * b; i += nt) Bs[i] = B[i];
+  } else if (async) {
+    for (int ch = 0; ch < kRotBufs - 1; ++ch) stage_chunk(ch);
+  }
   pdl_wait();
   const __nv_bfloat16* src = in + static_cast<int64_t>(t) * d;
   if (kSynth) {
-#pragma unroll 8
-    for (int i = threadIdx.x; i < d; i += nt) V[i] = signs[i] * __bfloat162float(src[i]);
+#pragma unroll 4
+    for (int i = tid; i < d; i += nt) V[i] = signs[i] * __bfloat162float(src[i]);
   } else {
-#pragma unroll 8
-    for (int i = threadIdx.x; i < d; i += nt) V[perm[i]] = __bfloat162float(src[i]);
+#pragma unroll 4
+    for (int i = tid; i < d; i += nt) V[perm[i]] = __bfloat162float(src[i]);
   }
   __syncthreads();
-  float acc[kMaxRotRows];
+  float acc[kRotRows];
+  // T1 = A[rows] V: this thread's partial over i = kg, kg + KG, ...
 #pragma unroll
-  for (int g = 0; g < kMaxRotRows; ++g) acc[g] = 0.f;
-  if (col) {
+  for (int g = 0; g < kRotRows; ++g) acc[g] = 0.f;
+  if (active) {
 #pragma unroll 4
-    for (int r = 0; r < a; ++r) {
-      const float v = V[r * b + c];
+    for (int i = kg; i < a; i += KG) fma8(acc, At + i * kRotRows, V[i * b + c]);
 #pragma unroll
-      for (int g = 0; g < kMaxRotRows; ++g)
-        if (g < rows) acc[g] = fmaf(Ar[g * a + r], v, acc[g]);
-    }
-#pragma unroll
-    for (int g = 0; g < kMaxRotRows; ++g)
-      if (g < rows) T1[g * b + c] = acc[g];
+    for (int g = 0; g < kRotRows; ++g) P[(kg * kRotRows + g) * bp + c] = acc[g];
   }
+  __syncthreads();
+  for (int e = tid; e < b * kRotRows; e += nt) {
+    const int k = e / kRotRows, g = e % kRotRows;
+    float s = 0.f;
+    for (int q = 0; q < KG; ++q) s += P[(q * kRotRows + g) * bp + k];
+    T1t[e] = s;
+  }
+  __syncthreads();
+  // Y = T1 B: this thread's partial over k = kg, kg + KG, ...
 #pragma unroll
-  for (int g = 0; g < kMaxRotRows; ++g) acc[g] = 0.f;
-  const int chunk = whole_b ? b : kRotChunk;
-  for (int k0 = 0; k0 < b; k0 += chunk) {
-    const int kn = min(chunk, b - k0);
-    __syncthreads();            // T1 written (first chunk), the previous chunk consumed
-    if (!whole_b) {
-#pragma unroll 8
-      for (int i = threadIdx.x; i < kn * b; i += nt) Bs[i] = B[static_cast<int64_t>(k0) * b + i];
-      __syncthreads();
-    }
-    const float* Bk = whole_b ? Bs + static_cast<int64_t>(k0) * b : Bs;
-    if (col) {
+  for (int g = 0; g < kRotRows; ++g) acc[g] = 0.f;
+  if (staged) {
+    if (active) {
 #pragma unroll 4
-      for (int kk = 0; kk < kn; ++kk) {
-        const float w = Bk[kk * b + c];
-#pragma unroll
-        for (int g = 0; g < kMaxRotRows; ++g)
-          if (g < rows) acc[g] = fmaf(T1[g * b + k0 + kk], w, acc[g]);
+      for (int k = kg; k < b; k += KG) fma8(acc, T1t + k * kRotRows, Bs[k * b + c]);
+    }
+  } else {
+    for (int ch = 0; ch < nch; ++ch) {
+      const int k0 = ch * kRotChunk, k1 = min(b, k0 + kRotChunk);
+      const float* Bc = Bs;
+      if (async) {
+        stage_chunk(ch + kRotBufs - 1);
+        cp_async_wait_pending();     // chunk ch has landed (for this thread's copies)
+        __syncthreads();             // ... and for every thread's
+        Bc = Bs + (ch % kRotBufs) * kRotChunk * b;
+      } else {
+        for (int i = tid; i < (k1 - k0) * b; i += nt) Bs[i] = B[static_cast<int64_t>(k0) * b + i];
+        __syncthreads();
       }
+      if (active) {
+        const int first = k0 + ((kg - k0 % KG) % KG + KG) % KG;
+        for (int k = first; k < k1; k += KG) fma8(acc, T1t + k * kRotRows, Bc[(k - k0) * b + c]);
+      }
+      __syncthreads();               // the buffer is read before it is refilled
     }
   }
-  if (!col) return;
-  __nv_bfloat16* dst = out + static_cast<int64_t>(t) * d;
+  if (active) {
 #pragma unroll
-  for (int g = 0; g < kMaxRotRows; ++g) {
-    if (g >= rows) continue;
-    const int e = (r0 + g) * b + c;
+    for (int g = 0; g < kRotRows; ++g) P[(kg * kRotRows + g) * bp + c] = acc[g];
+  }
+  __syncthreads();
+  __nv_bfloat16* dst = out + static_cast<int64_t>(t) * d;
+  for (int e = tid; e < rows * b; e += nt) {
+    const int g = e / b, cc = e - g * b;
+    float y = 0.f;
+    for (int q = 0; q < KG; ++q) y += P[(q * kRotRows + g) * bp + cc];
+    const int o = (r0 + g) * b + cc;
     if (kSynth)
-      dst[iperm[e]] = __float2bfloat16_rn(acc[g]);
+      dst[iperm[o]] = __float2bfloat16_rn(y);
     else
-      dst[e] = __float2bfloat16_rn(signs[e] * acc[g]);
+      dst[o] = __float2bfloat16_rn(signs[o] * y);
   }
 }
 
@@ -298,9 +364,21 @@ ImplWs impl_ws(int M, int d_in, int n_in, int n_out, int d_out) {
   return L;
 }
 
-size_t rot_smem(const fq_frame& f, int G) {
-  const size_t brows = f.b <= kRotWholeB ? static_cast<size_t>(f.b) : kRotChunk;
-  return (static_cast<size_t>(f.d) + static_cast<size_t>(G) * (f.a + f.b) + brows * f.b) * 4;
+// a rotation CTA's column slots (b rounded up to a warp), reduction groups and threads
+int rot_slots(int b) { return static_cast<int>(round_up(b, 32)); }
+int rot_groups(int b, int nt) {
+  return std::max(1, std::min(kRotMaxGroups, nt / rot_slots(b)));
+}
+int rot_threads(int b) {
+  return rot_slots(b) * std::max(1, std::min(kRotMaxGroups, 1024 / rot_slots(b)));
+}
+
+size_t rot_smem(const fq_frame& f, int KG) {
+  const size_t bb = f.b <= kRotStageB ? static_cast<size_t>(f.b) * f.b
+                                      : static_cast<size_t>(kRotBufs) * kRotChunk * f.b;
+  return (static_cast<size_t>(round_up(f.d, 4)) + static_cast<size_t>(kRotRows) * (f.a + f.b) +
+          static_cast<size_t>(KG) * kRotRows * rot_slots(f.b) + bb) *
+         4;
 }
 
 constexpr size_t kMaxSmem = 227 * 1024;
@@ -309,7 +387,8 @@ bool frame_fits(const fq_frame& f) {
   if (ceil_div(static_cast<int64_t>(f.k) * f.rho, kTR) > kWsMaxTiles ||
       ceil_div(f.d, kTR) > kWsMaxTiles)
     return false;
-  return f.a == 0 || (f.b <= 1024 && rot_smem(f, kMaxRotRows) <= kMaxSmem);
+  return f.a == 0 ||
+         (f.b <= 1024 && rot_smem(f, rot_groups(f.b, rot_threads(f.b))) <= kMaxSmem);
 }
 
 cudaError_t set_smem_attributes() {
@@ -347,29 +426,25 @@ cudaError_t launch_pdl(void (*kern)(KArgs...), dim3 grid, dim3 block, size_t sme
   return cudaLaunchKernelEx(&cfg, kern, static_cast<KArgs>(args)...);
 }
 
-int rot_rows_per_cta(int a, int M) {
-  return std::max(1, std::min(kMaxRotRows, static_cast<int>(ceil_div(static_cast<int64_t>(a) * M, 296))));
-}
-
 // R^T x (analysis) or R s (synthesis) for M tokens of n layers in one launch, bf16 in and out;
 // layers without a rotation are skipped
 template <bool kSynth>
 cudaError_t rotate_batch(int n, const fq_frame* const* f, const void* const* in,
                          void* const* out, int M, cudaStream_t s) {
   RotBatch rb{};
-  int nb = 0, gx = 1, threads = 256;
+  int nb = 0, gx = 1, threads = 32;
   size_t smem = 0;
+  for (int l = 0; l < n; ++l)
+    if (f[l]->a != 0) threads = std::max(threads, rot_threads(f[l]->b));
   for (int l = 0; l < n; ++l) {
     if (f[l]->a == 0) continue;
     const fq_frame& F = *f[l];
-    const int G = rot_rows_per_cta(F.a, M);
+    const int KG = rot_groups(F.b, threads);
     rb.L[nb] = RotLayer{static_cast<const __nv_bfloat16*>(in[l]), static_cast<__nv_bfloat16*>(out[l]),
-                        F.d, F.a, F.b, G, kSynth ? F.Qa : F.QaT, kSynth ? F.QbT : F.Qb, F.perm,
-                        F.iperm, F.signs};
-    gx = std::max(gx, static_cast<int>(ceil_div(F.a, G)));
-    // one thread per column of the a x b block, at least 256 for the loads
-    threads = std::max(threads, static_cast<int>(std::min<int64_t>(1024, round_up(F.b, 32))));
-    smem = std::max(smem, rot_smem(F, G));
+                        F.d, F.a, F.b, rot_slots(F.b), KG, kSynth ? F.Qa : F.QaT,
+                        kSynth ? F.QbT : F.Qb, F.perm, F.iperm, F.signs};
+    gx = std::max(gx, static_cast<int>(ceil_div(F.a, kRotRows)));
+    smem = std::max(smem, rot_smem(F, KG));
     ++nb;
   }
   if (nb == 0) return cudaSuccess;
