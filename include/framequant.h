@@ -428,10 +428,10 @@ size_t fq_implicit_workspace_bytes(int M, int d_in, int n_in, int n_out, int d_o
  *          zero-filled before its first use (the header rules of fq_linear_forward)
  *   max_sms  as in fq_linear_forward_sms (0: the whole device)
  * Requirements: 1 <= M <= 64; for each frame at most 640 row tiles of 128 per orientation and,
- * with a rotation, b <= 1024 and (d + 8 (a + b) + 8 g r + (b * b if b <= 128 else 64 b)) * 4
- * bytes of shared memory at most 227 KiB, with d rounded up to a multiple of 4, r = b rounded
- * up to a multiple of 32 and g = max(1, min(4, 1024 / r)); sizes and alignment as in
- * fq_linear_forward.
+ * with a rotation, b <= 1024 and (d + 8 (a + b) + 8 g r + B) * 4 bytes of shared memory at
+ * most 227 KiB, with d rounded up to a multiple of 4, r = b rounded up to a multiple of 32,
+ * g = max(1, min(4, 1024 / r)), and B = b * b when b <= 128 and that total stays within
+ * 110 KiB, else 64 b; sizes and alignment as in fq_linear_forward.
  * Errors: FQ_ERR_INVALID_ARG, FQ_ERR_ALIGNMENT, FQ_ERR_WORKSPACE, FQ_ERR_UNSUPPORTED (M > 64, a
  * frame above those limits, device not compute capability 10.3), FQ_ERR_CUDA. */
 fq_status fq_linear_forward_implicit(const void* x, int M, const fq_frame* F_in,

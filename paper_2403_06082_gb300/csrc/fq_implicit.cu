@@ -43,11 +43,14 @@ namespace {
 // accumulators; the eight row values of a reduction index are one 32-byte broadcast read of a
 // row-interleaved copy).  The KG partial sums of an entry are added in group order through
 // shared memory.  The factors do not depend on the previous kernel: A's rows, and all of B
-// when b <= kRotStageB, are staged in shared memory before the wait for the input; a larger B
-// streams through kRotBufs buffers of kRotChunk rows with asynchronous copies, so that its
-// loads overlap the products (the first chunks are requested before the wait).
+// when b <= kRotStageB and the CTA's shared memory stays within kRotSmemStaged (so that two
+// CTAs fit an SM), are requested in shared memory before the wait for the input, with
+// asynchronous copies all in flight at once; otherwise B streams through kRotBufs buffers of
+// kRotChunk rows, so that its loads overlap the products (the first chunks are requested
+// before the wait).
 constexpr int kRotRows = 8;        // rows of the a x b block per rotation CTA
 constexpr int kRotStageB = 128;
+constexpr size_t kRotSmemStaged = 110 * 1024;
 constexpr int kRotChunk = 16;
 constexpr int kRotBufs = 4;
 constexpr int kRotMaxGroups = 4;
@@ -58,6 +61,7 @@ struct RotLayer {
   __nv_bfloat16* out;
   int d, a, b;
   int bp, KG;             // column slots (b rounded up to 32) and reduction groups
+  int staged;             // all of B in shared memory (else streamed in chunks)
   const float* A;
   const float* B;
   const int32_t* perm;
@@ -77,6 +81,9 @@ __device__ __forceinline__ void cp_async_commit() {
 }
 __device__ __forceinline__ void cp_async_wait_pending() {
   asm volatile("cp.async.wait_group %0;" ::"n"(kRotBufs - 1) : "memory");
+}
+__device__ __forceinline__ void cp_async_wait_all() {
+  asm volatile("cp.async.wait_group 0;" ::: "memory");
 }
 
 __device__ __forceinline__ void fma8(float (&acc)[kRotRows], const float* r8, float v) {
@@ -119,8 +126,8 @@ __global__ void __launch_bounds__(1024) rotate_kernel(const __grid_constant__ Ro
   const int rows = min(kRotRows, a - r0);
   const int c = tid % bp, kg = tid / bp;
   const bool active = c < b && kg < KG;
-  const bool staged = b <= kRotStageB;
-  const bool async = !staged && (b & 3) == 0;
+  const bool staged = ly.staged != 0;
+  const bool async = (b & 3) == 0;
   const int nch = (b + kRotChunk - 1) / kRotChunk;
   // chunk ch of B (rows ch * kRotChunk ..) into buffer ch mod kRotBufs; every thread commits a
   // group per call, so that the group count stays uniform
@@ -138,20 +145,26 @@ __global__ void __launch_bounds__(1024) rotate_kernel(const __grid_constant__ Ro
     At[i] = g < rows ? A[static_cast<int64_t>(r0 + g) * a + ii] : 0.f;
   }
   if (staged) {
-#pragma unroll 4
-    for (int i = tid; i < b * b; i += nt) Bs[i] = B[i];
+    if (async) {
+      for (int i = tid; i < b * b / 4; i += nt) cp_async16(Bs + 4 * i, B + 4 * i);
+      cp_async_commit();
+    } else {
+#pragma unroll 8
+      for (int i = tid; i < b * b; i += nt) Bs[i] = B[i];
+    }
   } else if (async) {
     for (int ch = 0; ch < kRotBufs - 1; ++ch) stage_chunk(ch);
   }
   pdl_wait();
   const __nv_bfloat16* src = in + static_cast<int64_t>(t) * d;
   if (kSynth) {
-#pragma unroll 4
+#pragma unroll 8
     for (int i = tid; i < d; i += nt) V[i] = signs[i] * __bfloat162float(src[i]);
   } else {
-#pragma unroll 4
+#pragma unroll 8
     for (int i = tid; i < d; i += nt) V[perm[i]] = __bfloat162float(src[i]);
   }
+  if (staged && async) cp_async_wait_all();
   __syncthreads();
   float acc[kRotRows];
   // T1 = A[rows] V: this thread's partial over i = kg, kg + KG, ...
@@ -373,13 +386,18 @@ int rot_threads(int b) {
   return rot_slots(b) * std::max(1, std::min(kRotMaxGroups, 1024 / rot_slots(b)));
 }
 
-size_t rot_smem(const fq_frame& f, int KG) {
-  const size_t bb = f.b <= kRotStageB ? static_cast<size_t>(f.b) * f.b
-                                      : static_cast<size_t>(kRotBufs) * kRotChunk * f.b;
+size_t rot_smem_with(const fq_frame& f, int KG, bool staged) {
+  const size_t bb = staged ? static_cast<size_t>(f.b) * f.b
+                           : static_cast<size_t>(kRotBufs) * kRotChunk * f.b;
   return (static_cast<size_t>(round_up(f.d, 4)) + static_cast<size_t>(kRotRows) * (f.a + f.b) +
           static_cast<size_t>(KG) * kRotRows * rot_slots(f.b) + bb) *
          4;
 }
+// all of B in shared memory when it is small and leaves room for two CTAs per SM
+bool rot_staged(const fq_frame& f, int KG) {
+  return f.b <= kRotStageB && rot_smem_with(f, KG, true) <= kRotSmemStaged;
+}
+size_t rot_smem(const fq_frame& f, int KG) { return rot_smem_with(f, KG, rot_staged(f, KG)); }
 
 constexpr size_t kMaxSmem = 227 * 1024;
 
@@ -441,7 +459,8 @@ cudaError_t rotate_batch(int n, const fq_frame* const* f, const void* const* in,
     const fq_frame& F = *f[l];
     const int KG = rot_groups(F.b, threads);
     rb.L[nb] = RotLayer{static_cast<const __nv_bfloat16*>(in[l]), static_cast<__nv_bfloat16*>(out[l]),
-                        F.d, F.a, F.b, rot_slots(F.b), KG, kSynth ? F.Qa : F.QaT,
+                        F.d, F.a, F.b, rot_slots(F.b), KG, rot_staged(F, KG) ? 1 : 0,
+                        kSynth ? F.Qa : F.QaT,
                         kSynth ? F.QbT : F.Qb, F.perm, F.iperm, F.signs};
     gx = std::max(gx, static_cast<int>(ceil_div(F.a, kRotRows)));
     smem = std::max(smem, rot_smem(F, KG));
