@@ -214,3 +214,34 @@ def test_group_refusals():
         fq.fq_linear_forward_implicit_group(8, [one, one], ws, nb)      # one output twice
     assert e.value.status == 1
     assert fq.fq_implicit_group_workspace_bytes(65, [one]) == 0         # decode batches only
+
+
+@pytest.mark.parametrize("d,a,b", [
+    (512, 16, 32),     # B staged whole with asynchronous copies (b <= 128, b % 4 == 0)
+    (160, 16, 10),     # B staged whole with plain loads (b % 4 != 0)
+    (2176, 16, 136),   # B streamed in chunks with asynchronous copies (b > 128)
+    (2080, 16, 130),   # B streamed in chunks with plain loads, a partial last chunk
+])
+def test_rotation_kernel_paths(d, a, b):
+    """Each way the rotation kernel stages its second factor, on square layers whose rotation
+    factor pairs select it, against the structured oracle (seeded uniform codes)."""
+    k = d // RHO + 1
+    n = k * RHO
+    key = ("rotation-paths", str(d), str(a))
+    dr_in = wl.rotation_draws_ab(7, *key, "in", d=d, a=a, b=b)
+    dr_out = wl.rotation_draws_ab(7, *key, "out", d=d, a=a, b=b)
+    codes = wl.random_codes(7, *key, n_out=n, n_in=n)
+    scale, zero = wl.random_scale_zero(7, *key, n_out=n, mag=0.01)
+    M = 17
+    X = torch.from_numpy(wl.rng(7, *key, "x").standard_normal((M, d))).to(BF16).double().numpy()
+    Fi = fq.fq_frame_implicit(k, RHO, d, (a, b, dr_in.ga, dr_in.gb, dr_in.perm, dr_in.signs), DEV)
+    Fo = fq.fq_frame_implicit(k, RHO, d, (a, b, dr_out.ga, dr_out.gb, dr_out.perm, dr_out.signs),
+                              DEV)
+    words = torch.zeros(fq.fq_packed_words(n, n), dtype=torch.int32, device=DEV)
+    C = fq.fq_pack(torch.from_numpy(codes).to(DEV), torch.from_numpy(scale.view(np.int16)).to(DEV),
+                   torch.from_numpy(zero.view(np.int16)).to(DEV), n, n, words)
+    got = _run(X, Fi, C, Fo, None, d)
+    Z = frames.analysis_apply(k, RHO, d, dr_in, X)
+    U = forward.core(Z, codes, scale, zero)
+    ref = frames.synthesis_apply(k, RHO, d, dr_out, U)
+    assert_parity(got, ref, 1e-2)

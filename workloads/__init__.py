@@ -188,6 +188,13 @@ class RotationDraws:
 
 def rotation_draws(seed: int, *key: str, d: int) -> RotationDraws:
     a, b = factor_pair(d)
+    return rotation_draws_ab(seed, *key, d=d, a=a, b=b)
+
+
+def rotation_draws_ab(seed: int, *key: str, d: int, a: int, b: int) -> RotationDraws:
+    """The draws of rotation_draws for a given factor pair a * b = d (the same stream when
+    (a, b) is factor_pair(d))."""
+    assert a * b == d
     g = rng(seed, *key, "rotation", str(d))
     ga = g.standard_normal((a, a))
     gb = g.standard_normal((b, b))
