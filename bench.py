@@ -460,6 +460,7 @@ def cpu_baseline(seconds=12.0):
     per_layer_us = (4 * tq + 3 * tl) / 7 * 1e6
     n = sum(len(v) for v in times.values())
     return {"value": round(per_layer_us, 1), "unit": UNIT, "cores": os.cpu_count(),
+            "tokens_per_s": round(16 / (per_layer_us * 1e-6), 1),
             "cpu": cpu_model(), "kind": "oracle",
             "sample": (f"fp64 numpy oracle forward, M=16, {n} layer calls over "
                        f"{seconds:.0f}+ s: q-shape median {tq * 1e3:.1f} ms, "
