@@ -39,3 +39,21 @@ def synthesis(T_out: np.ndarray, U: np.ndarray) -> np.ndarray:
 def layer_forward(X, T_in, codes, scale, zero, T_out, gamma=None) -> np.ndarray:
     """Y = T_out^T diag(gamma) C_hat T_in X^T, returned token-major (M x d_out)."""
     return synthesis(T_out, core(analysis(T_in, X), codes, scale, zero, gamma))
+
+
+def round_bf16(A) -> np.ndarray:
+    """Values of A (taken to fp32 first) rounded to the nearest bfloat16, ties to even, returned
+    in fp64.  bfloat16 keeps the top 16 bits of an IEEE binary32: the 16 dropped bits decide
+    the rounding, and a carry out of the mantissa moves the exponent (finite inputs)."""
+    bits = np.asarray(A, dtype=np.float32).view(np.uint32).astype(np.uint64)
+    keep_lsb = (bits >> 16) & 1
+    rounded = ((bits + 0x7FFF + keep_lsb) >> 16) << 16
+    return rounded.astype(np.uint32).view(np.float32).astype(np.float64)
+
+
+def layer_forward_bf16_operands(X, T_in, codes, scale, zero, T_out, gamma=None) -> np.ndarray:
+    """Diagnostic: layer_forward with T_in and T_out first rounded to bfloat16 (through fp32,
+    as the bf16 path receives them), the rest of the arithmetic in fp64.  Its distance to
+    layer_forward is the part of a bf16 result's error that the frame operands' precision
+    alone causes."""
+    return layer_forward(X, round_bf16(T_in), codes, scale, zero, round_bf16(T_out), gamma)

@@ -123,3 +123,42 @@ def test_redundancy_lowers_quantization_error():
         Y = forward.layer_forward(X, L.T_in, L.codes, L.scale, L.zero, L.T_out)
         errs.append(np.linalg.norm(Y - ref) / np.linalg.norm(ref))
     assert errs[0] > errs[1] > errs[2]
+
+
+def test_round_bf16_matches_the_format():
+    """The oracle's bfloat16 rounding against torch's conversion (a library routine) on values
+    that exercise ties, carries into the exponent, subnormals and signs."""
+    torch = pytest.importorskip("torch")
+    from oracle.forward import round_bf16
+    vals = np.array([1.0, 1.0 + 2.0 ** -8, 1.0 + 3 * 2.0 ** -8, 1.0 + 2.0 ** -9, -3.14159,
+                     2.0 - 2.0 ** -9, 255.9, 1e-40, -1e-38, 65504.0, 0.0, -0.0], dtype=np.float64)
+    g = np.random.default_rng(3)
+    vals = np.concatenate([vals, g.standard_normal(2000) * 10.0 ** g.integers(-6, 6, 2000)])
+    want = torch.from_numpy(vals.astype(np.float32)).to(torch.bfloat16).double().numpy()
+    got = round_bf16(vals)
+    assert np.array_equal(got.view(np.uint64), want.view(np.uint64))
+    assert round_bf16(np.array([1.0 + 2.0 ** -8]))[0] == 1.0          # a tie goes to even
+    assert round_bf16(np.array([1.0 + 3 * 2.0 ** -8]))[0] == 1.0 + 2.0 ** -6
+
+
+def test_bf16_operand_diagnostic():
+    """The diagnostic forward equals the exact one when the frames are exact in bfloat16 (the
+    trivial frame without rotation is the identity), and otherwise differs by about the
+    operands' rounding (bf16 keeps 8 significant bits)."""
+    from oracle import forward, frames
+    g = np.random.default_rng(11)
+    d, M = 64, 5
+    W = g.standard_normal((d, d)) / 8.0
+    X = g.standard_normal((M, d))
+    T = frames.frame(1, d, d, None)
+    C = T @ W @ T.T
+    codes, scale, zero = quant.rtn(C)
+    exact = forward.layer_forward(X, T, codes, scale, zero, T)
+    diag = forward.layer_forward_bf16_operands(X, T, codes, scale, zero, T)
+    assert np.array_equal(exact, diag)
+    L = layer.from_workload("single256", "single")
+    Xs = g.standard_normal((M, L.d_in))
+    exact = forward.layer_forward(Xs, L.T_in, L.codes, L.scale, L.zero, L.T_out)
+    diag = forward.layer_forward_bf16_operands(Xs, L.T_in, L.codes, L.scale, L.zero, L.T_out)
+    rel = np.linalg.norm(diag - exact) / np.linalg.norm(exact)
+    assert 1e-5 < rel < 1e-2
